@@ -1,0 +1,111 @@
+"""Model shapes and tree-workload recipes for the verify-step workloads.
+
+Five decoder shapes: a tiny fp32 decoder for exhaustive parity checks and four
+random-init bf16 decoders shaped like the targets the paper evaluates
+(Qwen3-0.6B / Qwen3-8B, Llama-3.1-8B and Qwen2.5-32B; experimental setup,
+"Targets, Workloads, and Protocol").  Only shapes live here: no arithmetic of
+the method.
+
+Tree recipes follow the paper's accepted lengths (#MAT between 3.86 and 8.71
+in the main comparison table): one greedy path of `plant` draft nodes is
+planted under the root, the remaining nodes are random draft tokens.
+"""
+
+from dataclasses import dataclass, field, asdict
+
+
+@dataclass(frozen=True)
+class ModelConfig:
+    name: str
+    n_layers: int
+    hidden: int
+    n_q_heads: int
+    n_kv_heads: int
+    head_dim: int
+    intermediate: int
+    vocab: int
+    rms_eps: float
+    rope_theta: float
+    dtype: str            # "f32" or "bf16": storage type of weights and KV
+    qk_norm: bool         # Qwen3: per-head RMSNorm of q and k before RoPE
+    qkv_bias: bool        # Qwen2.5: bias on the q, k, v projections
+    tied: bool            # LM head shares the embedding matrix
+    init_std: float = 0.02
+
+    @property
+    def q_dim(self):
+        return self.n_q_heads * self.head_dim
+
+    @property
+    def kv_dim(self):
+        return self.n_kv_heads * self.head_dim
+
+    def as_dict(self):
+        return asdict(self)
+
+
+@dataclass(frozen=True)
+class Workload:
+    model: ModelConfig
+    ctx_len: int          # committed positions already in the KV cache
+    T: int                # tree nodes, root included
+    plant: int            # draft nodes on the planted greedy path (below the root)
+    tree: dict = field(default_factory=dict)
+    prefill: bool = False  # tiny only: the cache holds a real prefill of ctx_len tokens
+
+    @property
+    def name(self):
+        return self.model.name
+
+
+TINY = ModelConfig("tiny", n_layers=2, hidden=256, n_q_heads=4, n_kv_heads=2,
+                   head_dim=64, intermediate=512, vocab=1024, rms_eps=1e-6,
+                   rope_theta=1e6, dtype="f32", qk_norm=False, qkv_bias=False,
+                   tied=False)
+
+QWEN3_0_6B = ModelConfig("qwen3-0.6b", n_layers=28, hidden=1024, n_q_heads=16,
+                         n_kv_heads=8, head_dim=128, intermediate=3072,
+                         vocab=151936, rms_eps=1e-6, rope_theta=1e6,
+                         dtype="bf16", qk_norm=True, qkv_bias=False, tied=True)
+
+QWEN3_8B = ModelConfig("qwen3-8b", n_layers=36, hidden=4096, n_q_heads=32,
+                       n_kv_heads=8, head_dim=128, intermediate=12288,
+                       vocab=151936, rms_eps=1e-6, rope_theta=1e6,
+                       dtype="bf16", qk_norm=True, qkv_bias=False, tied=False)
+
+LLAMA31_8B = ModelConfig("llama3.1-8b", n_layers=32, hidden=4096, n_q_heads=32,
+                         n_kv_heads=8, head_dim=128, intermediate=14336,
+                         vocab=128256, rms_eps=1e-5, rope_theta=5e5,
+                         dtype="bf16", qk_norm=False, qkv_bias=False, tied=False)
+
+QWEN25_32B = ModelConfig("qwen2.5-32b", n_layers=64, hidden=5120, n_q_heads=40,
+                         n_kv_heads=8, head_dim=128, intermediate=27648,
+                         vocab=152064, rms_eps=1e-6, rope_theta=1e6,
+                         dtype="bf16", qk_norm=False, qkv_bias=True, tied=False)
+
+WORKLOADS = {
+    "tiny": Workload(TINY, ctx_len=128, T=8, plant=3,
+                     tree=dict(kind="uniform", max_depth=4), prefill=True),
+    "qwen3-0.6b": Workload(QWEN3_0_6B, ctx_len=1024, T=32, plant=6,
+                           tree=dict(kind="branch", bmin=1, bmax=4, max_depth=8)),
+    "qwen3-8b": Workload(QWEN3_8B, ctx_len=2048, T=64, plant=10,
+                         tree=dict(kind="branch", bmin=1, bmax=4, max_depth=12)),
+    "llama3.1-8b": Workload(LLAMA31_8B, ctx_len=8192, T=128, plant=12,
+                            tree=dict(kind="wide", level_branch=8, max_depth=16)),
+    "qwen2.5-32b": Workload(QWEN25_32B, ctx_len=4096, T=64, plant=10,
+                            tree=dict(kind="branch", bmin=1, bmax=4, max_depth=12)),
+}
+
+MODELS = {w.model.name: w.model for w in WORKLOADS.values()}
+
+
+def weight_bytes(cfg: ModelConfig) -> dict:
+    """Bytes of every weight tensor class of one model (embedding excluded)."""
+    esz = 4 if cfg.dtype == "f32" else 2
+    H, I = cfg.hidden, cfg.intermediate
+    per_layer = (cfg.q_dim + 2 * cfg.kv_dim) * H + H * cfg.q_dim + 3 * H * I
+    small = 2 * H + (2 * cfg.head_dim if cfg.qk_norm else 0) + \
+        ((cfg.q_dim + 2 * cfg.kv_dim) if cfg.qkv_bias else 0)
+    return dict(layers=cfg.n_layers * (per_layer + small) * esz,
+                lm_head=cfg.vocab * H * esz,
+                final_norm=H * esz)
