@@ -1,0 +1,382 @@
+"""Benchmark of the GB300 tree-verification step.
+
+One step = one pass of the whole hot path on one synthetic batch: the
+target's forward pass over the packed tree (ancestor-masked attention over the
+committed cache), the fused LM-head argmax, the greedy acceptance walk, and
+the KV compaction of the accepted path.  Default workload: the Qwen3-8B-shaped
+bf16 decoder at T = 64 tree nodes over ctx_len = 2048 committed positions.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl ours|reference]
+
+Prints one JSON line.  N > 1 (under torchrun) runs independent replicas, one
+per GPU (the step does not shard); value = tree tokens verified per second
+summed over ranks.  `--impl reference` times the CPU checker (oracle) on the
+host cores instead.
+"""
+
+import argparse
+import dataclasses
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+from synth import gen, trees  # noqa: E402
+from synth.configs import WORKLOADS  # noqa: E402
+from synth.model import TREE_SHAPE, SynthModel, synthetic_kv  # noqa: E402
+
+METRIC = "tree-verify step µs and tree tokens/s at 1 GB300; achieved HBM GB/s vs ~8 TB/s"
+UNIT = "tree tokens/s"
+PLANTED = os.path.join(ROOT, "tests", "golden", "planted.json")
+TRAFFIC = os.path.join(ROOT, "profiles", "traffic.json")
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def workload_tree(name):
+    """Tree of the workload: planted greedy path (from golden/planted.json,
+    written by the CPU checker) plus uniform-random draft tokens."""
+    w = WORKLOADS[name]
+    cfg = w.model
+    with open(PLANTED) as f:
+        p = json.load(f)[name]
+    seed, root = p["seed"], p["root"]
+    tokens, parent, path = trees.make_tree(w.tree, w.T, root, p["planted"], cfg.vocab,
+                                           gen.tensor_key(seed, TREE_SHAPE, w.T))
+    return seed, tokens, parent, path
+
+
+def step_bytes(cfg, ctx, T):
+    """Algorithmic HBM bytes of one step: every weight matrix once (layers and
+    LM head), K/V of ctx committed positions read, T positions written."""
+    es = 2 if cfg.dtype == "bf16" else 4
+    H, I = cfg.hidden, cfg.intermediate
+    per_layer = (cfg.q_dim + 2 * cfg.kv_dim) * H + H * cfg.q_dim + 3 * H * I
+    weights = (cfg.n_layers * per_layer + cfg.vocab * H) * es
+    kv = cfg.n_layers * 2 * (ctx + T) * cfg.kv_dim * es
+    return weights + kv
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons during the timed region."""
+
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, dev):
+        self.proc = None
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(dev), "--query-gpu=" + self.FIELDS,
+                                          "--format=csv,noheader,nounits", "-lms", "200"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except (OSError, ValueError):
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 7:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx.append(float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[3:7]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def traffic_for(kernel_key, src_files):
+    """dram bytes per launch of a kernel from the committed ncu summary, or
+    None when the kernel source changed since the counters were taken."""
+    try:
+        with open(TRAFFIC) as f:
+            d = json.load(f)
+    except (OSError, ValueError):
+        return None
+    e = d.get(kernel_key)
+    if not e:
+        return None
+    h = hashlib.sha256()
+    for p in src_files:
+        with open(os.path.join(ROOT, p), "rb") as f:
+            h.update(f.read())
+    return e["dram_bytes_per_launch"] if e.get("source_sha256") == h.hexdigest() else None
+
+
+def src_hash(src_files):
+    h = hashlib.sha256()
+    for p in src_files:
+        with open(os.path.join(ROOT, p), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()
+
+
+GEMM_SRC = ["paper_2608_00814_gb300/csrc/gemm.cu", "paper_2608_00814_gb300/csrc/common.cuh"]
+
+
+# ---------------------------------------------------------------- CPU checker timing
+
+def oracle_step_estimate(name, n_layers_sample=1, lm_time=None):
+    """Time the CPU checker on a bounded sample of the workload: the full tree
+    through the first n_layers_sample layers plus the LM head, extrapolated to
+    all layers.  Returns (seconds per full step, seconds of CPU work spent, lm_time)."""
+    import oracle
+    w = WORKLOADS[name]
+    cfg = w.model
+    seed, tokens, parent, _ = workload_tree(name)
+    sub = dataclasses.replace(cfg, n_layers=n_layers_sample)
+    view = SynthModel(sub, seed).oracle_view()
+    ck = [synthetic_kv(cfg, seed, l, w.ctx_len, "f64", "k") for l in range(n_layers_sample)]
+    cv = [synthetic_kv(cfg, seed, l, w.ctx_len, "f64", "v") for l in range(n_layers_sample)]
+    t0 = time.perf_counter()
+    r = oracle.verify_tree(view, ck, cv, w.ctx_len, tokens, parent)
+    t_run = time.perf_counter() - t0
+    spent = t_run
+    if lm_time is None:
+        t1 = time.perf_counter()
+        oracle.lm_head_argmax(view, r["final_hidden"])
+        lm_time = time.perf_counter() - t1
+        spent += lm_time
+    per_layer = max(t_run - lm_time, 0.0) / n_layers_sample
+    return per_layer * cfg.n_layers + lm_time, spent, lm_time
+
+
+def cpu_cores():
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count()
+
+
+def run_reference(args):
+    """--impl reference: the CPU checker timed on the host cores (rank 0 only)."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    w = WORKLOADS[args.workload]
+    lm = None
+    for _ in range(args.warmup):
+        _, _, lm = oracle_step_estimate(args.workload, 1, lm)
+    est = []
+    for _ in range(args.steps):
+        s, _, _ = oracle_step_estimate(args.workload, 1, lm)
+        est.append(s)
+    step_s = statistics.mean(est)
+    value = w.T / step_s
+    sample = ("CPU checker (fp64 NumPy) on the %s tree (T=%d, ctx=%d): first layer for every node each step, "
+              "LM head timed once; extrapolated to %d layers" % (args.workload, w.T, w.ctx_len, w.model.n_layers))
+    print(json.dumps({
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_s * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": "%s T=%d ctx_len=%d" % (args.workload, w.T, w.ctx_len), "T": w.T,
+                   "ctx_len": w.ctx_len},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }), flush=True)
+
+
+# ---------------------------------------------------------------- GPU arm
+
+def run_ours(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_00814_gb300 import binding as B
+    from synth.device import upload_cache, upload_model
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        dist.init_process_group("nccl", init_method="env://")
+    torch.cuda.set_device(local)
+    dev = torch.cuda.current_device()
+    w = WORKLOADS[args.workload]
+    cfg = w.model
+    T, ctx = w.T, w.ctx_len
+    seed, tokens_np, parent_np, path = workload_tree(args.workload)
+
+    t0 = time.time()
+    sm = SynthModel(cfg, seed)
+    weights = upload_model(sm)
+    native = [(synthetic_kv(cfg, seed, l, ctx, "native", "k"), synthetic_kv(cfg, seed, l, ctx, "native", "v"))
+              for l in range(cfg.n_layers)]
+    k, v = upload_cache(cfg, native, ctx + T)
+    del native
+    kv = B.KVCache(k, v)
+    model = B.OosModel(cfg, weights, max_T=T, use_graph=True)
+    log("setup %.1fs" % (time.time() - t0))
+
+    stream = torch.cuda.current_stream()
+    tok = torch.as_tensor(tokens_np, dtype=torch.int32, device="cuda")
+    par = torch.as_tensor(parent_np, dtype=torch.int32, device="cuda")
+    outs = B.VerifyOutputs(T)
+
+    def step():
+        B.oos_tree_verify(model, kv, ctx, tok, par, T, outs.accepted_len, outs.accepted_nodes, outs.accepted_tokens,
+                          outs.bonus, stream)
+        B.oos_kv_compact(model, kv, ctx, outs.accepted_nodes, outs.accepted_len, T, stream)
+
+    for _ in range(max(args.warmup, 3)):
+        step()
+    torch.cuda.synchronize()
+    status = B.oos_last_status(model)
+    if status != B.OOS_OK:
+        raise RuntimeError("verify status %s" % B.oos_status_string(status))
+    acc_len = int(outs.accepted_len.item())
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+
+    # ---- device-timed steps (inputs resident in HBM; 15+ GB of weights per step: larger than L2)
+    clocks = ClockSampler(dev)
+    time.sleep(0.3)
+    e0 = torch.cuda.Event(enable_timing=True)
+    e1 = torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    ms = e0.elapsed_time(e1) / args.steps
+    if world > 1:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+        dist.barrier()
+
+    # ---- end to end through the C ABI with host buffers (pinned), copies inside the timed region
+    h_tok = torch.as_tensor(tokens_np, dtype=torch.int32).pin_memory()
+    h_par = torch.as_tensor(parent_np, dtype=torch.int32).pin_memory()
+    h_len = torch.zeros(1, dtype=torch.int32).pin_memory()
+    h_nodes = torch.zeros(T, dtype=torch.int32).pin_memory()
+    h_toks = torch.zeros(T, dtype=torch.int32).pin_memory()
+    h_bonus = torch.zeros(1, dtype=torch.int32).pin_memory()
+    torch.cuda.synchronize()
+    e2e_steps = max(3, args.steps // 2)
+    t_start = time.perf_counter()
+    for _ in range(e2e_steps):
+        tok.copy_(h_tok, non_blocking=True)
+        par.copy_(h_par, non_blocking=True)
+        step()
+        h_len.copy_(outs.accepted_len, non_blocking=True)
+        h_nodes.copy_(outs.accepted_nodes, non_blocking=True)
+        h_toks.copy_(outs.accepted_tokens, non_blocking=True)
+        h_bonus.copy_(outs.bonus, non_blocking=True)
+        stream.synchronize()
+        assert int(h_len.item()) == acc_len
+    e2e_s = (time.perf_counter() - t_start) / e2e_steps
+    h2d = 2 * T * 4
+    d2h = (2 + 2 * T) * 4
+
+    # ---- dominant kernel: the gate/up weight GEMM, timed alone with events over every layer
+    n_rep = 3
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+          for _ in range(cfg.n_layers * n_rep)]
+    for i in range(cfg.n_layers):   # warm
+        B.oos_launch_stage(model, i, B.OOS_STAGE_GATE_UP, T, stream)
+    torch.cuda.synchronize()
+    for r in range(n_rep):
+        for l in range(cfg.n_layers):
+            a, b = ev[r * cfg.n_layers + l]
+            a.record(stream)
+            B.oos_launch_stage(model, l, B.OOS_STAGE_GATE_UP, T, stream)
+            b.record(stream)
+    torch.cuda.synchronize()
+    k_ms = statistics.mean(a.elapsed_time(b) for a, b in ev)
+    N, K = 2 * cfg.intermediate, cfg.hidden
+    k_bytes = 2 * N * K + 2 * T * K + 2 * T * N
+    with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) if os.path.exists(os.path.join(ROOT, "MEASURED_PEAKS.json")) \
+            else open(os.devnull) as f:
+        try:
+            peaks = json.load(f)
+            peak, peak_src = peaks["hbm_gbs"], "measured"
+        except ValueError:
+            peak, peak_src = 6800.0, "fallback"
+    k_gbs = k_bytes / (k_ms * 1e-3) / 1e9
+    traffic = traffic_for("gemm_gate_up_%s_T%d" % (args.workload, T), GEMM_SRC)
+
+    # ---- CPU checker on the host cores (rank 0, N = 1 only)
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        s_est, spent, _ = oracle_step_estimate(args.workload, 2)
+        cpu = {"value": T / s_est, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+               "sample": "fp64 NumPy checker on the same tree: first 2 of %d layers for all %d nodes plus the "
+                         "LM head (%.1f s of CPU work), extrapolated to the full step (%.2f s)"
+                         % (cfg.n_layers, T, spent, s_est)}
+
+    step_b = step_bytes(cfg, ctx, T)
+    value = world * T / (ms * 1e-3)
+    launches_per_step = 2 + cfg.n_layers * 10 + 2 + 1
+    if rank == 0:
+        print(json.dumps({
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16" if cfg.dtype == "bf16" else "f32", "data": "synthetic",
+            "config": {"workload": "%s T=%d ctx_len=%d" % (args.workload, T, ctx), "T": T, "ctx_len": ctx,
+                       "accepted_len": acc_len, "l2": "inputs larger than L2 (weights streamed once per step)",
+                       "parallelism": "replicas" if world > 1 else "single GPU"},
+            "us_per_step": ms * 1e3,
+            "step_gbs": step_b / (ms * 1e-3) / 1e9,
+            "step_frac_of_measured_hbm": step_b / (ms * 1e-3) / 1e9 / peak,
+            "roofline": {"bound": "hbm", "kernel": "gate/up weight GEMM (tcgen05, stream-K)",
+                         "achieved": k_gbs, "peak": peak, "unit": "GB/s", "frac": k_gbs / peak,
+                         "traffic": traffic, "peak_source": peak_src, "bytes_per_launch": k_bytes,
+                         "ms_per_launch": k_ms},
+            "cpu_baseline": cpu,
+            "e2e": {"value": world * T / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+            "gpu_launches": launches_per_step * args.steps,
+            "clocks": clk,
+        }), flush=True)
+    model.close()
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--workload", default="qwen3-8b", choices=sorted(n for n, w in WORKLOADS.items()
+                                                                      if w.model.dtype == "bf16"))
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,228 @@
+/*
+ * oos.h -- C ABI of the GB300 tree-verification step.
+ *
+ * The step is the target verifier of OoO-Spec (arXiv 2608.00814):
+ *   - Eq. 1 ("Target authority"): under greedy decoding the committed token is
+ *     y_t = argmax_v p_T(v | x, y_<t); only the target extends the output.
+ *   - Sec. "Target-Only Verification and Recovery", "Verify and commit": the
+ *     candidate tree is evaluated in ONE forward pass of the target, the
+ *     longest prefix allowed by the greedy rule is committed, the first
+ *     mismatch is replaced by the target's own next token, and only states on
+ *     the accepted path enter the committed KV cache.
+ *   - Sec. "Background" (the ToolSpec loop): each round packs candidates into
+ *     a tree, the target commits the longest approved prefix and the next
+ *     tree is built from all committed tokens.
+ *
+ * Readings of what the paper leaves open (the verifier implements exactly
+ * these):
+ *   - Node 0 of a tree is the ROOT: the last committed token, whose K/V is not
+ *     cached yet.  It is always accepted.  Nodes are numbered parents-first:
+ *     parent[0] == -1 and 0 <= parent[i] < i.
+ *   - Node i attends to the ctx_len committed cache positions and to its own
+ *     ancestors (itself included); its RoPE position is ctx_len + depth(i).
+ *   - A draft node is accepted when its parent is accepted and its token equals
+ *     the target's argmax at the parent.  The committed path is root -> the
+ *     deepest accepted node (lowest node id among equally deep ones).  The
+ *     bonus token is the target's argmax at that node.  Argmax ties go to the
+ *     lowest vocabulary id.
+ *   - The decoder is a pre-norm Llama/Qwen block: RMSNorm, q/k/v projections
+ *     (optional bias), optional per-head q/k RMSNorm before RoPE (Qwen3),
+ *     rotate-half RoPE, grouped-query attention, output projection, RMSNorm,
+ *     SwiGLU MLP (down(silu(gate h) * up h)), final RMSNorm, LM head.
+ *
+ * Conventions for every entry point:
+ *   - Pointers marked DEVICE are CUDA device addresses on the current device;
+ *     HOST pointers are ordinary host memory read during the call only.
+ *   - The caller owns every buffer: weights, KV cache, inputs, outputs and the
+ *     workspace.  The library allocates no device memory; oos_model_create
+ *     allocates the small host-side handle (and a CUDA stream and events used
+ *     for graph capture).
+ *   - Work is enqueued on `stream` (a cudaStream_t passed as void*; NULL is the
+ *     legacy default stream) and runs asynchronously; nothing here blocks the
+ *     host except oos_last_status.
+ *   - Matrices are row-major in the PyTorch nn.Linear layout [out, in];
+ *     element type per oos_model_config.dtype (fp32 or bf16).  Norm gains and
+ *     biases use the same element type.
+ *   - Return value: OOS_OK (0) or a negative OOS_E* code.  Host-side argument
+ *     errors are returned before anything is enqueued.  Errors that only the
+ *     device can see (a malformed tree, an out-of-range token, a pipeline wait
+ *     that ran out of time) are recorded in a device status word of the model
+ *     and reported by oos_last_status; on such an error the verify outputs
+ *     hold accepted_len = 0.
+ */
+#ifndef OOS_H
+#define OOS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ---- status codes ---------------------------------------------------- */
+#define OOS_OK 0
+#define OOS_EINVAL (-1)        /* bad argument: NULL, T outside [1, max_T], ctx_len < 0, shape mismatch */
+#define OOS_ECAPACITY (-2)     /* ctx_len + T exceeds the KV cache capacity */
+#define OOS_ECUDA (-3)         /* a CUDA runtime or driver call failed */
+#define OOS_ETREE (-4)         /* parent[] is not a parents-first tree, or a token is outside [0, vocab) */
+#define OOS_ETIMEOUT (-5)      /* a device pipeline wait exceeded its limit; outputs are not valid */
+#define OOS_EUNSUPPORTED (-6)  /* shape outside what the kernels handle (see oos_model_create) */
+#define OOS_EWORKSPACE (-7)    /* workspace NULL, misaligned (256 B) or smaller than oos_workspace_bytes */
+
+#define OOS_DTYPE_F32 0
+#define OOS_DTYPE_BF16 1
+
+/* Model shape.  Supported: dtype BF16 with head_dim 128, hidden, q_dim and
+ * intermediate multiples of 128 (tcgen05 path); dtype F32 with head_dim <= 128
+ * even (CUDA-core path, meant for small models).  n_q_heads % n_kv_heads == 0,
+ * n_layers <= 128, 1 <= max_T <= 128. */
+typedef struct {
+    int32_t n_layers;
+    int32_t hidden;        /* H */
+    int32_t n_q_heads;     /* nq */
+    int32_t n_kv_heads;    /* nkv */
+    int32_t head_dim;      /* d */
+    int32_t intermediate;  /* I (SwiGLU width) */
+    int32_t vocab;         /* V */
+    int32_t dtype;         /* OOS_DTYPE_F32 or OOS_DTYPE_BF16: weights, KV cache, gains, biases */
+    int32_t qk_norm;       /* nonzero: per-head RMSNorm of q and k before RoPE (Qwen3) */
+    int32_t qkv_bias;      /* nonzero: bias on the q, k, v projections (Qwen2.5) */
+    float rms_eps;
+    float rope_theta;      /* RoPE base; pair (m, m + d/2) turns by pos * theta^(-2m/d) */
+    int32_t max_T;         /* largest tree this handle verifies, 1..128 */
+    int32_t use_graph;     /* nonzero: replay a captured CUDA graph when the call's shape repeats */
+} oos_model_config;
+
+/* Per-layer weights, all DEVICE pointers. */
+typedef struct {
+    const void* attn_norm;  /* [H] */
+    const void* w_q;        /* [nq*d, H] */
+    const void* w_k;        /* [nkv*d, H] */
+    const void* w_v;        /* [nkv*d, H] */
+    const void* b_q;        /* [nq*d]  or NULL (required iff qkv_bias) */
+    const void* b_k;        /* [nkv*d] or NULL */
+    const void* b_v;        /* [nkv*d] or NULL */
+    const void* q_norm;     /* [d] or NULL (required iff qk_norm) */
+    const void* k_norm;     /* [d] or NULL */
+    const void* w_o;        /* [H, nq*d] */
+    const void* mlp_norm;   /* [H] */
+    const void* w_gate;     /* [I, H] */
+    const void* w_up;       /* [I, H] */
+    const void* w_down;     /* [H, I] */
+} oos_layer_weights;
+
+typedef struct {
+    const void* embed;               /* DEVICE [V, H] */
+    const void* final_norm;          /* DEVICE [H] */
+    const void* lm_head;             /* DEVICE [V, H]; may equal embed (tied embeddings) */
+    const oos_layer_weights* layers; /* HOST array of n_layers entries, copied by oos_model_create */
+} oos_weights;
+
+/* Committed KV cache: per layer one K and one V buffer of `capacity` slots.
+ * Slot p holds the post-RoPE K (resp. V) of committed position p for all
+ * kv heads: layout [capacity][nkv][d], element type = model dtype.  During
+ * oos_tree_verify the tree's K/V are written to slots ctx_len .. ctx_len+T-1;
+ * oos_kv_compact then moves the accepted path to ctx_len .. ctx_len+len-1. */
+typedef struct {
+    int32_t n_layers;
+    int32_t capacity;
+    void* const* k;   /* HOST array of n_layers DEVICE pointers */
+    void* const* v;   /* HOST array of n_layers DEVICE pointers */
+} oos_kv_cache;
+
+typedef struct oos_model oos_model;
+
+/* Bytes of DEVICE workspace one model handle needs (depends on the shape,
+ * max_T and the current device's SM count).  Returns 0 on a bad config. */
+size_t oos_workspace_bytes(const oos_model_config* cfg);
+
+/* Validate the shape, copy the weight pointers, carve the caller's workspace
+ * (DEVICE, >= oos_workspace_bytes, 256-byte aligned; owned by the caller and
+ * bound to the handle until oos_model_destroy) and encode the TMA descriptors
+ * of every weight matrix.  Weights must stay valid while the handle lives.
+ * Uses the current CUDA device. */
+int oos_model_create(const oos_model_config* cfg, const oos_weights* w, void* workspace,
+                     size_t ws_bytes, oos_model** out);
+
+int oos_model_destroy(oos_model* m);
+
+/* One verification step (Eq. 1; "Verify and commit").
+ *   kv            committed cache; slots [0, ctx_len) are read, slots
+ *                 [ctx_len, ctx_len+T) are overwritten with the tree's K/V.
+ *   ctx_len       committed positions already in the cache (>= 0).
+ *   tree_tokens   DEVICE int32[T]: token of each node, node 0 = root.
+ *   tree_parent   DEVICE int32[T]: parent of each node, parent[0] = -1.
+ *   T             nodes, 1..max_T.
+ * Outputs (DEVICE):
+ *   out_accepted_len     int32[1]: nodes on the committed path, root included
+ *                        (>= 1; the per-call "accepted tokens" of the paper's
+ *                        #MAT metric), 0 on a device-detected error.
+ *   out_accepted_nodes   int32[T]: node ids root-first; entries past len are -1.
+ *   out_accepted_tokens  int32[T]: their tokens; entries past len are -1.
+ *   out_bonus_token      int32[1]: the target's next token after the path.
+ * The tree's K/V stay in slots ctx_len.. until oos_kv_compact. */
+int oos_tree_verify(oos_model* m, const oos_kv_cache* kv, int32_t ctx_len,
+                    const int32_t* tree_tokens, const int32_t* tree_parent, int32_t T,
+                    int32_t* out_accepted_len, int32_t* out_accepted_nodes,
+                    int32_t* out_accepted_tokens, int32_t* out_bonus_token, void* stream);
+
+/* oos_tree_verify plus intermediate results for checking (DEVICE outputs):
+ *   out_final_hidden  float[T, H]: output of the final RMSNorm per node (fp32)
+ *   out_argmax        int32[T]:  the target's greedy token at every node
+ *   out_top1/out_top2 float[T]:  largest and second-largest logit per node
+ * Any of the four may be NULL. */
+int oos_tree_verify_debug(oos_model* m, const oos_kv_cache* kv, int32_t ctx_len,
+                          const int32_t* tree_tokens, const int32_t* tree_parent, int32_t T,
+                          int32_t* out_accepted_len, int32_t* out_accepted_nodes,
+                          int32_t* out_accepted_tokens, int32_t* out_bonus_token,
+                          float* out_final_hidden, int32_t* out_argmax, float* out_top1,
+                          float* out_top2, void* stream);
+
+/* Commit the accepted path's K/V ("only states on the accepted target path
+ * enter the committed KV cache").  For every layer and for K and V:
+ * slot ctx_len + j <- slot ctx_len + accepted_nodes[j], j < *accepted_len, read
+ * as a gather from the cache as it was before the call (sources never get
+ * overwritten before they are read).  accepted_nodes / accepted_len are the
+ * DEVICE outputs of oos_tree_verify (no host round trip); max_len is an upper
+ * bound on *accepted_len (the T of that call).  The new committed length is
+ * ctx_len + *accepted_len. */
+int oos_kv_compact(oos_model* m, const oos_kv_cache* kv, int32_t ctx_len,
+                   const int32_t* accepted_nodes, const int32_t* accepted_len, int32_t max_len,
+                   void* stream);
+
+/* Standalone greedy-acceptance walk over given argmax values (DEVICE in/out):
+ * the same rule oos_tree_verify applies after its LM head.  Also validates the
+ * tree; on a malformed tree *out_accepted_len = 0 and the call still returns
+ * OOS_OK (the status is in *out_status: OOS_OK or OOS_ETREE). */
+int oos_accept_walk(const int32_t* tree_tokens, const int32_t* tree_parent, const int32_t* argmax,
+                    int32_t T, int32_t* out_accepted_len, int32_t* out_accepted_nodes,
+                    int32_t* out_accepted_tokens, int32_t* out_bonus_token, int32_t* out_status,
+                    void* stream);
+
+/* Benchmarking aid: enqueue ONE weight-streaming kernel of the verify step,
+ * launched exactly as oos_tree_verify launches it, on the activations the last
+ * verify of this handle left in its workspace.  stage: OOS_STAGE_QKV,
+ * OOS_STAGE_O, OOS_STAGE_GATE_UP, OOS_STAGE_DOWN (of layer `layer`) or
+ * OOS_STAGE_LM_HEAD (layer ignored).  T as in that verify.  Writes only
+ * workspace scratch (partial sums, LM-head partial maxima); the KV cache and
+ * the outputs of the last verify are left as they were. */
+#define OOS_STAGE_QKV 0
+#define OOS_STAGE_O 1
+#define OOS_STAGE_GATE_UP 2
+#define OOS_STAGE_DOWN 3
+#define OOS_STAGE_LM_HEAD 4
+int oos_launch_stage(oos_model* m, int32_t layer, int32_t stage, int32_t T, void* stream);
+
+/* Synchronise `stream` and return the device status of the last verify on
+ * this handle: OOS_OK, OOS_ETREE or OOS_ETIMEOUT (or OOS_ECUDA). */
+int oos_last_status(oos_model* m, void* stream);
+
+/* Static description of a status code. */
+const char* oos_status_string(int code);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* OOS_H */

@@ -1,0 +1,384 @@
+// Tree attention of the verify step.
+//
+// Node i, query head h (kv head g = h / (nq/nkv)) attends to the committed
+// cache positions [0, ctx) and to the tree slots ctx + a for every ancestor a
+// of i (itself included): softmax(q k / sqrt(d)) v.
+//
+// bf16 path: split-K over the cache (flash-decoding).  A block owns 64 query
+// rows of one kv head -- the (node, q-head) pairs of the group, so GQA reuses
+// every K/V tile for nq/nkv heads -- and one range of cache keys; the last
+// split also takes the tree tail, masked with the 128-bit ancestor sets.  K/V
+// tiles are staged in shared memory by cp.async (double buffered); scores and
+// P.V run on the tensor cores (mma.sync m16n8k16, fp32 accumulate) with an
+// online softmax in fp32.  Splits are merged by log-sum-exp in a second kernel.
+//
+// fp32 path: one block per (node, head), CUDA cores (small models only).
+#include <math.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace oos {
+
+constexpr int kAttnRows = 64;     // query rows per block (4 warps x 16)
+constexpr int kAttnKeys = 64;     // keys per tile
+constexpr int kAttnD = 128;       // head dim of the bf16 path
+constexpr int kAttnLd = kAttnD + 8;   // padded smem row (272 bytes): conflict-free ldmatrix
+constexpr int kAttnSmem = (kAttnRows + 4 * kAttnKeys) * kAttnLd * 2;
+
+struct AttnArgs {
+  const __nv_bfloat16* q;   // [T][nq][d]
+  const __nv_bfloat16* kc;  // [cap][nkv][d]
+  const __nv_bfloat16* vc;
+  const unsigned long long* anc;
+  int T, nq, nkv, group, ctx;
+  int splits, cache_blocks;
+  float scale_log2;         // log2(e) / sqrt(d)
+  float* o_part;            // [split][T*nq][d]
+  float* ml_part;           // [split][T*nq][2]
+};
+
+OOS_DEV void cp_async16(void* smem, const void* gmem, bool valid) {
+  const int n = valid ? 16 : 0;
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_addr(smem)), "l"(gmem), "r"(n) : "memory");
+}
+OOS_DEV void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+OOS_DEV void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
+
+OOS_DEV void ldsm_x4(uint32_t (&r)[4], const void* p) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(smem_addr(p)));
+}
+OOS_DEV void ldsm_x4_t(uint32_t (&r)[4], const void* p) {
+  asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
+               : "r"(smem_addr(p)));
+}
+OOS_DEV void mma_bf16(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+OOS_DEV uint32_t pack_bf16(float lo, float hi) {
+  __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+  return *reinterpret_cast<uint32_t*>(&v);
+}
+
+// stage 64 keys (cache positions or tree slots) of kv head g into smem
+OOS_DEV void load_kv_tile(__nv_bfloat16* ks, __nv_bfloat16* vs, const AttnArgs& a, int g, int key0, int key_end) {
+  for (int c = threadIdx.x; c < kAttnKeys * (kAttnD / 8); c += blockDim.x) {
+    const int r = c >> 4, col = (c & 15) * 8;
+    const int key = key0 + r;
+    const bool valid = key < key_end;
+    const size_t off = ((size_t)(valid ? key : key0) * a.nkv + g) * kAttnD + col;
+    cp_async16(ks + r * kAttnLd + col, a.kc + off, valid);
+    cp_async16(vs + r * kAttnLd + col, a.vc + off, valid);
+  }
+}
+
+__global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  __nv_bfloat16* Qs = reinterpret_cast<__nv_bfloat16*>(smem_raw);
+  __nv_bfloat16* Ks = Qs + kAttnRows * kAttnLd;          // [2][64][ld]
+  __nv_bfloat16* Vs = Ks + 2 * kAttnKeys * kAttnLd;      // [2][64][ld]
+  pdl_trigger();
+  pdl_wait();
+  const int rb = blockIdx.x, g = blockIdx.y, split = blockIdx.z;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int R = a.T * a.group;
+
+  // key tiles of this block: cache blocks [cb0, cb1), then (last split) the tree tail
+  const int cb0 = (int)((long long)split * a.cache_blocks / a.splits);
+  const int cb1 = (int)((long long)(split + 1) * a.cache_blocks / a.splits);
+  const int tree_tiles = (split == a.splits - 1) ? (a.T + kAttnKeys - 1) / kAttnKeys : 0;
+  const int n_tiles = (cb1 - cb0) + tree_tiles;
+
+  // Q rows: row r -> node r / group, head g*group + r % group
+  for (int c = threadIdx.x; c < kAttnRows * (kAttnD / 8); c += blockDim.x) {
+    const int r = c >> 4, col = (c & 15) * 8;
+    const int row = rb * kAttnRows + r;
+    const bool valid = row < R;
+    const int node = valid ? row / a.group : 0, hq = g * a.group + (valid ? row % a.group : 0);
+    cp_async16(Qs + r * kAttnLd + col, a.q + ((size_t)node * a.nq + hq) * kAttnD + col, valid);
+  }
+  auto tile_keys = [&](int ti, int& key0, int& key_end, bool& tree) {
+    if (ti < cb1 - cb0) {
+      key0 = (cb0 + ti) * kAttnKeys;
+      key_end = min(a.ctx, key0 + kAttnKeys);
+      tree = false;
+    } else {
+      const int tt = ti - (cb1 - cb0);
+      key0 = a.ctx + tt * kAttnKeys;
+      key_end = a.ctx + a.T;
+      tree = true;
+    }
+  };
+  if (n_tiles > 0) {
+    int k0, ke;
+    bool tr;
+    tile_keys(0, k0, ke, tr);
+    load_kv_tile(Ks, Vs, a, g, k0, ke);
+  }
+  cp_async_commit();
+
+  // per-thread rows: r_lo = warp*16 + lane/4, r_hi = r_lo + 8
+  const int r_lo = rb * kAttnRows + warp * 16 + (lane >> 2);
+  const int r_hi = r_lo + 8;
+  const int node_lo = min(r_lo, R - 1) / a.group, node_hi = min(r_hi, R - 1) / a.group;
+  const unsigned long long anc_lo0 = a.anc[2 * node_lo], anc_lo1 = a.anc[2 * node_lo + 1];
+  const unsigned long long anc_hi0 = a.anc[2 * node_hi], anc_hi1 = a.anc[2 * node_hi + 1];
+
+  float o[16][4];
+#pragma unroll
+  for (int n = 0; n < 16; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
+  float m_lo = -INFINITY, m_hi = -INFINITY, l_lo = 0.f, l_hi = 0.f;
+  uint32_t qf[8][4];
+
+  for (int ti = 0; ti < n_tiles; ++ti) {
+    const int buf = ti & 1;
+    if (ti + 1 < n_tiles) {
+      int k0, ke;
+      bool tr;
+      tile_keys(ti + 1, k0, ke, tr);
+      load_kv_tile(Ks + (buf ^ 1) * kAttnKeys * kAttnLd, Vs + (buf ^ 1) * kAttnKeys * kAttnLd, a, g, k0, ke);
+    }
+    cp_async_commit();
+    cp_async_wait<1>();
+    __syncthreads();
+    if (ti == 0) {
+#pragma unroll
+      for (int ks = 0; ks < 8; ++ks) {
+        const int row = warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+        const int col = ks * 16 + (lane >> 4) * 8;
+        ldsm_x4(qf[ks], Qs + row * kAttnLd + col);
+      }
+    }
+    const __nv_bfloat16* kt = Ks + buf * kAttnKeys * kAttnLd;
+    const __nv_bfloat16* vt = Vs + buf * kAttnKeys * kAttnLd;
+    int key0, key_end;
+    bool tree;
+    tile_keys(ti, key0, key_end, tree);
+
+    // S = Q K^T  (16 rows x 64 keys per warp)
+    float s[8][4];
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+      s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+#pragma unroll
+      for (int ks = 0; ks < 8; ks += 2) {
+        uint32_t b[4];
+        ldsm_x4(b, kt + (nt * 8 + (lane & 7)) * kAttnLd + ks * 16 + (lane >> 3) * 8);
+        mma_bf16(s[nt], qf[ks], b[0], b[1]);
+        mma_bf16(s[nt], qf[ks + 1], b[2], b[3]);
+      }
+    }
+    // mask + scale, tile row maxima
+    float tmax_lo = -INFINITY, tmax_hi = -INFINITY;
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        const int key = key0 + nt * 8 + (lane & 3) * 2 + (e & 1);
+        bool valid = key < key_end;
+        if (tree && valid) {
+          const int j = key - a.ctx;
+          const unsigned long long w0 = (e < 2) ? anc_lo0 : anc_hi0;
+          const unsigned long long w1 = (e < 2) ? anc_lo1 : anc_hi1;
+          valid = ((j < 64 ? (w0 >> j) : (w1 >> (j - 64))) & 1ull) != 0;
+        }
+        const float v = valid ? s[nt][e] * a.scale_log2 : -INFINITY;
+        s[nt][e] = v;
+        if (e < 2) tmax_lo = fmaxf(tmax_lo, v); else tmax_hi = fmaxf(tmax_hi, v);
+      }
+    }
+#pragma unroll
+    for (int off = 1; off <= 2; off <<= 1) {
+      tmax_lo = fmaxf(tmax_lo, __shfl_xor_sync(0xffffffffu, tmax_lo, off));
+      tmax_hi = fmaxf(tmax_hi, __shfl_xor_sync(0xffffffffu, tmax_hi, off));
+    }
+    const float mn_lo = fmaxf(m_lo, tmax_lo), mn_hi = fmaxf(m_hi, tmax_hi);
+    const float base_lo = mn_lo == -INFINITY ? 0.f : mn_lo;
+    const float base_hi = mn_hi == -INFINITY ? 0.f : mn_hi;
+    const float corr_lo = exp2f(m_lo - base_lo), corr_hi = exp2f(m_hi - base_hi);
+    m_lo = mn_lo;
+    m_hi = mn_hi;
+    float sum_lo = 0.f, sum_hi = 0.f;
+#pragma unroll
+    for (int nt = 0; nt < 8; ++nt) {
+      s[nt][0] = exp2f(s[nt][0] - base_lo);
+      s[nt][1] = exp2f(s[nt][1] - base_lo);
+      s[nt][2] = exp2f(s[nt][2] - base_hi);
+      s[nt][3] = exp2f(s[nt][3] - base_hi);
+      sum_lo += s[nt][0] + s[nt][1];
+      sum_hi += s[nt][2] + s[nt][3];
+    }
+    l_lo = l_lo * corr_lo + sum_lo;
+    l_hi = l_hi * corr_hi + sum_hi;
+#pragma unroll
+    for (int n = 0; n < 16; ++n) {
+      o[n][0] *= corr_lo;
+      o[n][1] *= corr_lo;
+      o[n][2] *= corr_hi;
+      o[n][3] *= corr_hi;
+    }
+    // O += P V
+#pragma unroll
+    for (int kk = 0; kk < 4; ++kk) {
+      uint32_t pa[4];
+      pa[0] = pack_bf16(s[2 * kk][0], s[2 * kk][1]);
+      pa[1] = pack_bf16(s[2 * kk][2], s[2 * kk][3]);
+      pa[2] = pack_bf16(s[2 * kk + 1][0], s[2 * kk + 1][1]);
+      pa[3] = pack_bf16(s[2 * kk + 1][2], s[2 * kk + 1][3]);
+#pragma unroll
+      for (int n2 = 0; n2 < 16; n2 += 2) {
+        uint32_t b[4];
+        const int mi = lane >> 3;
+        ldsm_x4_t(b, vt + (kk * 16 + (mi & 1) * 8 + (lane & 7)) * kAttnLd + (n2 + (mi >> 1)) * 8);
+        mma_bf16(o[n2], pa, b[0], b[1]);
+        mma_bf16(o[n2 + 1], pa, b[2], b[3]);
+      }
+    }
+    __syncthreads();
+  }
+  cp_async_wait<0>();
+
+  // quad sums of l, then write unnormalised O and (m, l)
+#pragma unroll
+  for (int off = 1; off <= 2; off <<= 1) {
+    l_lo += __shfl_xor_sync(0xffffffffu, l_lo, off);
+    l_hi += __shfl_xor_sync(0xffffffffu, l_hi, off);
+  }
+  const size_t rows_total = (size_t)a.T * a.nq;
+#pragma unroll
+  for (int half = 0; half < 2; ++half) {
+    const int r = half ? r_hi : r_lo;
+    if (r >= R) continue;
+    const int node = r / a.group, hq = g * a.group + r % a.group;
+    const size_t grow = (size_t)node * a.nq + hq;
+    float* dst = a.o_part + ((size_t)split * rows_total + grow) * kAttnD;
+#pragma unroll
+    for (int n = 0; n < 16; ++n) {
+      const int col = n * 8 + (lane & 3) * 2;
+      *reinterpret_cast<float2*>(dst + col) = half ? make_float2(o[n][2], o[n][3]) : make_float2(o[n][0], o[n][1]);
+    }
+    if ((lane & 3) == 0) {
+      float* ml = a.ml_part + ((size_t)split * rows_total + grow) * 2;
+      ml[0] = half ? m_hi : m_lo;
+      ml[1] = half ? l_hi : l_lo;
+    }
+  }
+}
+
+// merge the splits of one (node, head) row: log-sum-exp weights in base 2
+__global__ void __launch_bounds__(kAttnD) k_attn_merge(const float* __restrict__ o_part, const float* __restrict__ ml,
+                                                       int splits, int rows_total, __nv_bfloat16* __restrict__ out) {
+  pdl_trigger();
+  pdl_wait();
+  const int row = blockIdx.x, c = threadIdx.x;
+  float M = -INFINITY;
+  for (int s = 0; s < splits; ++s) M = fmaxf(M, ml[((size_t)s * rows_total + row) * 2]);
+  float num = 0.f, den = 0.f;
+  for (int s = 0; s < splits; ++s) {
+    const float ms = ml[((size_t)s * rows_total + row) * 2];
+    if (ms == -INFINITY) continue;
+    const float w = exp2f(ms - M);
+    den += w * ml[((size_t)s * rows_total + row) * 2 + 1];
+    num += w * o_part[((size_t)s * rows_total + row) * kAttnD + c];
+  }
+  out[(size_t)row * kAttnD + c] = __float2bfloat16_rn(num / den);
+}
+
+// ------------------------------------------------------------ fp32 path
+__global__ void __launch_bounds__(128) k_attn_f32(const float* __restrict__ q, const float* __restrict__ kc,
+                                                  const float* __restrict__ vc, const unsigned long long* __restrict__ anc,
+                                                  int T, int nq, int nkv, int d, int ctx, float scale,
+                                                  float* __restrict__ out) {
+  __shared__ float qs[128];
+  __shared__ float ps[128];
+  __shared__ int kpos[128];
+  __shared__ float red[32];
+  pdl_trigger();
+  pdl_wait();
+  const int i = blockIdx.x, h = blockIdx.y, g = h / (nq / nkv), tid = threadIdx.x;
+  if (tid < d) qs[tid] = q[((size_t)i * nq + h) * d + tid];
+  const unsigned long long w0 = anc[2 * i], w1 = anc[2 * i + 1];
+  __syncthreads();
+  float m = -INFINITY, l = 0.f, acc = 0.f;
+  const int n_keys = ctx + T;
+  for (int base = 0; base < n_keys; base += blockDim.x) {
+    const int kk = base + tid;
+    bool valid = kk < n_keys;
+    if (valid && kk >= ctx) {
+      const int j = kk - ctx;
+      valid = ((j < 64 ? (w0 >> j) : (w1 >> (j - 64))) & 1ull) != 0;
+    }
+    float sc = -INFINITY;
+    if (valid) {
+      const float* kr = kc + ((size_t)kk * nkv + g) * d;
+      float dot = 0.f;
+      for (int c = 0; c < d; ++c) dot += qs[c] * kr[c];
+      sc = dot * scale;
+    }
+    const float cmax = block_max(sc, red);
+    const float mn = fmaxf(m, cmax);
+    const float p = valid ? expf(sc - mn) : 0.f;
+    const float corr = (m == -INFINITY) ? 0.f : expf(m - mn);
+    const float psum = block_sum(p, red);
+    l = l * corr + psum;
+    ps[tid] = p;
+    kpos[tid] = kk;
+    __syncthreads();
+    if (tid < d) {
+      acc *= corr;
+      const int nk = min((int)blockDim.x, n_keys - base);
+      for (int k = 0; k < nk; ++k)
+        if (ps[k] != 0.f) acc += ps[k] * vc[((size_t)kpos[k] * nkv + g) * d + tid];
+    }
+    m = mn;
+    __syncthreads();
+  }
+  if (tid < d) out[(size_t)i * nq * d + (size_t)h * d + tid] = acc / l;
+}
+
+cudaError_t attn_setup() {
+  return cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmem);
+}
+
+cudaError_t launch_attention(Model& m, const void* kc, const void* vc, int ctx, int T, cudaStream_t st) {
+  const auto& c = m.cfg;
+  if (c.dtype != OOS_DTYPE_BF16) {
+    return launch(m.pdl, k_attn_f32, dim3(T, c.n_q_heads), dim3(128), 0, st, (const float*)m.ws.q, (const float*)kc,
+                  (const float*)vc, (const unsigned long long*)m.ws.anc, T, c.n_q_heads, c.n_kv_heads, c.head_dim, ctx,
+                  1.0f / sqrtf((float)c.head_dim), (float*)m.ws.attn);
+  }
+  AttnArgs a;
+  a.q = (const __nv_bfloat16*)m.ws.q;
+  a.kc = (const __nv_bfloat16*)kc;
+  a.vc = (const __nv_bfloat16*)vc;
+  a.anc = m.ws.anc;
+  a.T = T;
+  a.nq = c.n_q_heads;
+  a.nkv = c.n_kv_heads;
+  a.group = c.n_q_heads / c.n_kv_heads;
+  a.ctx = ctx;
+  a.cache_blocks = (ctx + kAttnKeys - 1) / kAttnKeys;
+  const int R = T * a.group;
+  const int RB = (R + kAttnRows - 1) / kAttnRows;
+  int splits = (2 * m.num_sms + a.nkv * RB - 1) / (a.nkv * RB);
+  const int max_splits = a.cache_blocks > 0 ? (a.cache_blocks < kMaxAttnSplits ? a.cache_blocks : kMaxAttnSplits) : 1;
+  splits = splits < 1 ? 1 : (splits > max_splits ? max_splits : splits);
+  a.splits = splits;
+  a.scale_log2 = 1.4426950408889634f / sqrtf((float)kAttnD);
+  a.o_part = m.ws.attn_o;
+  a.ml_part = m.ws.attn_ml;
+  cudaError_t e = launch(m.pdl, k_attn_tc, dim3(RB, a.nkv, splits), dim3(128), (size_t)kAttnSmem, st, a);
+  if (e != cudaSuccess) return e;
+  return launch(m.pdl, k_attn_merge, dim3(T * c.n_q_heads), dim3(kAttnD), 0, st, (const float*)m.ws.attn_o,
+                (const float*)m.ws.attn_ml, splits, T * c.n_q_heads, (__nv_bfloat16*)m.ws.attn);
+}
+
+}  // namespace oos

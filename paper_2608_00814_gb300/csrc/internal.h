@@ -1,0 +1,177 @@
+// Host-side model handle, workspace carve-out and kernel launchers.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <utility>
+#include <vector>
+
+#include "oos.h"
+
+namespace oos {
+
+constexpr int kMaxT = 128;          // largest tree (ancestor sets are 128-bit masks)
+constexpr int kTile = 128;          // output features per GEMM tile (tcgen05 M)
+constexpr int kBK = 64;             // reduction elements per pipeline stage (128 bytes of bf16)
+constexpr int kMaxLayers = 128;
+constexpr int kMaxAttnSplits = 16;  // cache splits of the attention kernel
+constexpr int kMaxGridCTAs = 1024;  // upper bound on CTAs of a stream-K GEMM / LM head
+
+// Stream-K partition of a weight GEMM: the (tile, k-block) units of all tiles,
+// tile-major, are cut into `grid` contiguous equal ranges, one per CTA.  CTA c
+// owns units [c*total/grid, (c+1)*total/grid).  Each CTA writes one fp32
+// partial tile per tile it touches, into slice (c - first contributor of the
+// tile); a reduce kernel adds the slices in slice order (deterministic).
+struct StreamK {
+  int n_tiles;
+  int kbt;     // k-blocks per tile
+  int total;   // n_tiles * kbt
+  int grid;    // CTAs
+  __host__ __device__ int cta_of_unit(long long u) const {
+    // largest c with floor(c*total/grid) <= u
+    return (int)(((u + 1) * (long long)grid + total - 1) / total) - 1;
+  }
+  __host__ __device__ void contributors(int tile, int& c0, int& c1) const {
+    c0 = cta_of_unit((long long)tile * kbt);
+    c1 = cta_of_unit((long long)tile * kbt + kbt - 1);
+  }
+  int max_slices() const {
+    int m = 1;
+    for (int t = 0; t < n_tiles; ++t) {
+      int a, b;
+      contributors(t, a, b);
+      m = (b - a + 1) > m ? (b - a + 1) : m;
+    }
+    return m;
+  }
+};
+
+StreamK make_streamk(int n_rows, int K, int n_sms);
+StreamK make_single_slice(int n_rows);   // one contributor per tile (CUDA-core GEMM)
+
+// One weight GEMM of the bf16 path: up to three row-stacked segments (q|k|v,
+// gate|up), each with its own TMA descriptor.
+struct GemmW {
+  CUtensorMap map[3];
+  const void* ptr[3];
+  int seg_tiles[3];   // cumulative tile counts at the end of each segment
+  int n_seg;
+  int N, K;
+  StreamK plan;
+};
+
+struct Workspace {
+  uint32_t* status;
+  int32_t* depth;
+  int32_t* pos;
+  unsigned long long* anc;   // [kMaxT][2]
+  float* x;                  // residual stream, fp32 [kMaxT][H]
+  void* xn;                  // normalised GEMM input [kMaxT][H] (model dtype)
+  void* q;                   // [kMaxT][nq][d]
+  void* attn;                // attention output [kMaxT][nq*d]
+  void* act;                 // SwiGLU activation [kMaxT][I]
+  float* part;               // GEMM partial slices
+  size_t part_floats;
+  float* attn_o;             // [kMaxAttnSplits][kMaxT*nq][d]
+  float* attn_ml;            // [kMaxAttnSplits][kMaxT*nq][2]
+  float* lm_v1;              // LM-head partial states [kMaxGridCTAs][kMaxT]
+  int32_t* lm_i;
+  float* lm_v2;
+  double* inv_freq;          // RoPE frequencies theta^(-2j/d), j < d/2
+  int32_t* argmax;           // [kMaxT]
+  float* top1;
+  float* top2;
+};
+
+// shape + addresses a captured verify graph was recorded with
+struct GraphKey {
+  unsigned long long kv_hash;   // FNV-1a over every layer's K and V pointer
+  int capacity, ctx_len, T;
+  const void* io[10];
+  bool operator==(const GraphKey& o) const {
+    if (kv_hash != o.kv_hash || capacity != o.capacity || ctx_len != o.ctx_len || T != o.T) return false;
+    for (int i = 0; i < 10; ++i)
+      if (io[i] != o.io[i]) return false;
+    return true;
+  }
+};
+
+struct Model {
+  oos_model_config cfg;
+  std::vector<oos_layer_weights> layers;
+  oos_weights w;
+  int num_sms;
+  int esize;            // bytes per weight / activation element
+  Workspace ws;
+  size_t ws_bytes;
+  bool pdl = true;
+  // bf16 tensor-core path
+  std::vector<GemmW> g_qkv, g_o, g_gu, g_down;
+  GemmW g_lm;
+  CUtensorMap amap_xn[4], amap_attn[4], amap_act[4];  // per N-tile variant 16/32/64/128
+  int lm_grid;
+  // fp32 path plans (one slice)
+  StreamK p_qkv, p_o, p_gu, p_down;
+  // CUDA graph of the last call shape
+  cudaStream_t cap_stream = nullptr;
+  cudaGraphExec_t gexec = nullptr;
+  GraphKey gkey{};
+  bool have_graph = false;
+};
+
+size_t carve_workspace(const oos_model_config& c, int n_sms, uint8_t* base, Workspace* ws);
+
+// launch with or without programmatic dependent launch (PDL)
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch(bool pdl, void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                          cudaStream_t st, Args&&... args) {
+  cudaLaunchConfig_t lc = {};
+  lc.gridDim = grid;
+  lc.blockDim = block;
+  lc.dynamicSmemBytes = smem;
+  lc.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  lc.attrs = attr;
+  lc.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&lc, kernel, std::forward<Args>(args)...);
+}
+
+// ---- small kernels (small.cu)
+cudaError_t launch_tree_prep(Model& m, const int32_t* tokens, const int32_t* parent, int T, int ctx,
+                             cudaStream_t st);
+cudaError_t launch_embed_norm(Model& m, const int32_t* tokens, int T, cudaStream_t st);
+cudaError_t launch_qkv_post(Model& m, int layer, const StreamK& plan, void* kc, void* vc, int ctx, int T,
+                            cudaStream_t st);
+cudaError_t launch_resid_norm(Model& m, const StreamK& plan, const void* gain, float* hidden_out, int T,
+                              cudaStream_t st);
+cudaError_t launch_silu_mul(Model& m, const StreamK& plan, int T, cudaStream_t st);
+cudaError_t launch_argmax_accept(Model& m, const int32_t* tokens, const int32_t* parent, int T, int n_parts,
+                                 int32_t* len, int32_t* nodes, int32_t* toks, int32_t* bonus,
+                                 int32_t* dbg_argmax, float* dbg_top1, float* dbg_top2, cudaStream_t st);
+cudaError_t launch_kv_compact(Model& m, const oos_kv_cache& kv, int ctx, const int32_t* nodes,
+                              const int32_t* len, int max_len, cudaStream_t st);
+cudaError_t compact_setup();
+cudaError_t launch_accept_walk(const int32_t* tokens, const int32_t* parent, const int32_t* argmax, int T,
+                               int32_t* len, int32_t* nodes, int32_t* toks, int32_t* bonus, int32_t* status,
+                               cudaStream_t st);
+
+// ---- GEMMs (gemm.cu)
+bool encode_weight_map(CUtensorMap* map, const void* ptr, int rows, int K);
+bool encode_act_map(CUtensorMap* map, const void* ptr, int K, int box_rows);
+int bn_index(int T);   // N-tile variant for T tree nodes: 0..3 -> 16/32/64/128
+cudaError_t gemm_setup();
+cudaError_t launch_gemm_tc(Model& m, const GemmW& g, const CUtensorMap& amap, int T, cudaStream_t st);
+cudaError_t launch_lm_head_tc(Model& m, int T, cudaStream_t st);
+cudaError_t launch_gemm_f32(Model& m, const void* w0, const void* w1, const void* w2, int rows0, int rows1,
+                            int rows2, int K, const void* x, int T, cudaStream_t st);
+cudaError_t launch_lm_head_f32(Model& m, int T, cudaStream_t st);
+
+// ---- attention (attn.cu)
+cudaError_t attn_setup();
+cudaError_t launch_attention(Model& m, const void* kc, const void* vc, int ctx, int T, cudaStream_t st);
+
+}  // namespace oos

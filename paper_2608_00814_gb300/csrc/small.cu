@@ -1,0 +1,472 @@
+// Small kernels of the verify step: tree preparation, embedding, the GEMM
+// reduce-epilogues (q/k/v with RoPE, residual + RMSNorm, SwiGLU), the argmax
+// merge with the greedy-acceptance walk, and KV compaction.
+#include <math.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace oos {
+
+// ============================================================ tree preparation
+// Tree encoding: parents-first numbering (parent[0] = -1, parent[i] < i).  Node
+// i attends to the committed cache and its ancestors (itself included); its
+// RoPE position is ctx + depth(i).  Ancestor sets are 128-bit masks.
+__global__ void __launch_bounds__(kMaxT) k_tree_prep(const int32_t* __restrict__ tokens,
+                                                     const int32_t* __restrict__ parent, int T, int ctx,
+                                                     int vocab, uint32_t* status, int32_t* depth_out,
+                                                     int32_t* pos_out, unsigned long long* anc_out) {
+  __shared__ int s_parent[kMaxT];
+  __shared__ int s_bad;
+  pdl_wait();
+  const int i = threadIdx.x;
+  if (i == 0) s_bad = 0;
+  __syncthreads();
+  if (i < T) {
+    const int p = parent[i];
+    const int tok = tokens[i];
+    const bool ok = (i == 0 ? p == -1 : (p >= 0 && p < i)) && tok >= 0 && tok < vocab;
+    s_parent[i] = p;
+    if (!ok) atomicOr(&s_bad, 1);
+  }
+  __syncthreads();
+  if (i == 0) *status = s_bad ? ST_TREE : 0u;
+  if (i < T) {
+    int d = 0;
+    unsigned long long lo = 0, hi = 0;
+    if (!s_bad) {
+      for (int a = i; a >= 0; a = (a == 0 ? -1 : s_parent[a])) {
+        if (a < 64) lo |= 1ull << a; else hi |= 1ull << (a - 64);
+        if (a != i) ++d;
+      }
+    } else {
+      if (i < 64) lo = 1ull << i; else hi = 1ull << (i - 64);
+    }
+    depth_out[i] = d;
+    pos_out[i] = ctx + d;
+    anc_out[2 * i] = lo;
+    anc_out[2 * i + 1] = hi;
+  }
+  pdl_trigger();
+}
+
+cudaError_t launch_tree_prep(Model& m, const int32_t* tokens, const int32_t* parent, int T, int ctx,
+                             cudaStream_t st) {
+  return launch(m.pdl, k_tree_prep, dim3(1), dim3(kMaxT), 0, st, tokens, parent, T, ctx, m.cfg.vocab,
+                m.ws.status, m.ws.depth, m.ws.pos, m.ws.anc);
+}
+
+// ============================================================ embedding + first RMSNorm
+// x[t] = E[token_t] (fp32 residual); xn[t] = x * rsqrt(mean(x^2) + eps) * g.
+template <typename E>
+__global__ void __launch_bounds__(256) k_embed_norm(const int32_t* __restrict__ tokens, const E* __restrict__ emb,
+                                                    const E* __restrict__ gain, int H, int vocab, float eps,
+                                                    float* __restrict__ x, E* __restrict__ xn) {
+  __shared__ float red[32];
+  pdl_wait();
+  const int t = blockIdx.x;
+  int tok = tokens[t];
+  tok = tok < 0 ? 0 : (tok >= vocab ? vocab - 1 : tok);   // invalid trees are flagged by tree_prep
+  const E* row = emb + (size_t)tok * H;
+  float ss = 0.f;
+  for (int f = threadIdx.x; f < H; f += blockDim.x) {
+    const float v = to_f32(row[f]);
+    x[(size_t)t * H + f] = v;
+    ss += v * v;
+  }
+  ss = block_sum(ss, red);
+  const float r = rsqrtf(ss / (float)H + eps);
+  for (int f = threadIdx.x; f < H; f += blockDim.x)
+    xn[(size_t)t * H + f] = from_f32<E>(x[(size_t)t * H + f] * r * to_f32(gain[f]));
+  pdl_trigger();
+}
+
+cudaError_t launch_embed_norm(Model& m, const int32_t* tokens, int T, cudaStream_t st) {
+  const auto& c = m.cfg;
+  if (c.dtype == OOS_DTYPE_BF16)
+    return launch(m.pdl, k_embed_norm<__nv_bfloat16>, dim3(T), dim3(256), 0, st, tokens,
+                  (const __nv_bfloat16*)m.w.embed, (const __nv_bfloat16*)m.layers[0].attn_norm, c.hidden,
+                  c.vocab, c.rms_eps, m.ws.x, (__nv_bfloat16*)m.ws.xn);
+  return launch(m.pdl, k_embed_norm<float>, dim3(T), dim3(256), 0, st, tokens, (const float*)m.w.embed,
+                (const float*)m.layers[0].attn_norm, c.hidden, c.vocab, c.rms_eps, m.ws.x, (float*)m.ws.xn);
+}
+
+// sum of the fp32 partial slices of GEMM output (t, f)
+OOS_DEV float gather_partial(const float* __restrict__ part, const StreamK& plan, int N, int t, int f) {
+  int c0, c1;
+  plan.contributors(f / kTile, c0, c1);
+  float v = 0.f;
+  const size_t slice = (size_t)kMaxT * N;
+  for (int s = 0; s <= c1 - c0; ++s) v += part[s * slice + (size_t)t * N + f];
+  return v;
+}
+
+// ============================================================ q/k/v epilogue
+// One block per (node t, head slot hs in [0, nq + 2 nkv)); thread j owns the
+// rotate-half pair (j, j + d/2).  q/k: optional per-head RMSNorm, then RoPE at
+// pos[t]; q goes to the query buffer, k and v to cache slot ctx + t.
+struct QkvPostArgs {
+  const float* part;
+  StreamK plan;
+  int N, nq, nkv, d;
+  const void* bq;
+  const void* bk;
+  const void* bv;
+  const void* gq;
+  const void* gk;
+  float eps;
+  const int32_t* pos;
+  const double* inv_freq;
+  void* q;
+  void* kc;
+  void* vc;
+  int ctx;
+};
+
+template <typename E>
+__global__ void k_qkv_post(QkvPostArgs a) {
+  __shared__ float red[32];
+  pdl_wait();
+  const int t = blockIdx.x, hs = blockIdx.y, j = threadIdx.x, half = a.d / 2;
+  const int f0 = hs * a.d + j, f1 = f0 + half;
+  float v0 = gather_partial(a.part, a.plan, a.N, t, f0);
+  float v1 = gather_partial(a.part, a.plan, a.N, t, f1);
+  int kind, h;  // 0 = q, 1 = k, 2 = v
+  if (hs < a.nq) { kind = 0; h = hs; }
+  else if (hs < a.nq + a.nkv) { kind = 1; h = hs - a.nq; }
+  else { kind = 2; h = hs - a.nq - a.nkv; }
+  const E* bias = (const E*)(kind == 0 ? a.bq : kind == 1 ? a.bk : a.bv);
+  if (bias) {
+    v0 += to_f32(bias[h * a.d + j]);
+    v1 += to_f32(bias[h * a.d + j + half]);
+  }
+  if (kind < 2) {
+    const E* g = (const E*)(kind == 0 ? a.gq : a.gk);
+    if (g) {
+      const float ss = block_sum(v0 * v0 + v1 * v1, red);
+      const float r = rsqrtf(ss / (float)a.d + a.eps);
+      v0 = v0 * r * to_f32(g[j]);
+      v1 = v1 * r * to_f32(g[j + half]);
+    }
+    // angle = pos * theta^(-2j/d), reduced to [-pi, pi] before the fp32 sincos
+    const double ang = (double)a.pos[t] * a.inv_freq[j];
+    const double two_pi = 6.283185307179586476925286766559;
+    const float red_ang = (float)(ang - two_pi * rint(ang / two_pi));
+    float s, c;
+    sincosf(red_ang, &s, &c);
+    const float o0 = v0 * c - v1 * s;
+    const float o1 = v1 * c + v0 * s;
+    v0 = o0;
+    v1 = o1;
+  }
+  E* dst;
+  if (kind == 0) dst = (E*)a.q + ((size_t)t * a.nq + h) * a.d;
+  else dst = (E*)(kind == 1 ? a.kc : a.vc) + ((size_t)(a.ctx + t) * a.nkv + h) * a.d;
+  dst[j] = from_f32<E>(v0);
+  dst[j + half] = from_f32<E>(v1);
+  pdl_trigger();
+}
+
+cudaError_t launch_qkv_post(Model& m, int layer, const StreamK& plan, void* kc, void* vc, int ctx, int T,
+                            cudaStream_t st) {
+  const auto& c = m.cfg;
+  const auto& L = m.layers[layer];
+  QkvPostArgs a;
+  a.part = m.ws.part;
+  a.plan = plan;
+  a.nq = c.n_q_heads;
+  a.nkv = c.n_kv_heads;
+  a.d = c.head_dim;
+  a.N = (c.n_q_heads + 2 * c.n_kv_heads) * c.head_dim;
+  a.bq = c.qkv_bias ? L.b_q : nullptr;
+  a.bk = c.qkv_bias ? L.b_k : nullptr;
+  a.bv = c.qkv_bias ? L.b_v : nullptr;
+  a.gq = c.qk_norm ? L.q_norm : nullptr;
+  a.gk = c.qk_norm ? L.k_norm : nullptr;
+  a.eps = c.rms_eps;
+  a.pos = m.ws.pos;
+  a.inv_freq = m.ws.inv_freq;
+  a.q = m.ws.q;
+  a.kc = kc;
+  a.vc = vc;
+  a.ctx = ctx;
+  dim3 grid(T, c.n_q_heads + 2 * c.n_kv_heads);
+  if (c.dtype == OOS_DTYPE_BF16) return launch(m.pdl, k_qkv_post<__nv_bfloat16>, grid, dim3(c.head_dim / 2), 0, st, a);
+  return launch(m.pdl, k_qkv_post<float>, grid, dim3(c.head_dim / 2), 0, st, a);
+}
+
+// ============================================================ residual add + RMSNorm
+// x[t] += sum of partial slices (O-projection or down-projection output);
+// xn[t] = RMSNorm(x[t]) * gain (input of the next GEMM).  For the final norm
+// the fp32 normalised row is also written to hidden_out (when given).
+template <typename E>
+__global__ void __launch_bounds__(256) k_resid_norm(const float* __restrict__ part, StreamK plan, int H,
+                                                    const E* __restrict__ gain, float eps, float* __restrict__ x,
+                                                    E* __restrict__ xn, float* __restrict__ hidden_out) {
+  __shared__ float red[32];
+  pdl_wait();
+  const int t = blockIdx.x;
+  float* xr = x + (size_t)t * H;
+  float ss = 0.f;
+  for (int f = threadIdx.x; f < H; f += blockDim.x) {
+    const float v = xr[f] + gather_partial(part, plan, H, t, f);
+    xr[f] = v;
+    ss += v * v;
+  }
+  ss = block_sum(ss, red);
+  const float r = rsqrtf(ss / (float)H + eps);
+  for (int f = threadIdx.x; f < H; f += blockDim.x) {
+    const float y = xr[f] * r * to_f32(gain[f]);
+    xn[(size_t)t * H + f] = from_f32<E>(y);
+    if (hidden_out) hidden_out[(size_t)t * H + f] = y;
+  }
+  pdl_trigger();
+}
+
+cudaError_t launch_resid_norm(Model& m, const StreamK& plan, const void* gain, float* hidden_out, int T,
+                              cudaStream_t st) {
+  const auto& c = m.cfg;
+  if (c.dtype == OOS_DTYPE_BF16)
+    return launch(m.pdl, k_resid_norm<__nv_bfloat16>, dim3(T), dim3(256), 0, st, (const float*)m.ws.part, plan,
+                  c.hidden, (const __nv_bfloat16*)gain, c.rms_eps, m.ws.x, (__nv_bfloat16*)m.ws.xn, hidden_out);
+  return launch(m.pdl, k_resid_norm<float>, dim3(T), dim3(256), 0, st, (const float*)m.ws.part, plan, c.hidden,
+                (const float*)gain, c.rms_eps, m.ws.x, (float*)m.ws.xn, hidden_out);
+}
+
+// ============================================================ SwiGLU
+// act[t][i] = silu(gate) * up, gate/up = rows i and I + i of the stacked GEMM.
+template <typename E>
+__global__ void __launch_bounds__(256) k_silu_mul(const float* __restrict__ part, StreamK plan, int I,
+                                                  E* __restrict__ act) {
+  pdl_wait();
+  const int t = blockIdx.y;
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i < I) {
+    const float g = gather_partial(part, plan, 2 * I, t, i);
+    const float u = gather_partial(part, plan, 2 * I, t, I + i);
+    act[(size_t)t * I + i] = from_f32<E>(g / (1.f + expf(-g)) * u);
+  }
+  pdl_trigger();
+}
+
+cudaError_t launch_silu_mul(Model& m, const StreamK& plan, int T, cudaStream_t st) {
+  const auto& c = m.cfg;
+  dim3 grid((c.intermediate + 255) / 256, T);
+  if (c.dtype == OOS_DTYPE_BF16)
+    return launch(m.pdl, k_silu_mul<__nv_bfloat16>, grid, dim3(256), 0, st, (const float*)m.ws.part, plan,
+                  c.intermediate, (__nv_bfloat16*)m.ws.act);
+  return launch(m.pdl, k_silu_mul<float>, grid, dim3(256), 0, st, (const float*)m.ws.part, plan, c.intermediate,
+                (float*)m.ws.act);
+}
+
+// ============================================================ argmax merge + acceptance walk
+// Running greedy state: largest logit, its (lowest) vocab id, second largest
+// logit counted with multiplicity.
+struct Top2 {
+  float v1;
+  int i1;
+  float v2;
+};
+OOS_DEV Top2 top2_merge(Top2 a, Top2 b) {
+  Top2 r;
+  if (a.v1 > b.v1 || (a.v1 == b.v1 && a.i1 <= b.i1)) {
+    r.v1 = a.v1;
+    r.i1 = a.i1;
+  } else {
+    r.v1 = b.v1;
+    r.i1 = b.i1;
+  }
+  r.v2 = fmaxf(fminf(a.v1, b.v1), fmaxf(a.v2, b.v2));
+  return r;
+}
+
+// Greedy longest-prefix acceptance (Eq. 1; "Verify and commit") by one warp.
+// ok(0) = 1; ok(i) = ok(parent) and token_i == argmax(parent).  The committed
+// path ends at the deepest ok node (lowest id on ties); bonus = its argmax.
+OOS_DEV void accept_walk_warp(const int32_t* tokens, const int32_t* parent, const int32_t* depth,
+                              const int32_t* argmax, int T, bool bad, int32_t* len_out, int32_t* nodes_out,
+                              int32_t* toks_out, int32_t* bonus_out) {
+  const int lane = threadIdx.x & 31;
+  if (bad) {
+    for (int i = lane; i < T; i += 32) {
+      nodes_out[i] = -1;
+      toks_out[i] = -1;
+    }
+    if (lane == 0) {
+      *len_out = 0;
+      *bonus_out = -1;
+    }
+    return;
+  }
+  int best_key = 0x7fffffff;  // key = (kMaxT - depth) * 256 + node: min = deepest, then lowest id
+  for (int i = lane; i < T; i += 32) {
+    bool ok = true;
+    for (int a = i; a != 0; a = parent[a]) {
+      const int p = parent[a];
+      if (tokens[a] != argmax[p]) {
+        ok = false;
+        break;
+      }
+    }
+    if (ok) {
+      const int key = (kMaxT - depth[i]) * 256 + i;
+      best_key = key < best_key ? key : best_key;
+    }
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const int other = __shfl_xor_sync(0xffffffffu, best_key, o);
+    best_key = other < best_key ? other : best_key;
+  }
+  const int deepest = best_key & 255;
+  const int len = depth[deepest] + 1;
+  for (int j = len + lane; j < T; j += 32) {
+    nodes_out[j] = -1;
+    toks_out[j] = -1;
+  }
+  if (lane == 0) {
+    for (int a = deepest; a >= 0; a = (a == 0 ? -1 : parent[a])) {
+      nodes_out[depth[a]] = a;
+      toks_out[depth[a]] = tokens[a];
+    }
+    *len_out = len;
+    *bonus_out = argmax[deepest];
+  }
+}
+
+__global__ void __launch_bounds__(kMaxT) k_argmax_accept(const float* __restrict__ v1, const int32_t* __restrict__ i1,
+                                                         const float* __restrict__ v2, int n_parts,
+                                                         const int32_t* __restrict__ tokens,
+                                                         const int32_t* __restrict__ parent,
+                                                         const int32_t* __restrict__ depth, const uint32_t* status,
+                                                         int T, int32_t* argmax_ws, float* top1_ws, float* top2_ws,
+                                                         int32_t* len, int32_t* nodes, int32_t* toks, int32_t* bonus,
+                                                         int32_t* dbg_argmax, float* dbg_top1, float* dbg_top2) {
+  __shared__ int32_t s_tok[kMaxT], s_par[kMaxT], s_dep[kMaxT], s_arg[kMaxT];
+  pdl_wait();
+  const int t = threadIdx.x;
+  if (t < T) {
+    Top2 r{-INFINITY, 0x7fffffff, -INFINITY};
+    for (int c = 0; c < n_parts; ++c) {
+      const size_t k = (size_t)c * kMaxT + t;
+      r = top2_merge(r, Top2{v1[k], i1[k], v2[k]});
+    }
+    argmax_ws[t] = r.i1;
+    top1_ws[t] = r.v1;
+    top2_ws[t] = r.v2;
+    if (dbg_argmax) dbg_argmax[t] = r.i1;
+    if (dbg_top1) dbg_top1[t] = r.v1;
+    if (dbg_top2) dbg_top2[t] = r.v2;
+    s_arg[t] = r.i1;
+    s_tok[t] = tokens[t];
+    s_par[t] = parent[t];
+    s_dep[t] = depth[t];
+  }
+  __syncthreads();
+  if (t < 32) accept_walk_warp(s_tok, s_par, s_dep, s_arg, T, (*status & ST_TREE) != 0, len, nodes, toks, bonus);
+  pdl_trigger();
+}
+
+cudaError_t launch_argmax_accept(Model& m, const int32_t* tokens, const int32_t* parent, int T, int n_parts,
+                                 int32_t* len, int32_t* nodes, int32_t* toks, int32_t* bonus, int32_t* dbg_argmax,
+                                 float* dbg_top1, float* dbg_top2, cudaStream_t st) {
+  return launch(m.pdl, k_argmax_accept, dim3(1), dim3(kMaxT), 0, st, (const float*)m.ws.lm_v1,
+                (const int32_t*)m.ws.lm_i, (const float*)m.ws.lm_v2, n_parts, tokens, parent,
+                (const int32_t*)m.ws.depth, (const uint32_t*)m.ws.status, T, m.ws.argmax, m.ws.top1, m.ws.top2,
+                len, nodes, toks, bonus, dbg_argmax, dbg_top1, dbg_top2);
+}
+
+// standalone walk: validates the tree itself
+__global__ void k_accept_walk(const int32_t* tokens, const int32_t* parent, const int32_t* argmax, int T,
+                              int32_t* len, int32_t* nodes, int32_t* toks, int32_t* bonus, int32_t* status) {
+  __shared__ int32_t s_tok[kMaxT], s_par[kMaxT], s_dep[kMaxT], s_arg[kMaxT];
+  __shared__ int s_bad;
+  const int i = threadIdx.x;
+  if (i == 0) s_bad = 0;
+  __syncthreads();
+  if (i < T) {
+    s_tok[i] = tokens[i];
+    s_par[i] = parent[i];
+    s_arg[i] = argmax[i];
+    const bool ok = i == 0 ? s_par[i] == -1 : (s_par[i] >= 0 && s_par[i] < i);
+    if (!ok) atomicOr(&s_bad, 1);
+  }
+  __syncthreads();
+  if (i < T) {
+    int d = 0;
+    if (!s_bad)
+      for (int a = i; a != 0; a = s_par[a]) ++d;
+    s_dep[i] = d;
+  }
+  __syncthreads();
+  if (i < 32) accept_walk_warp(s_tok, s_par, s_dep, s_arg, T, s_bad != 0, len, nodes, toks, bonus);
+  if (i == 0) *status = s_bad ? OOS_ETREE : OOS_OK;
+}
+
+cudaError_t launch_accept_walk(const int32_t* tokens, const int32_t* parent, const int32_t* argmax, int T,
+                               int32_t* len, int32_t* nodes, int32_t* toks, int32_t* bonus, int32_t* status,
+                               cudaStream_t st) {
+  k_accept_walk<<<1, kMaxT, 0, st>>>(tokens, parent, argmax, T, len, nodes, toks, bonus, status);
+  return cudaGetLastError();
+}
+
+// ============================================================ KV compaction
+// Slot ctx + j <- slot ctx + nodes[j] for j < len, per layer, for K and V.
+// One block per (layer, K|V, kv head): all sources are staged in shared
+// memory before any destination is written, so a source that is also a later
+// destination is read before it is overwritten.
+struct KvPtrs {
+  void* k[kMaxLayers];
+  void* v[kMaxLayers];
+};
+
+template <typename E>
+__global__ void k_kv_compact(KvPtrs p, int nkv, int d, int ctx, const int32_t* __restrict__ nodes,
+                             const int32_t* __restrict__ len_ptr, int max_len) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  E* buf = reinterpret_cast<E*>(smem_raw);
+  pdl_wait();
+  const int layer = blockIdx.x, which = blockIdx.y, g = blockIdx.z;
+  E* base = (E*)(which == 0 ? p.k[layer] : p.v[layer]);
+  int len = *len_ptr;
+  len = len < 0 ? 0 : (len > max_len ? max_len : len);
+  for (int e = threadIdx.x; e < len * d; e += blockDim.x) {
+    const int j = e / d, c = e % d;
+    const int src = nodes[j];
+    if (src >= 0 && src < max_len) buf[e] = base[((size_t)(ctx + src) * nkv + g) * d + c];
+  }
+  __syncthreads();
+  for (int e = threadIdx.x; e < len * d; e += blockDim.x) {
+    const int j = e / d, c = e % d;
+    const int src = nodes[j];
+    if (src >= 0 && src < max_len) base[((size_t)(ctx + j) * nkv + g) * d + c] = buf[e];
+  }
+  pdl_trigger();
+}
+
+cudaError_t compact_setup() {
+  cudaError_t e = cudaFuncSetAttribute(k_kv_compact<float>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       kMaxT * 128 * 4);
+  if (e != cudaSuccess) return e;
+  return cudaFuncSetAttribute(k_kv_compact<__nv_bfloat16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              kMaxT * 128 * 2);
+}
+
+cudaError_t launch_kv_compact(Model& m, const oos_kv_cache& kv, int ctx, const int32_t* nodes, const int32_t* len,
+                              int max_len, cudaStream_t st) {
+  const auto& c = m.cfg;
+  KvPtrs p;
+  for (int l = 0; l < c.n_layers; ++l) {
+    p.k[l] = kv.k[l];
+    p.v[l] = kv.v[l];
+  }
+  dim3 grid(c.n_layers, 2, c.n_kv_heads);
+  const size_t smem = (size_t)max_len * c.head_dim * m.esize;
+  if (c.dtype == OOS_DTYPE_BF16)
+    return launch(m.pdl, k_kv_compact<__nv_bfloat16>, grid, dim3(256), smem, st, p, c.n_kv_heads, c.head_dim, ctx,
+                  nodes, len, max_len);
+  return launch(m.pdl, k_kv_compact<float>, grid, dim3(256), smem, st, p, c.n_kv_heads, c.head_dim, ctx, nodes, len,
+                max_len);
+}
+
+}  // namespace oos

@@ -96,7 +96,23 @@ WORKLOADS = {
                             tree=dict(kind="branch", bmin=1, bmax=4, max_depth=12)),
 }
 
-MODELS = {w.model.name: w.model for w in WORKLOADS.values()}
+# A small bf16 decoder with the head_dim of the real targets: runs every
+# tensor-core kernel of the bf16 path at sizes the CPU checker finishes in
+# seconds (tests and the smoke check only; not a benchmark workload).
+MINI_BF16 = ModelConfig("mini-bf16", n_layers=2, hidden=256, n_q_heads=4, n_kv_heads=2,
+                        head_dim=128, intermediate=512, vocab=4096, rms_eps=1e-6,
+                        rope_theta=1e6, dtype="bf16", qk_norm=True, qkv_bias=False, tied=False)
+
+TEST_WORKLOADS = {
+    "mini-bf16": Workload(MINI_BF16, ctx_len=200, T=16, plant=3,
+                          tree=dict(kind="uniform", max_depth=6), prefill=True),
+}
+
+MODELS = {w.model.name: w.model for w in list(WORKLOADS.values()) + list(TEST_WORKLOADS.values())}
+
+
+def workload(name):
+    return WORKLOADS[name] if name in WORKLOADS else TEST_WORKLOADS[name]
 
 
 def weight_bytes(cfg: ModelConfig) -> dict:

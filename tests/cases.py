@@ -13,7 +13,7 @@ import numpy as np
 
 import oracle
 from synth import gen, trees
-from synth.configs import WORKLOADS
+from synth.configs import workload
 from synth.model import PROMPT, ROOT, TREE_SHAPE, SynthModel, synthetic_kv
 
 GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
@@ -71,9 +71,9 @@ def root_token(cfg, seed):
 
 
 def build_case(name="tiny", seed=0, T=None, recipe=None, plant=None, ctx_len=None,
-               cfg_overrides=None, gain_std=0.0, planted=None, prefill=None):
+               cfg_overrides=None, gain_std=0.0, planted=None, prefill=None, root=None):
     """A verify-step case for workload `name` (defaults from its recipe)."""
-    w = WORKLOADS[name]
+    w = workload(name)
     cfg = w.model if not cfg_overrides else dataclasses.replace(w.model, **cfg_overrides)
     T = w.T if T is None else T
     recipe = w.tree if recipe is None else recipe
@@ -86,7 +86,7 @@ def build_case(name="tiny", seed=0, T=None, recipe=None, plant=None, ctx_len=Non
         native, k64, v64 = tiny_cache(cfg, model, view, seed, ctx_len)
     else:
         native, k64, v64 = synthetic_cache(cfg, seed, ctx_len)
-    root = root_token(cfg, seed)
+    root = root_token(cfg, seed) if root is None else int(root)
     if planted is None:
         if plant > 0:
             planted, margins = oracle.greedy_continuation(view, k64, v64, ctx_len, root, plant)

@@ -1,0 +1,83 @@
+"""Write golden/planted.json: a root token and the target's own greedy
+continuation per bf16 workload.
+
+Calls only the CPU checker (oracle) on seeded synthetic inputs.  For each
+workload (weights seed 0, synthetic committed cache) it draws candidate root
+tokens from the seeded ROOT stream, k = 0, 1, ..., and decodes greedily from
+each (Eq. 1 applied repeatedly) until `plant` tokens plus the bonus token are
+found whose top-1/top-2 logit margins all exceed MIN_MARGIN.  A path with a
+near-tie could be decided either way by a bf16 verifier, so exact comparison of
+the accept outputs is only meaningful on such well-separated paths.
+
+Usage: python tests/golden/make_planted.py [workload ...]
+"""
+
+import json
+import os
+import sys
+import time
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+ROOT = os.path.dirname(os.path.dirname(HERE))
+sys.path.insert(0, ROOT)
+sys.path.insert(0, os.path.dirname(HERE))
+
+import oracle  # noqa: E402
+from cases import synthetic_cache  # noqa: E402
+from synth import gen  # noqa: E402
+from synth.configs import WORKLOADS  # noqa: E402
+from synth.model import ROOT as ROOT_KIND, SynthModel  # noqa: E402
+
+OUT = os.path.join(HERE, "planted.json")
+MIN_MARGIN = 0.06       # the tests gate at 0.05
+MAX_ROOTS = 64
+
+
+def plant_one(name, seed=0):
+    w = WORKLOADS[name]
+    cfg = w.model
+    view = SynthModel(cfg, seed).oracle_view()
+    _, k64, v64 = synthetic_cache(cfg, seed, w.ctx_len)
+    roots = gen.uniform_int(gen.tensor_key(seed, ROOT_KIND), MAX_ROOTS, cfg.vocab)
+    for k in range(MAX_ROOTS):
+        root = int(roots[k])
+        ck = [np.array(c) for c in k64]
+        cv = [np.array(c) for c in v64]
+        n_pos, tok, toks, margins = w.ctx_len, root, [], []
+        while len(toks) < w.plant + 1:
+            _, a, t1, t2, ks, vs = oracle.decode_step(view, ck, cv, n_pos, tok)
+            margins.append(t1 - t2)
+            if t1 - t2 <= MIN_MARGIN:
+                break
+            toks.append(a)
+            ck = [np.concatenate([c, x[None]]) for c, x in zip(ck, ks)]
+            cv = [np.concatenate([c, x[None]]) for c, x in zip(cv, vs)]
+            n_pos += 1
+            tok = a
+        print("  %s root #%d: %d/%d decisions above margin" % (name, k, len(toks), w.plant + 1), flush=True)
+        if len(toks) == w.plant + 1:
+            return dict(seed=seed, ctx_len=w.ctx_len, root_index=k, root=root, planted=toks[:w.plant],
+                        bonus=toks[w.plant], margins=margins,
+                        note="oracle greedy continuation after the root on the synthetic cache; every margin "
+                             "> %.2f" % MIN_MARGIN)
+    raise RuntimeError("no well-separated greedy path found for %s" % name)
+
+
+def main(names):
+    data = {}
+    if os.path.exists(OUT):
+        with open(OUT) as f:
+            data = json.load(f)
+    for name in names:
+        t0 = time.time()
+        data[name] = plant_one(name)
+        print(name, data[name]["planted"], ["%.3f" % m for m in data[name]["margins"]],
+              "%.0fs" % (time.time() - t0), flush=True)
+        with open(OUT, "w") as f:
+            json.dump(data, f, indent=1)
+
+
+if __name__ == "__main__":
+    main(sys.argv[1:] or [n for n, w in WORKLOADS.items() if w.model.dtype == "bf16"])
