@@ -101,7 +101,8 @@ WORKLOADS = {
 # seconds (tests and the smoke check only; not a benchmark workload).
 MINI_BF16 = ModelConfig("mini-bf16", n_layers=2, hidden=256, n_q_heads=4, n_kv_heads=2,
                         head_dim=128, intermediate=512, vocab=4096, rms_eps=1e-6,
-                        rope_theta=1e6, dtype="bf16", qk_norm=True, qkv_bias=False, tied=False)
+                        rope_theta=1e6, dtype="bf16", qk_norm=True, qkv_bias=False, tied=False,
+                        init_std=0.08)
 
 TEST_WORKLOADS = {
     "mini-bf16": Workload(MINI_BF16, ctx_len=200, T=16, plant=3,

@@ -58,14 +58,14 @@ uint64_t synth_stream_at(uint64_t key, uint64_t i) { return stream_at(key, i); }
 /* out[j] = bf16 bits of element offset+j; mult = fp32(sigma*sqrt(3)/65536). */
 void synth_normal_bf16(uint64_t key, uint64_t offset, int64_t n, float mult,
                        uint16_t *out) {
-#pragma omp parallel for schedule(static)
+#pragma omp parallel for schedule(static) if (n >= (1 << 20))
   for (int64_t j = 0; j < n; ++j)
     out[j] = bf16_rne(ih4(stream_at(key, offset + (uint64_t)j), mult));
 }
 
 void synth_normal_f32(uint64_t key, uint64_t offset, int64_t n, float mult,
                       float *out) {
-#pragma omp parallel for schedule(static)
+#pragma omp parallel for schedule(static) if (n >= (1 << 20))
   for (int64_t j = 0; j < n; ++j)
     out[j] = ih4(stream_at(key, offset + (uint64_t)j), mult);
 }
@@ -73,14 +73,14 @@ void synth_normal_f32(uint64_t key, uint64_t offset, int64_t n, float mult,
 /* The same values widened exactly to fp64 (for the fp64 checker). */
 void synth_normal_bf16_f64(uint64_t key, uint64_t offset, int64_t n, float mult,
                            double *out) {
-#pragma omp parallel for schedule(static)
+#pragma omp parallel for schedule(static) if (n >= (1 << 20))
   for (int64_t j = 0; j < n; ++j)
     out[j] = bf16_to_f64(bf16_rne(ih4(stream_at(key, offset + (uint64_t)j), mult)));
 }
 
 void synth_normal_f32_f64(uint64_t key, uint64_t offset, int64_t n, float mult,
                           double *out) {
-#pragma omp parallel for schedule(static)
+#pragma omp parallel for schedule(static) if (n >= (1 << 20))
   for (int64_t j = 0; j < n; ++j)
     out[j] = (double)ih4(stream_at(key, offset + (uint64_t)j), mult);
 }
@@ -88,7 +88,7 @@ void synth_normal_f32_f64(uint64_t key, uint64_t offset, int64_t n, float mult,
 /* Uniform integers in [0, bound): high 32 bits times bound, shifted (Lemire). */
 void synth_uniform_int(uint64_t key, uint64_t offset, int64_t n, uint32_t bound,
                        int32_t *out) {
-#pragma omp parallel for schedule(static)
+#pragma omp parallel for schedule(static) if (n >= (1 << 20))
   for (int64_t j = 0; j < n; ++j)
     out[j] = (int32_t)(((stream_at(key, offset + (uint64_t)j) >> 32) * (uint64_t)bound) >> 32);
 }
