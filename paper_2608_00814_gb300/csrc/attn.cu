@@ -275,7 +275,8 @@ __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
 
 // merge the splits of one (node, head) row: log-sum-exp weights in base 2
 __global__ void __launch_bounds__(kAttnD) k_attn_merge(const float* __restrict__ o_part, const float* __restrict__ ml,
-                                                       int splits, int rows_total, __nv_bfloat16* __restrict__ out) {
+                                                       int splits, int rows_total, size_t rows_lo_off,
+                                                       __nv_bfloat16* __restrict__ out) {
   pdl_trigger();
   pdl_wait();
   const int row = blockIdx.x, c = threadIdx.x;
@@ -289,7 +290,7 @@ __global__ void __launch_bounds__(kAttnD) k_attn_merge(const float* __restrict__
     den += w * ml[((size_t)s * rows_total + row) * 2 + 1];
     num += w * o_part[((size_t)s * rows_total + row) * kAttnD + c];
   }
-  out[(size_t)row * kAttnD + c] = __float2bfloat16_rn(num / den);
+  store_act(out, (size_t)row * kAttnD + c, (size_t)rows_lo_off, num / den);
 }
 
 // ------------------------------------------------------------ fp32 path
@@ -378,7 +379,8 @@ cudaError_t launch_attention(Model& m, const void* kc, const void* vc, int ctx, 
   cudaError_t e = launch(m.pdl, k_attn_tc, dim3(RB, a.nkv, splits), dim3(128), (size_t)kAttnSmem, st, a);
   if (e != cudaSuccess) return e;
   return launch(m.pdl, k_attn_merge, dim3(T * c.n_q_heads), dim3(kAttnD), 0, st, (const float*)m.ws.attn_o,
-                (const float*)m.ws.attn_ml, splits, T * c.n_q_heads, (__nv_bfloat16*)m.ws.attn);
+                (const float*)m.ws.attn_ml, splits, T * c.n_q_heads, (size_t)kMaxT * c.n_q_heads * kAttnD,
+                (__nv_bfloat16*)m.ws.attn);
 }
 
 }  // namespace oos

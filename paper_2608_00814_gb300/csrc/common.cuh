@@ -31,6 +31,16 @@ template <typename T> OOS_DEV T from_f32(float v);
 template <> OOS_DEV float from_f32<float>(float v) { return v; }
 template <> OOS_DEV __nv_bfloat16 from_f32<__nv_bfloat16>(float v) { return __float2bfloat16_rn(v); }
 
+// GEMM activations of the bf16 path are stored as a pair hi = bf16(v),
+// lo = bf16(v - hi) (lo at element offset lo_off): the tensor cores see v to
+// about 16 mantissa bits while the weights stay bf16.  fp32 models store v.
+OOS_DEV void store_act(float* p, size_t i, size_t lo_off, float v) { p[i] = v; }
+OOS_DEV void store_act(__nv_bfloat16* p, size_t i, size_t lo_off, float v) {
+  const __nv_bfloat16 hi = __float2bfloat16_rn(v);
+  p[i] = hi;
+  p[i + lo_off] = __float2bfloat16_rn(v - __bfloat162float(hi));
+}
+
 // ---- block reductions (deterministic order)
 OOS_DEV float warp_sum(float v) {
 #pragma unroll

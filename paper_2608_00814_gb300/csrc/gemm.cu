@@ -37,8 +37,8 @@ struct GemmArgs {
 template <int BN>
 struct TcCfg {
   static constexpr int A_BYTES = kTile * kBK * 2;              // 16 KB weight tile
-  static constexpr int B_BYTES = BN * kBK * 2;                 // activation slice
-  static constexpr int STAGE = A_BYTES + B_BYTES;
+  static constexpr int B_BYTES = BN * kBK * 2;                 // one activation half (hi or lo)
+  static constexpr int STAGE = A_BYTES + 2 * B_BYTES;
   static constexpr int S_RAW = (200 * 1024) / STAGE;
   static constexpr int S = S_RAW > 8 ? 8 : S_RAW;
   static constexpr int NCOLS = (2 * BN) < 32 ? 32 : 2 * BN;    // two accumulators, power of two
@@ -74,7 +74,7 @@ __global__ void __launch_bounds__(192, 1)
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   unsigned char* sA = smem;
-  unsigned char* sB = smem + S * C::A_BYTES;
+  unsigned char* sB = smem + S * C::A_BYTES;      // [stage][hi|lo][BN rows x 128 B]
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + S * C::STAGE);
   uint64_t* empty = full + S;
   uint64_t* accf = empty + S;
@@ -158,7 +158,9 @@ __global__ void __launch_bounds__(192, 1)
       auto load_x = [&](int j, int stage) {
         int tile, kb;
         unit_tile(j, tile, kb);
-        tma_load_2d(sB + stage * C::B_BYTES, &am, &full[stage], kb * kBK, 0, pol_a);
+        unsigned char* dst = sB + stage * 2 * C::B_BYTES;
+        tma_load_2d(dst, &am, &full[stage], kb * kBK, 0, pol_a);                   // hi rows
+        tma_load_2d(dst + C::B_BYTES, &am, &full[stage], kb * kBK, kMaxT, pol_a);  // lo rows
       };
       // weights do not depend on the previous kernel: start streaming them
       // before waiting for it (programmatic dependent launch)
@@ -219,10 +221,13 @@ __global__ void __launch_bounds__(192, 1)
           }
           tc_fence_after();
           const uint64_t ad = smem_desc_sw128(smem_addr(sA + stage * C::A_BYTES));
-          const uint64_t bd = smem_desc_sw128(smem_addr(sB + stage * C::B_BYTES));
+          const uint64_t bh = smem_desc_sw128(smem_addr(sB + stage * 2 * C::B_BYTES));
+          const uint64_t bl = smem_desc_sw128(smem_addr(sB + stage * 2 * C::B_BYTES + C::B_BYTES));
 #pragma unroll
-          for (int k = 0; k < kBK / 16; ++k)
-            tc_mma_bf16(d_tmem, ad + 2 * k, bd + 2 * k, idesc, (jj > j || k > 0) ? 1u : 0u);
+          for (int k = 0; k < kBK / 16; ++k) {
+            tc_mma_bf16(d_tmem, ad + 2 * k, bh + 2 * k, idesc, (jj > j || k > 0) ? 1u : 0u);
+            tc_mma_bf16(d_tmem, ad + 2 * k, bl + 2 * k, idesc, 1u);
+          }
           tc_commit(&empty[stage]);
           if (++stage == S) {
             stage = 0;
@@ -365,7 +370,7 @@ bool encode_weight_map(CUtensorMap* map, const void* ptr, int rows, int K) {
   return encode_2d(map, ptr, rows, K, kTile);
 }
 bool encode_act_map(CUtensorMap* map, const void* ptr, int K, int box_rows) {
-  return encode_2d(map, ptr, kMaxT, K, box_rows);
+  return encode_2d(map, ptr, 2 * kMaxT, K, box_rows);   // hi rows [0, 128), lo rows [128, 256)
 }
 
 int bn_index(int T) { return T <= 16 ? 0 : T <= 32 ? 1 : T <= 64 ? 2 : 3; }

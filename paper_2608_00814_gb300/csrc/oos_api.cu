@@ -56,11 +56,12 @@ size_t carve_workspace(const oos_model_config& c, int n_sms, uint8_t* base, Work
   w.depth = (int32_t*)take(kMaxT * 4);
   w.pos = (int32_t*)take(kMaxT * 4);
   w.anc = (unsigned long long*)take(kMaxT * 16);
+  const size_t halves = c.dtype == OOS_DTYPE_BF16 ? 2 : 1;   // bf16: hi rows then lo rows
   w.x = (float*)take(kMaxT * H * 4);
-  w.xn = take(kMaxT * H * es);
+  w.xn = take(halves * kMaxT * H * es);
   w.q = take(kMaxT * qd * es);
-  w.attn = take(kMaxT * qd * es);
-  w.act = take(kMaxT * I * es);
+  w.attn = take(halves * kMaxT * qd * es);
+  w.act = take(halves * kMaxT * I * es);
   size_t pf = 0;
   const int Nq = (int)(qd + 2 * kvd);
   if (c.dtype == OOS_DTYPE_BF16) {

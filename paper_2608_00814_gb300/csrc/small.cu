@@ -77,7 +77,7 @@ __global__ void __launch_bounds__(256) k_embed_norm(const int32_t* __restrict__ 
   ss = block_sum(ss, red);
   const float r = rsqrtf(ss / (float)H + eps);
   for (int f = threadIdx.x; f < H; f += blockDim.x)
-    xn[(size_t)t * H + f] = from_f32<E>(x[(size_t)t * H + f] * r * to_f32(gain[f]));
+    store_act(xn, (size_t)t * H + f, (size_t)kMaxT * H, x[(size_t)t * H + f] * r * to_f32(gain[f]));
   pdl_trigger();
 }
 
@@ -217,7 +217,7 @@ __global__ void __launch_bounds__(256) k_resid_norm(const float* __restrict__ pa
   const float r = rsqrtf(ss / (float)H + eps);
   for (int f = threadIdx.x; f < H; f += blockDim.x) {
     const float y = xr[f] * r * to_f32(gain[f]);
-    xn[(size_t)t * H + f] = from_f32<E>(y);
+    store_act(xn, (size_t)t * H + f, (size_t)kMaxT * H, y);
     if (hidden_out) hidden_out[(size_t)t * H + f] = y;
   }
   pdl_trigger();
@@ -244,7 +244,7 @@ __global__ void __launch_bounds__(256) k_silu_mul(const float* __restrict__ part
   if (i < I) {
     const float g = gather_partial(part, plan, 2 * I, t, i);
     const float u = gather_partial(part, plan, 2 * I, t, I + i);
-    act[(size_t)t * I + i] = from_f32<E>(g / (1.f + expf(-g)) * u);
+    store_act(act, (size_t)t * I + i, (size_t)kMaxT * I, g / (1.f + expf(-g)) * u);
   }
   pdl_trigger();
 }
