@@ -336,7 +336,7 @@ def run_ours(args):
 
     step_b = step_bytes(cfg, ctx, T)
     value = world * T / (ms * 1e-3)
-    launches_per_step = 2 + cfg.n_layers * 10 + 2 + 1
+    launches_per_step = 2 + cfg.n_layers * 5 + 2 + 1   # prep, embed, 5 per layer, LM head, accept, compact
     if rank == 0:
         print(json.dumps({
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,

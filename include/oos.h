@@ -200,13 +200,14 @@ int oos_accept_walk(const int32_t* tree_tokens, const int32_t* tree_parent, cons
                     int32_t* out_accepted_tokens, int32_t* out_bonus_token, int32_t* out_status,
                     void* stream);
 
-/* Benchmarking aid: enqueue ONE weight-streaming kernel of the verify step,
- * launched exactly as oos_tree_verify launches it, on the activations the last
- * verify of this handle left in its workspace.  stage: OOS_STAGE_QKV,
- * OOS_STAGE_O, OOS_STAGE_GATE_UP, OOS_STAGE_DOWN (of layer `layer`) or
- * OOS_STAGE_LM_HEAD (layer ignored).  T as in that verify.  Writes only
- * workspace scratch (partial sums, LM-head partial maxima); the KV cache and
- * the outputs of the last verify are left as they were. */
+/* Benchmarking aid: enqueue ONE weight-streaming kernel of the verify step
+ * (with its fused epilogue), launched exactly as oos_tree_verify launches it,
+ * on whatever activations the workspace holds.  stage: OOS_STAGE_O,
+ * OOS_STAGE_GATE_UP, OOS_STAGE_DOWN (of layer `layer`) or OOS_STAGE_LM_HEAD
+ * (layer ignored); T as in the last verify.  It writes only workspace scratch,
+ * so the KV cache and the outputs of the last verify stay as they were, but
+ * the workspace no longer holds that verify's intermediates.  OOS_STAGE_QKV
+ * returns OOS_EINVAL for bf16 models: its epilogue writes the KV cache. */
 #define OOS_STAGE_QKV 0
 #define OOS_STAGE_O 1
 #define OOS_STAGE_GATE_UP 2

@@ -8,9 +8,10 @@
 // rows of one kv head -- the (node, q-head) pairs of the group, so GQA reuses
 // every K/V tile for nq/nkv heads -- and one range of cache keys; the last
 // split also takes the tree tail, masked with the 128-bit ancestor sets.  K/V
-// tiles are staged in shared memory by cp.async (double buffered); scores and
-// P.V run on the tensor cores (mma.sync m16n8k16, fp32 accumulate) with an
-// online softmax in fp32.  Splits are merged by log-sum-exp in a second kernel.
+// tiles are staged in shared memory by a 3-deep cp.async ring; scores and P.V
+// run on the tensor cores (mma.sync m16n8k16, fp32 accumulate) with an online
+// softmax in fp32.  The last split of a row block to finish merges all splits
+// by log-sum-exp (fixed split order) and writes the hi/lo bf16 GEMM input.
 //
 // fp32 path: one block per (node, head), CUDA cores (small models only).
 #include <math.h>
@@ -24,7 +25,9 @@ constexpr int kAttnRows = 64;     // query rows per block (4 warps x 16)
 constexpr int kAttnKeys = 64;     // keys per tile
 constexpr int kAttnD = 128;       // head dim of the bf16 path
 constexpr int kAttnLd = kAttnD + 8;   // padded smem row (272 bytes): conflict-free ldmatrix
-constexpr int kAttnSmem = (kAttnRows + 4 * kAttnKeys) * kAttnLd * 2;
+constexpr int kAttnStages = 3;        // cp.async ring of K/V tiles
+constexpr int kAttnStageElems = 2 * kAttnKeys * kAttnLd;   // K tile then V tile
+constexpr int kAttnSmem = kAttnStages * kAttnStageElems * 2;
 
 struct AttnArgs {
   const __nv_bfloat16* q;   // [T][nq][d]
@@ -32,10 +35,13 @@ struct AttnArgs {
   const __nv_bfloat16* vc;
   const unsigned long long* anc;
   int T, nq, nkv, group, ctx;
-  int splits, cache_blocks;
+  int splits, cache_blocks, row_blocks;
   float scale_log2;         // log2(e) / sqrt(d)
   float* o_part;            // [split][T*nq][d]
   float* ml_part;           // [split][T*nq][2]
+  int* cnt;                 // [nkv * row_blocks] split arrival counters
+  __nv_bfloat16* out;       // [T][nq*d] hi rows, lo rows at out_lo_off
+  size_t out_lo_off;
 };
 
 OOS_DEV void cp_async16(void* smem, const void* gmem, bool valid) {
@@ -82,9 +88,8 @@ OOS_DEV void load_kv_tile(__nv_bfloat16* ks, __nv_bfloat16* vs, const AttnArgs& 
 
 __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
-  __nv_bfloat16* Qs = reinterpret_cast<__nv_bfloat16*>(smem_raw);
-  __nv_bfloat16* Ks = Qs + kAttnRows * kAttnLd;          // [2][64][ld]
-  __nv_bfloat16* Vs = Ks + 2 * kAttnKeys * kAttnLd;      // [2][64][ld]
+  __nv_bfloat16* ring = reinterpret_cast<__nv_bfloat16*>(smem_raw);   // [stage][K | V][64][ld]
+  __shared__ int s_last;
   pdl_trigger();
   pdl_wait();
   const int rb = blockIdx.x, g = blockIdx.y, split = blockIdx.z;
@@ -96,15 +101,6 @@ __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
   const int cb1 = (int)((long long)(split + 1) * a.cache_blocks / a.splits);
   const int tree_tiles = (split == a.splits - 1) ? (a.T + kAttnKeys - 1) / kAttnKeys : 0;
   const int n_tiles = (cb1 - cb0) + tree_tiles;
-
-  // Q rows: row r -> node r / group, head g*group + r % group
-  for (int c = threadIdx.x; c < kAttnRows * (kAttnD / 8); c += blockDim.x) {
-    const int r = c >> 4, col = (c & 15) * 8;
-    const int row = rb * kAttnRows + r;
-    const bool valid = row < R;
-    const int node = valid ? row / a.group : 0, hq = g * a.group + (valid ? row % a.group : 0);
-    cp_async16(Qs + r * kAttnLd + col, a.q + ((size_t)node * a.nq + hq) * kAttnD + col, valid);
-  }
   auto tile_keys = [&](int ti, int& key0, int& key_end, bool& tree) {
     if (ti < cb1 - cb0) {
       key0 = (cb0 + ti) * kAttnKeys;
@@ -117,13 +113,43 @@ __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
       tree = true;
     }
   };
-  if (n_tiles > 0) {
-    int k0, ke;
-    bool tr;
-    tile_keys(0, k0, ke, tr);
-    load_kv_tile(Ks, Vs, a, g, k0, ke);
+  auto stage_k = [&](int s) { return ring + s * kAttnStageElems; };
+  auto stage_v = [&](int s) { return ring + s * kAttnStageElems + kAttnKeys * kAttnLd; };
+  auto issue = [&](int ti) {
+    if (ti < n_tiles) {
+      int k0, ke;
+      bool tr;
+      tile_keys(ti, k0, ke, tr);
+      load_kv_tile(stage_k(ti % kAttnStages), stage_v(ti % kAttnStages), a, g, k0, ke);
+    }
+    cp_async_commit();
+  };
+
+  // Q rows (row r -> node r / group, head g*group + r % group), staged through
+  // the last ring slot, then kept in registers as mma A fragments
+  {
+    __nv_bfloat16* Qs = stage_k(kAttnStages - 1);
+    for (int c = threadIdx.x; c < kAttnRows * (kAttnD / 8); c += blockDim.x) {
+      const int r = c >> 4, col = (c & 15) * 8;
+      const int row = rb * kAttnRows + r;
+      const bool valid = row < R;
+      const int node = valid ? row / a.group : 0, hq = g * a.group + (valid ? row % a.group : 0);
+      cp_async16(Qs + r * kAttnLd + col, a.q + ((size_t)node * a.nq + hq) * kAttnD + col, valid);
+    }
+    cp_async_commit();
+    cp_async_wait<0>();
+    __syncthreads();
   }
-  cp_async_commit();
+  uint32_t qf[8][4];
+#pragma unroll
+  for (int ks = 0; ks < 8; ++ks) {
+    const int row = warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
+    const int col = ks * 16 + (lane >> 4) * 8;
+    ldsm_x4(qf[ks], stage_k(kAttnStages - 1) + row * kAttnLd + col);
+  }
+  __syncthreads();
+  issue(0);
+  issue(1);
 
   // per-thread rows: r_lo = warp*16 + lane/4, r_hi = r_lo + 8
   const int r_lo = rb * kAttnRows + warp * 16 + (lane >> 2);
@@ -136,29 +162,13 @@ __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
 #pragma unroll
   for (int n = 0; n < 16; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
   float m_lo = -INFINITY, m_hi = -INFINITY, l_lo = 0.f, l_hi = 0.f;
-  uint32_t qf[8][4];
 
   for (int ti = 0; ti < n_tiles; ++ti) {
-    const int buf = ti & 1;
-    if (ti + 1 < n_tiles) {
-      int k0, ke;
-      bool tr;
-      tile_keys(ti + 1, k0, ke, tr);
-      load_kv_tile(Ks + (buf ^ 1) * kAttnKeys * kAttnLd, Vs + (buf ^ 1) * kAttnKeys * kAttnLd, a, g, k0, ke);
-    }
-    cp_async_commit();
-    cp_async_wait<1>();
+    issue(ti + 2);
+    cp_async_wait<2>();
     __syncthreads();
-    if (ti == 0) {
-#pragma unroll
-      for (int ks = 0; ks < 8; ++ks) {
-        const int row = warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
-        const int col = ks * 16 + (lane >> 4) * 8;
-        ldsm_x4(qf[ks], Qs + row * kAttnLd + col);
-      }
-    }
-    const __nv_bfloat16* kt = Ks + buf * kAttnKeys * kAttnLd;
-    const __nv_bfloat16* vt = Vs + buf * kAttnKeys * kAttnLd;
+    const __nv_bfloat16* kt = stage_k(ti % kAttnStages);
+    const __nv_bfloat16* vt = stage_v(ti % kAttnStages);
     int key0, key_end;
     bool tree;
     tile_keys(ti, key0, key_end, tree);
@@ -246,7 +256,7 @@ __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
   }
   cp_async_wait<0>();
 
-  // quad sums of l, then write unnormalised O and (m, l)
+  // quad sums of l, then this split's unnormalised O and (m, l)
 #pragma unroll
   for (int off = 1; off <= 2; off <<= 1) {
     l_lo += __shfl_xor_sync(0xffffffffu, l_lo, off);
@@ -271,26 +281,37 @@ __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
       ml[1] = half ? l_hi : l_lo;
     }
   }
-}
 
-// merge the splits of one (node, head) row: log-sum-exp weights in base 2
-__global__ void __launch_bounds__(kAttnD) k_attn_merge(const float* __restrict__ o_part, const float* __restrict__ ml,
-                                                       int splits, int rows_total, size_t rows_lo_off,
-                                                       __nv_bfloat16* __restrict__ out) {
-  pdl_trigger();
-  pdl_wait();
-  const int row = blockIdx.x, c = threadIdx.x;
-  float M = -INFINITY;
-  for (int s = 0; s < splits; ++s) M = fmaxf(M, ml[((size_t)s * rows_total + row) * 2]);
-  float num = 0.f, den = 0.f;
-  for (int s = 0; s < splits; ++s) {
-    const float ms = ml[((size_t)s * rows_total + row) * 2];
-    if (ms == -INFINITY) continue;
-    const float w = exp2f(ms - M);
-    den += w * ml[((size_t)s * rows_total + row) * 2 + 1];
-    num += w * o_part[((size_t)s * rows_total + row) * kAttnD + c];
+  // the last split of this (row block, kv head) to finish merges all splits:
+  // log-sum-exp weights in base 2, summed in split order
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    const int ci = g * a.row_blocks + rb;
+    const int old = atomicAdd(&a.cnt[ci], 1);
+    s_last = old == a.splits - 1;
+    if (s_last) a.cnt[ci] = 0;
   }
-  store_act(out, (size_t)row * kAttnD + c, (size_t)rows_lo_off, num / den);
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  for (int idx = threadIdx.x; idx < kAttnRows * kAttnD; idx += blockDim.x) {
+    const int r = rb * kAttnRows + idx / kAttnD, c = idx % kAttnD;
+    if (r >= R) break;
+    const int node = r / a.group, hq = g * a.group + r % a.group;
+    const size_t grow = (size_t)node * a.nq + hq;
+    float M = -INFINITY;
+    for (int sp = 0; sp < a.splits; ++sp) M = fmaxf(M, __ldcg(a.ml_part + ((size_t)sp * rows_total + grow) * 2));
+    float num = 0.f, den = 0.f;
+    for (int sp = 0; sp < a.splits; ++sp) {
+      const float ms = __ldcg(a.ml_part + ((size_t)sp * rows_total + grow) * 2);
+      if (ms == -INFINITY) continue;
+      const float w = exp2f(ms - M);
+      den += w * __ldcg(a.ml_part + ((size_t)sp * rows_total + grow) * 2 + 1);
+      num += w * __ldcg(a.o_part + ((size_t)sp * rows_total + grow) * kAttnD + c);
+    }
+    store_act(a.out, grow * kAttnD + c, a.out_lo_off, num / den);
+  }
 }
 
 // ------------------------------------------------------------ fp32 path
@@ -369,18 +390,19 @@ cudaError_t launch_attention(Model& m, const void* kc, const void* vc, int ctx, 
   a.cache_blocks = (ctx + kAttnKeys - 1) / kAttnKeys;
   const int R = T * a.group;
   const int RB = (R + kAttnRows - 1) / kAttnRows;
-  int splits = (2 * m.num_sms + a.nkv * RB - 1) / (a.nkv * RB);
+  a.row_blocks = RB;
+  // one wave at two blocks per SM
+  int splits = (2 * m.num_sms) / (a.nkv * RB);
   const int max_splits = a.cache_blocks > 0 ? (a.cache_blocks < kMaxAttnSplits ? a.cache_blocks : kMaxAttnSplits) : 1;
   splits = splits < 1 ? 1 : (splits > max_splits ? max_splits : splits);
   a.splits = splits;
   a.scale_log2 = 1.4426950408889634f / sqrtf((float)kAttnD);
   a.o_part = m.ws.attn_o;
   a.ml_part = m.ws.attn_ml;
-  cudaError_t e = launch(m.pdl, k_attn_tc, dim3(RB, a.nkv, splits), dim3(128), (size_t)kAttnSmem, st, a);
-  if (e != cudaSuccess) return e;
-  return launch(m.pdl, k_attn_merge, dim3(T * c.n_q_heads), dim3(kAttnD), 0, st, (const float*)m.ws.attn_o,
-                (const float*)m.ws.attn_ml, splits, T * c.n_q_heads, (size_t)kMaxT * c.n_q_heads * kAttnD,
-                (__nv_bfloat16*)m.ws.attn);
+  a.cnt = m.ws.attn_cnt;
+  a.out = (__nv_bfloat16*)m.ws.attn;
+  a.out_lo_off = (size_t)kMaxT * c.n_q_heads * kAttnD;
+  return launch(m.pdl, k_attn_tc, dim3(RB, a.nkv, splits), dim3(128), (size_t)kAttnSmem, st, a);
 }
 
 }  // namespace oos

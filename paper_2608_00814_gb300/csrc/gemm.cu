@@ -8,9 +8,9 @@
 // S-stage shared-memory ring; one thread issues tcgen05.mma into a TMEM
 // accumulator (two buffers, so the epilogue of one tile overlaps the MMAs of
 // the next); four epilogue warps drain TMEM with tcgen05.ld.
-//   MODE_PARTIAL: stream-K over (tile, k-block) units, fp32 partial tiles out.
-//   MODE_ARGMAX : LM head, whole tiles round-robin, per-node running
-//                 (max, argmax, second max) -- logits never reach memory.
+// The layer's elementwise steps run in the GEMM epilogues (see below); the LM
+// head keeps a per-node running (max, argmax, second max) so logits never
+// reach memory.
 //
 // fp32 path: CUDA-core warp-per-row GEMV kernels (small models only).
 #include <string.h>
@@ -20,18 +20,56 @@
 
 namespace oos {
 
-enum { MODE_PARTIAL = 0, MODE_ARGMAX = 1 };
+// Epilogues fused into the weight GEMMs (bf16 path).  Stream-K leaves a tile's
+// reduction split over up to a few CTAs: each writes its fp32 partial tile,
+// and the LAST contributor to arrive (a per-tile arrival counter) adds the
+// slices in slice order -- a fixed order, so results are deterministic -- and
+// applies the layer's elementwise step to the finished tile:
+//   EPI_QKV   : input RMSNorm scale, bias, per-head q/k RMSNorm, RoPE at
+//               ctx + depth; q to the query buffer, k/v to cache slot ctx + t.
+//   EPI_RESID : x += W.a (O- and down-projections), then y = g (.) x for the
+//               next RMSNorm (hi/lo bf16) and per-tile sums of x^2.
+//   EPI_SILU  : gate and up tiles are interleaved (tile 2i = gate rows of
+//               block i, 2i+1 = up rows); act = silu(r g) * (r u).
+//   EPI_ARGMAX: LM head -- whole tiles round-robin, logits scaled by the final
+//               RMSNorm factor and folded into a per-node running top-2.
+// RMSNorm is split across kernels by linearity: a producer stores y = g (.) x
+// and sum(x^2) per 128-feature chunk; the consumer GEMM computes W.y and
+// multiplies column t by r_t = rsqrt(sum x_t^2 / H + eps) in its epilogue.
+enum { EPI_QKV = 0, EPI_RESID = 1, EPI_SILU = 2, EPI_ARGMAX = 3 };
 
 struct GemmArgs {
   int seg_tiles[3];   // cumulative tile counts per weight segment
+  int interleave2;    // tile 2i -> segment 0 block i, tile 2i+1 -> segment 1 block i
   int n_tiles, kbt, total;
-  int N;              // output rows (features / vocab)
+  int N;              // output rows (features / vocab) of the stacked weight
   int T;              // valid columns (tree nodes)
-  float* part;        // MODE_PARTIAL: [slice][kMaxT][N]
-  float* am_v1;       // MODE_ARGMAX: [cta][kMaxT]
+  float* part;        // partial tiles [slice][kMaxT][n_tiles * 128]
+  int* cnt;           // arrival counters (per tile, per gate/up pair); zero between launches
+  uint32_t* status;
+  // RMSNorm scale of the GEMM input (EPI_QKV, EPI_SILU, EPI_ARGMAX)
+  const float* ss_in;   // [chunk][kMaxT]
+  int ss_chunks;
+  float inv_dim, eps;
+  // EPI_QKV
+  int nq, nkv;
+  const __nv_bfloat16 *bq, *bk, *bv, *gq, *gk;
+  const int32_t* pos;
+  const double* inv_freq;
+  __nv_bfloat16 *q_out, *kc, *vc;
+  int ctx;
+  // EPI_RESID
+  float* x;
+  const __nv_bfloat16* gain;
+  __nv_bfloat16* y_out;
+  float* ss_out;
+  // EPI_SILU
+  __nv_bfloat16* act_out;
+  int I;
+  // EPI_ARGMAX
+  float* am_v1;
   int32_t* am_i;
   float* am_v2;
-  uint32_t* status;
 };
 
 template <int BN>
@@ -42,9 +80,10 @@ struct TcCfg {
   static constexpr int S_RAW = (200 * 1024) / STAGE;
   static constexpr int S = S_RAW > 8 ? 8 : S_RAW;
   static constexpr int NCOLS = (2 * BN) < 32 ? 32 : 2 * BN;    // two accumulators, power of two
-  static constexpr int BAR_BYTES = 1024;
+  static constexpr int BAR_BYTES = 256;
+  static constexpr int EPI_BYTES = 4 * kMaxT * 4 + kMaxT * 4 + 64;   // column sums, rms, flags
   static constexpr int RED_BYTES = 4 * BN * 12 + BN * 12;      // argmax cross-warp scratch + running state
-  static constexpr int SMEM = 1024 /*align slack*/ + S * STAGE + BAR_BYTES + RED_BYTES;
+  static constexpr int SMEM = 1024 /*align slack*/ + S * STAGE + BAR_BYTES + EPI_BYTES + RED_BYTES;
 };
 
 struct Top2s {
@@ -65,12 +104,115 @@ OOS_DEV Top2s t2_merge(Top2s a, Top2s b) {
   return r;
 }
 
-template <int BN, int MODE>
+OOS_DEV void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
+
+// sum of the stream-K slices of element (t, n) of a partial tile
+OOS_DEV float slice_sum(const float* part, int nc, size_t slice, size_t idx) {
+  float v = 0.f;
+  for (int s = 0; s < nc; ++s) v += __ldcg(part + (size_t)s * slice + idx);
+  return v;
+}
+
+template <int EPI>
+OOS_DEV void finish_tile(const GemmArgs& a, int tile, const float* rms, float* col_red, float* pair_red) {
+  const int e = threadIdx.x - 64;     // 0..127
+  const int warp = e >> 5, lane = e & 31;
+  const int n_part = a.n_tiles * kTile;
+  const size_t slice = (size_t)kMaxT * n_part;
+  StreamK sk{a.n_tiles, a.kbt, a.total, (int)gridDim.x};
+  int c0, c1;
+  if (EPI == EPI_RESID) {
+    sk.contributors(tile, c0, c1);
+    const int nc = c1 - c0 + 1;
+    const int f = tile * kTile + e;
+    const bool fv = f < a.N;
+    const float g = fv ? __bfloat162float(a.gain[f]) : 0.f;
+    for (int t = 0; t < a.T; ++t) {
+      float sq = 0.f;
+      if (fv) {
+        const float xv = a.x[(size_t)t * a.N + f] + slice_sum(a.part, nc, slice, (size_t)t * n_part + f);
+        a.x[(size_t)t * a.N + f] = xv;
+        store_act(a.y_out, (size_t)t * a.N + f, (size_t)kMaxT * a.N, g * xv);
+        sq = xv * xv;
+      }
+      sq = warp_sum(sq);
+      if (lane == 0) col_red[warp * kMaxT + t] = sq;
+    }
+    epi_bar();
+    if (e < a.T) a.ss_out[(size_t)tile * kMaxT + e] = col_red[e] + col_red[kMaxT + e] + col_red[2 * kMaxT + e] + col_red[3 * kMaxT + e];
+    epi_bar();
+  } else if (EPI == EPI_SILU) {
+    int g0, g1, u0, u1;
+    sk.contributors(2 * (tile >> 1), g0, g1);
+    sk.contributors(2 * (tile >> 1) + 1, u0, u1);
+    const int i = (tile >> 1) * kTile + e;        // feature of the SwiGLU output
+    if (i < a.I) {
+      const int fg = 2 * (tile >> 1) * kTile + e, fu = fg + kTile;
+      for (int t = 0; t < a.T; ++t) {
+        const float gv = slice_sum(a.part, g1 - g0 + 1, slice, (size_t)t * n_part + fg) * rms[t];
+        const float uv = slice_sum(a.part, u1 - u0 + 1, slice, (size_t)t * n_part + fu) * rms[t];
+        store_act(a.act_out, (size_t)t * a.I + i, (size_t)kMaxT * a.I, gv / (1.f + expf(-gv)) * uv);
+      }
+    }
+  } else {  // EPI_QKV: tile = one head of 128 features (q heads, then k heads, then v heads)
+    sk.contributors(tile, c0, c1);
+    const int nc = c1 - c0 + 1;
+    int kind, h;
+    if (tile < a.nq) { kind = 0; h = tile; }
+    else if (tile < a.nq + a.nkv) { kind = 1; h = tile - a.nq; }
+    else { kind = 2; h = tile - a.nq - a.nkv; }
+    const __nv_bfloat16* bias = kind == 0 ? a.bq : kind == 1 ? a.bk : a.bv;
+    const __nv_bfloat16* gn = kind == 0 ? a.gq : kind == 1 ? a.gk : nullptr;
+    const int j = e & 63;
+    const double two_pi = 6.283185307179586476925286766559;
+    for (int t0 = 0; t0 < a.T; t0 += 2) {
+      const int t = t0 + (e >> 6);
+      const bool tv = t < a.T;
+      float v0 = 0.f, v1 = 0.f;
+      if (tv) {
+        const size_t base = (size_t)t * n_part + (size_t)tile * kTile + j;
+        v0 = slice_sum(a.part, nc, slice, base) * rms[t];
+        v1 = slice_sum(a.part, nc, slice, base + 64) * rms[t];
+        if (bias) {
+          v0 += __bfloat162float(bias[h * kTile + j]);
+          v1 += __bfloat162float(bias[h * kTile + j + 64]);
+        }
+      }
+      if (gn) {   // per-head RMSNorm over the 128 features of this token
+        const float ss = warp_sum(v0 * v0 + v1 * v1);
+        if (lane == 0) pair_red[warp] = ss;
+        epi_bar();
+        const float tot = pair_red[warp & 2] + pair_red[(warp & 2) + 1];
+        epi_bar();
+        const float r = rsqrtf(tot * (1.f / kTile) + a.eps);
+        v0 = v0 * r * __bfloat162float(gn[j]);
+        v1 = v1 * r * __bfloat162float(gn[j + 64]);
+      }
+      if (!tv) continue;
+      if (kind < 2) {   // rotate-half RoPE at position ctx + depth(t)
+        const double ang = (double)a.pos[t] * a.inv_freq[j];
+        const float ra = (float)(ang - two_pi * rint(ang / two_pi));
+        float sn, cs;
+        sincosf(ra, &sn, &cs);
+        const float o0 = v0 * cs - v1 * sn, o1 = v1 * cs + v0 * sn;
+        v0 = o0;
+        v1 = o1;
+      }
+      __nv_bfloat16* dst = kind == 0 ? a.q_out + ((size_t)t * a.nq + h) * kTile
+                                     : (kind == 1 ? a.kc : a.vc) + ((size_t)(a.ctx + t) * a.nkv + h) * kTile;
+      dst[j] = __float2bfloat16_rn(v0);
+      dst[j + 64] = __float2bfloat16_rn(v1);
+    }
+  }
+}
+
+template <int BN, int EPI>
 __global__ void __launch_bounds__(192, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap wm0, const __grid_constant__ CUtensorMap wm1,
               const __grid_constant__ CUtensorMap wm2, const __grid_constant__ CUtensorMap am, GemmArgs a) {
   using C = TcCfg<BN>;
   constexpr int S = C::S;
+  constexpr bool ARGMAX = EPI == EPI_ARGMAX;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   unsigned char* sA = smem;
@@ -82,15 +224,19 @@ __global__ void __launch_bounds__(192, 1)
   uint64_t* drain = acce + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  Top2s* red = reinterpret_cast<Top2s*>(smem + S * C::STAGE + C::BAR_BYTES);   // [4][BN]
-  Top2s* run = red + 4 * BN;                                                    // [BN]
+  float* col_red = reinterpret_cast<float*>(smem + S * C::STAGE + C::BAR_BYTES);   // [4][kMaxT]
+  float* rms = col_red + 4 * kMaxT;                                                 // [kMaxT]
+  float* pair_red = rms + kMaxT;                                                    // [4]
+  volatile int* s_last = reinterpret_cast<volatile int*>(pair_red + 4);
+  Top2s* red = reinterpret_cast<Top2s*>(smem + S * C::STAGE + C::BAR_BYTES + C::EPI_BYTES);   // [4][BN]
+  Top2s* run = red + 4 * BN;                                                                   // [BN]
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = gridDim.x, cta = blockIdx.x;
 
-  // this CTA's work: units [u0, u1) (stream-K) or tiles cta, cta+G, ... (argmax)
+  // this CTA's work: units [u0, u1) (stream-K) or tiles cta, cta+G, ... (LM head)
   long long u0, u1;
-  if (MODE == MODE_PARTIAL) {
+  if (!ARGMAX) {
     u0 = (long long)cta * a.total / G;
     u1 = (long long)(cta + 1) * a.total / G;
   } else {
@@ -100,7 +246,7 @@ __global__ void __launch_bounds__(192, 1)
   }
   const int n_units = (int)(u1 - u0);
   auto unit_tile = [&](int j, int& tile, int& kb) {
-    if (MODE == MODE_PARTIAL) {
+    if (!ARGMAX) {
       const long long u = u0 + j;
       tile = (int)(u / a.kbt);
       kb = (int)(u % a.kbt);
@@ -124,13 +270,14 @@ __global__ void __launch_bounds__(192, 1)
     mbar_fence_init();
   }
   if (warp == 2) tmem_alloc(tmem_slot, C::NCOLS);
-  if (MODE == MODE_ARGMAX && threadIdx.x >= 64) {
+  if (ARGMAX && threadIdx.x >= 64) {
     for (int e = threadIdx.x - 64; e < BN; e += 128) run[e] = Top2s{-INFINITY, 0x7fffffff, -INFINITY};
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
+  pdl_trigger();
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
@@ -144,7 +291,10 @@ __global__ void __launch_bounds__(192, 1)
         unit_tile(j, tile, kb);
         const CUtensorMap* wm = &wm0;
         int row = tile * kTile;
-        if (tile >= a.seg_tiles[0]) {
+        if (a.interleave2) {
+          wm = (tile & 1) ? &wm1 : &wm0;
+          row = (tile >> 1) * kTile;
+        } else if (tile >= a.seg_tiles[0]) {
           if (tile >= a.seg_tiles[1]) {
             wm = &wm2;
             row = (tile - a.seg_tiles[1]) * kTile;
@@ -197,7 +347,6 @@ __global__ void __launch_bounds__(192, 1)
     }
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
-    pdl_wait();
     if (lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(kTile, BN);
       int stage = 0;
@@ -252,6 +401,15 @@ __global__ void __launch_bounds__(192, 1)
     const int q = warp & 3;               // TMEM lane quarter this warp may access
     const int row = q * 32 + lane;
     const int e = threadIdx.x - 64;       // 0..127
+    if (EPI != EPI_RESID) {
+      if (e < a.T) {
+        float s = 0.f;
+        for (int c = 0; c < a.ss_chunks; ++c) s += a.ss_in[(size_t)c * kMaxT + e];
+        rms[e] = rsqrtf(s * a.inv_dim + a.eps);
+      }
+      epi_bar();
+    }
+    const int n_part = a.n_tiles * kTile;
     int acc = 0;
     uint32_t acc_use[2] = {0, 0};
     int j = 0;
@@ -263,26 +421,11 @@ __global__ void __launch_bounds__(192, 1)
       if (!mbar_wait(&accf[acc], acc_use[acc] & 1u, abort_flag, a.status)) break;
       tc_fence_after();
       const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
-      const int f = tile * kTile + row;
-      if (MODE == MODE_PARTIAL) {
+      if (!ARGMAX) {
         int c0, c1;
         StreamK sk{a.n_tiles, a.kbt, a.total, G};
         sk.contributors(tile, c0, c1);
-        float* dst = a.part + (size_t)(cta - c0) * kMaxT * a.N + f;
-#pragma unroll 1
-        for (int cc = 0; cc < BN / 16; ++cc) {
-          if (cc * 16 >= a.T) break;
-          float v[16];
-          tmem_ld16(taddr + cc * 16, v);
-          if (f < a.N) {
-#pragma unroll
-            for (int i = 0; i < 16; ++i) {
-              const int t = cc * 16 + i;
-              if (t < a.T) dst[(size_t)t * a.N] = v[i];
-            }
-          }
-        }
-      } else {
+        float* dst = a.part + (size_t)(cta - c0) * kMaxT * n_part + (size_t)tile * kTile + row;
 #pragma unroll 1
         for (int cc = 0; cc < BN / 16; ++cc) {
           if (cc * 16 >= a.T) break;
@@ -290,7 +433,46 @@ __global__ void __launch_bounds__(192, 1)
           tmem_ld16(taddr + cc * 16, v);
 #pragma unroll
           for (int i = 0; i < 16; ++i) {
-            Top2s s{f < a.N ? v[i] : -INFINITY, f, -INFINITY};
+            const int t = cc * 16 + i;
+            if (t < a.T) dst[(size_t)t * n_part] = v[i];
+          }
+        }
+        // accumulator drained: hand the TMEM buffer back to the MMA issuer
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&acce[acc]);
+        // arrival: the last contributor of the tile (or gate/up pair) finishes it
+        __threadfence();
+        epi_bar();
+        if (e == 0) {
+          int expected = c1 - c0 + 1;
+          int ci = tile;
+          if (EPI == EPI_SILU) {
+            int o0, o1;
+            sk.contributors(tile ^ 1, o0, o1);
+            expected += o1 - o0 + 1;
+            ci = tile >> 1;
+          }
+          const int old = atomicAdd(&a.cnt[ci], 1);
+          *s_last = (old == expected - 1);
+          if (old == expected - 1) a.cnt[ci] = 0;   // ready for the next launch
+        }
+        epi_bar();
+        if (*s_last) {
+          __threadfence();
+          finish_tile<EPI>(a, tile, rms, col_red, pair_red);
+        }
+        epi_bar();
+      } else {
+        const int f = tile * kTile + row;
+#pragma unroll 1
+        for (int cc = 0; cc < BN / 16; ++cc) {
+          if (cc * 16 >= a.T) break;
+          float v[16];
+          tmem_ld16(taddr + cc * 16, v);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) {
+            Top2s s{f < a.N ? v[i] * rms[cc * 16 + i] : -INFINITY, f, -INFINITY};
 #pragma unroll
             for (int o = 16; o > 0; o >>= 1) {
               Top2s y;
@@ -302,30 +484,29 @@ __global__ void __launch_bounds__(192, 1)
             if (lane == 0) red[q * BN + cc * 16 + i] = s;
           }
         }
-        asm volatile("bar.sync 1, 128;" ::: "memory");
+        tc_fence_before();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(&acce[acc]);
+        epi_bar();
         if (e < a.T) {
           Top2s r = run[e];
 #pragma unroll
           for (int w = 0; w < 4; ++w) r = t2_merge(r, red[w * BN + e]);
           run[e] = r;
         }
-        asm volatile("bar.sync 1, 128;" ::: "memory");
+        epi_bar();
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&acce[acc]);
       ++acc_use[acc];
       acc ^= 1;
       j = seg_end;
     }
-    if (MODE == MODE_ARGMAX && e < a.T) {
+    if (ARGMAX && e < a.T) {
       const Top2s r = run[e];
       a.am_v1[(size_t)cta * kMaxT + e] = r.v1;
       a.am_i[(size_t)cta * kMaxT + e] = r.i1;
       a.am_v2[(size_t)cta * kMaxT + e] = r.v2;
     }
   }
-  pdl_trigger();
   tc_fence_before();
   __syncthreads();
   if (warp == 2) {
@@ -375,67 +556,121 @@ bool encode_act_map(CUtensorMap* map, const void* ptr, int K, int box_rows) {
 
 int bn_index(int T) { return T <= 16 ? 0 : T <= 32 ? 1 : T <= 64 ? 2 : 3; }
 
-template <int BN, int MODE>
+template <int BN, int EPI>
 static cudaError_t set_smem() {
-  return cudaFuncSetAttribute(k_gemm_tc<BN, MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<BN>::SMEM);
+  return cudaFuncSetAttribute(k_gemm_tc<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<BN>::SMEM);
 }
 
-cudaError_t gemm_setup() {
-  cudaError_t e = cudaSuccess;
-  cudaError_t r;
-#define OOS_SET(BN)                                       \
-  if ((r = set_smem<BN, MODE_PARTIAL>()) != cudaSuccess) e = r; \
-  if ((r = set_smem<BN, MODE_ARGMAX>()) != cudaSuccess) e = r;
-  OOS_SET(16) OOS_SET(32) OOS_SET(64) OOS_SET(128)
-#undef OOS_SET
+template <int BN>
+static cudaError_t set_smem_all() {
+  cudaError_t e = set_smem<BN, EPI_QKV>();
+  if (e == cudaSuccess) e = set_smem<BN, EPI_RESID>();
+  if (e == cudaSuccess) e = set_smem<BN, EPI_SILU>();
+  if (e == cudaSuccess) e = set_smem<BN, EPI_ARGMAX>();
   return e;
 }
 
-template <int BN, int MODE>
-static cudaError_t launch_tc(Model& m, const GemmW& g, const CUtensorMap& amap, int T, int grid, GemmArgs& a,
+cudaError_t gemm_setup() {
+  cudaError_t e = set_smem_all<16>();
+  if (e == cudaSuccess) e = set_smem_all<32>();
+  if (e == cudaSuccess) e = set_smem_all<64>();
+  if (e == cudaSuccess) e = set_smem_all<128>();
+  return e;
+}
+
+template <int BN, int EPI>
+static cudaError_t launch_tc(Model& m, const GemmW& g, const CUtensorMap& amap, int grid, const GemmArgs& a,
                              cudaStream_t st) {
   const CUtensorMap& w1 = g.n_seg > 1 ? g.map[1] : g.map[0];
   const CUtensorMap& w2 = g.n_seg > 2 ? g.map[2] : g.map[0];
-  return launch(m.pdl, k_gemm_tc<BN, MODE>, dim3(grid), dim3(192), (size_t)TcCfg<BN>::SMEM, st, g.map[0], w1, w2,
+  return launch(m.pdl, k_gemm_tc<BN, EPI>, dim3(grid), dim3(192), (size_t)TcCfg<BN>::SMEM, st, g.map[0], w1, w2,
                 amap, a);
 }
 
-template <int MODE>
-static cudaError_t dispatch_tc(Model& m, const GemmW& g, const CUtensorMap& amap, int T, int grid, GemmArgs& a,
+template <int EPI>
+static cudaError_t dispatch_tc(Model& m, const GemmW& g, const CUtensorMap* amaps, int T, int grid, const GemmArgs& a,
                                cudaStream_t st) {
-  switch (bn_index(T)) {
-    case 0: return launch_tc<16, MODE>(m, g, amap, T, grid, a, st);
-    case 1: return launch_tc<32, MODE>(m, g, amap, T, grid, a, st);
-    case 2: return launch_tc<64, MODE>(m, g, amap, T, grid, a, st);
-    default: return launch_tc<128, MODE>(m, g, amap, T, grid, a, st);
+  const int bi = bn_index(T);
+  switch (bi) {
+    case 0: return launch_tc<16, EPI>(m, g, amaps[0], grid, a, st);
+    case 1: return launch_tc<32, EPI>(m, g, amaps[1], grid, a, st);
+    case 2: return launch_tc<64, EPI>(m, g, amaps[2], grid, a, st);
+    default: return launch_tc<128, EPI>(m, g, amaps[3], grid, a, st);
   }
 }
 
-static GemmArgs base_args(Model& m, const GemmW& g, int T) {
+static GemmArgs base_args(Model& m, const GemmW& g, int T, int* cnt) {
   GemmArgs a;
   memset(&a, 0, sizeof(a));
   for (int s = 0; s < 3; ++s) a.seg_tiles[s] = g.seg_tiles[s < g.n_seg ? s : g.n_seg - 1];
+  a.interleave2 = g.interleave2;
   a.n_tiles = g.plan.n_tiles;
   a.kbt = g.plan.kbt;
   a.total = g.plan.total;
   a.N = g.N;
   a.T = T;
+  a.part = m.ws.part;
+  a.cnt = cnt;
   a.status = m.ws.status;
+  a.ss_in = m.ws.ss;
+  a.ss_chunks = (m.cfg.hidden + kTile - 1) / kTile;
+  a.inv_dim = 1.0f / (float)m.cfg.hidden;
+  a.eps = m.cfg.rms_eps;
   return a;
 }
 
-cudaError_t launch_gemm_tc(Model& m, const GemmW& g, const CUtensorMap& amap, int T, cudaStream_t st) {
-  GemmArgs a = base_args(m, g, T);
-  a.part = m.ws.part;
-  return dispatch_tc<MODE_PARTIAL>(m, g, amap, T, g.plan.grid, a, st);
+cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int ctx, int T, cudaStream_t st) {
+  const auto& c = m.cfg;
+  const oos_layer_weights& L = m.layers[layer];
+  GemmArgs a = base_args(m, m.g_qkv[layer], T, m.ws.cnt + 0 * kCntStride);
+  a.nq = c.n_q_heads;
+  a.nkv = c.n_kv_heads;
+  a.bq = (const __nv_bfloat16*)(c.qkv_bias ? L.b_q : nullptr);
+  a.bk = (const __nv_bfloat16*)(c.qkv_bias ? L.b_k : nullptr);
+  a.bv = (const __nv_bfloat16*)(c.qkv_bias ? L.b_v : nullptr);
+  a.gq = (const __nv_bfloat16*)(c.qk_norm ? L.q_norm : nullptr);
+  a.gk = (const __nv_bfloat16*)(c.qk_norm ? L.k_norm : nullptr);
+  a.pos = m.ws.pos;
+  a.inv_freq = m.ws.inv_freq;
+  a.q_out = (__nv_bfloat16*)m.ws.q;
+  a.kc = (__nv_bfloat16*)kc;
+  a.vc = (__nv_bfloat16*)vc;
+  a.ctx = ctx;
+  return dispatch_tc<EPI_QKV>(m, m.g_qkv[layer], m.amap_xn, T, m.g_qkv[layer].plan.grid, a, st);
+}
+
+static cudaError_t launch_resid(Model& m, const GemmW& g, const CUtensorMap* amaps, const void* gain, int* cnt, int T,
+                                cudaStream_t st) {
+  GemmArgs a = base_args(m, g, T, cnt);
+  a.x = m.ws.x;
+  a.gain = (const __nv_bfloat16*)gain;
+  a.y_out = (__nv_bfloat16*)m.ws.xn;
+  a.ss_out = m.ws.ss;
+  return dispatch_tc<EPI_RESID>(m, g, amaps, T, g.plan.grid, a, st);
+}
+
+cudaError_t launch_gemm_o(Model& m, int layer, int T, cudaStream_t st) {
+  return launch_resid(m, m.g_o[layer], m.amap_attn, m.layers[layer].mlp_norm, m.ws.cnt + 1 * kCntStride, T, st);
+}
+
+cudaError_t launch_gemm_down(Model& m, int layer, int T, cudaStream_t st) {
+  const void* gain = layer + 1 < m.cfg.n_layers ? m.layers[layer + 1].attn_norm : m.w.final_norm;
+  return launch_resid(m, m.g_down[layer], m.amap_act, gain, m.ws.cnt + 3 * kCntStride, T, st);
+}
+
+cudaError_t launch_gemm_gu(Model& m, int layer, int T, cudaStream_t st) {
+  GemmArgs a = base_args(m, m.g_gu[layer], T, m.ws.cnt + 2 * kCntStride);
+  a.act_out = (__nv_bfloat16*)m.ws.act;
+  a.I = m.cfg.intermediate;
+  return dispatch_tc<EPI_SILU>(m, m.g_gu[layer], m.amap_xn, T, m.g_gu[layer].plan.grid, a, st);
 }
 
 cudaError_t launch_lm_head_tc(Model& m, int T, cudaStream_t st) {
-  GemmArgs a = base_args(m, m.g_lm, T);
+  GemmArgs a = base_args(m, m.g_lm, T, nullptr);
   a.am_v1 = m.ws.lm_v1;
   a.am_i = m.ws.lm_i;
   a.am_v2 = m.ws.lm_v2;
-  return dispatch_tc<MODE_ARGMAX>(m, m.g_lm, m.amap_xn[bn_index(T)], T, m.lm_grid, a, st);
+  return dispatch_tc<EPI_ARGMAX>(m, m.g_lm, m.amap_xn, T, m.lm_grid, a, st);
 }
 
 // ------------------------------------------------------------ fp32 CUDA-core path
@@ -443,6 +678,7 @@ cudaError_t launch_lm_head_tc(Model& m, int T, cudaStream_t st) {
 __global__ void __launch_bounds__(128) k_gemm_f32(const float* __restrict__ w0, const float* __restrict__ w1,
                                                   const float* __restrict__ w2, int r0, int r1, int r2, int K,
                                                   const float* __restrict__ x, int T, float* __restrict__ part) {
+  pdl_trigger();
   pdl_wait();
   const int N = r0 + r1 + r2;
   const int f = blockIdx.x * 4 + (threadIdx.x >> 5);
@@ -457,7 +693,6 @@ __global__ void __launch_bounds__(128) k_gemm_f32(const float* __restrict__ w0, 
       if (lane == 0) part[(size_t)t * N + f] = acc;
     }
   }
-  pdl_trigger();
 }
 
 cudaError_t launch_gemm_f32(Model& m, const void* w0, const void* w1, const void* w2, int rows0, int rows1, int rows2,
@@ -473,6 +708,7 @@ __global__ void __launch_bounds__(128) k_lm_head_f32(const float* __restrict__ W
                                                      const float* __restrict__ x, int T, float* am_v1, int32_t* am_i,
                                                      float* am_v2) {
   __shared__ Top2s st[4][kMaxT];
+  pdl_trigger();
   pdl_wait();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int t = lane; t < T; t += 32) st[warp][t] = Top2s{-INFINITY, 0x7fffffff, -INFINITY};
@@ -496,7 +732,6 @@ __global__ void __launch_bounds__(128) k_lm_head_f32(const float* __restrict__ W
     am_i[(size_t)blockIdx.x * kMaxT + t] = r.i1;
     am_v2[(size_t)blockIdx.x * kMaxT + t] = r.v2;
   }
-  pdl_trigger();
 }
 
 cudaError_t launch_lm_head_f32(Model& m, int T, cudaStream_t st) {

@@ -17,7 +17,10 @@ constexpr int kTile = 128;          // output features per GEMM tile (tcgen05 M)
 constexpr int kBK = 64;             // reduction elements per pipeline stage (128 bytes of bf16)
 constexpr int kMaxLayers = 128;
 constexpr int kMaxAttnSplits = 16;  // cache splits of the attention kernel
+constexpr int kAttnCnt = 4096;      // attention arrival counters (kv heads x row blocks)
 constexpr int kMaxGridCTAs = 1024;  // upper bound on CTAs of a stream-K GEMM / LM head
+constexpr int kMaxSsChunks = 64;    // hidden <= 8192: RMSNorm partial sums per 128 features
+constexpr int kCntStride = 1024;    // arrival counters per GEMM kind (tiles or gate/up pairs)
 
 // Stream-K partition of a weight GEMM: the (tile, k-block) units of all tiles,
 // tile-major, are cut into `grid` contiguous equal ranges, one per CTA.  CTA c
@@ -58,6 +61,7 @@ struct GemmW {
   const void* ptr[3];
   int seg_tiles[3];   // cumulative tile counts at the end of each segment
   int n_seg;
+  int interleave2;    // gate/up: tiles alternate between the two segments
   int N, K;
   StreamK plan;
 };
@@ -83,6 +87,9 @@ struct Workspace {
   int32_t* argmax;           // [kMaxT]
   float* top1;
   float* top2;
+  float* ss;                 // sum of x^2 per 128-feature chunk [kMaxSsChunks][kMaxT] (bf16 path)
+  int* cnt;                  // GEMM arrival counters [4][kCntStride]
+  int* attn_cnt;             // attention split arrival counters [kAttnCnt]
 };
 
 // shape + addresses a captured verify graph was recorded with
@@ -144,6 +151,8 @@ inline cudaError_t launch(bool pdl, void (*kernel)(KArgs...), dim3 grid, dim3 bl
 cudaError_t launch_tree_prep(Model& m, const int32_t* tokens, const int32_t* parent, int T, int ctx,
                              cudaStream_t st);
 cudaError_t launch_embed_norm(Model& m, const int32_t* tokens, int T, cudaStream_t st);
+cudaError_t launch_embed_tc(Model& m, const int32_t* tokens, int T, cudaStream_t st);
+cudaError_t launch_final_hidden(Model& m, float* hidden, int T, cudaStream_t st);
 cudaError_t launch_qkv_post(Model& m, int layer, const StreamK& plan, void* kc, void* vc, int ctx, int T,
                             cudaStream_t st);
 cudaError_t launch_resid_norm(Model& m, const StreamK& plan, const void* gain, float* hidden_out, int T,
@@ -164,7 +173,10 @@ bool encode_weight_map(CUtensorMap* map, const void* ptr, int rows, int K);
 bool encode_act_map(CUtensorMap* map, const void* ptr, int K, int box_rows);
 int bn_index(int T);   // N-tile variant for T tree nodes: 0..3 -> 16/32/64/128
 cudaError_t gemm_setup();
-cudaError_t launch_gemm_tc(Model& m, const GemmW& g, const CUtensorMap& amap, int T, cudaStream_t st);
+cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int ctx, int T, cudaStream_t st);
+cudaError_t launch_gemm_o(Model& m, int layer, int T, cudaStream_t st);
+cudaError_t launch_gemm_gu(Model& m, int layer, int T, cudaStream_t st);
+cudaError_t launch_gemm_down(Model& m, int layer, int T, cudaStream_t st);
 cudaError_t launch_lm_head_tc(Model& m, int T, cudaStream_t st);
 cudaError_t launch_gemm_f32(Model& m, const void* w0, const void* w1, const void* w2, int rows0, int rows1,
                             int rows2, int K, const void* x, int T, cudaStream_t st);

@@ -67,8 +67,7 @@ size_t carve_workspace(const oos_model_config& c, int n_sms, uint8_t* base, Work
   if (c.dtype == OOS_DTYPE_BF16) {
     const StreamK ps[4] = {make_streamk(Nq, (int)H, n_sms), make_streamk((int)H, (int)qd, n_sms),
                            make_streamk((int)(2 * I), (int)H, n_sms), make_streamk((int)H, (int)I, n_sms)};
-    const size_t Ns[4] = {(size_t)Nq, H, 2 * I, H};
-    for (int i = 0; i < 4; ++i) pf = std::max(pf, (size_t)ps[i].max_slices() * kMaxT * Ns[i]);
+    for (int i = 0; i < 4; ++i) pf = std::max(pf, (size_t)ps[i].max_slices() * kMaxT * ps[i].n_tiles * kTile);
   } else {
     pf = (size_t)kMaxT * std::max(std::max((size_t)Nq, H), 2 * I);
   }
@@ -86,6 +85,9 @@ size_t carve_workspace(const oos_model_config& c, int n_sms, uint8_t* base, Work
   w.argmax = (int32_t*)take(kMaxT * 4);
   w.top1 = (float*)take(kMaxT * 4);
   w.top2 = (float*)take(kMaxT * 4);
+  w.ss = (float*)take((size_t)kMaxSsChunks * kMaxT * 4);
+  w.cnt = (int*)take((size_t)4 * kCntStride * 4);
+  w.attn_cnt = (int*)take((size_t)kAttnCnt * 4);
   if (ws) *ws = w;
   return align_up(off, 256);
 }
@@ -103,8 +105,13 @@ static bool config_ok(const oos_model_config* c) {
 }
 
 static bool shape_supported(const oos_model_config* c) {
-  if (c->dtype == OOS_DTYPE_BF16)
-    return c->head_dim == 128 && c->hidden % 128 == 0 && c->intermediate % 128 == 0;
+  if (c->dtype == OOS_DTYPE_BF16) {
+    if (c->head_dim != 128 || c->hidden % 128 || c->intermediate % 128) return false;
+    if (c->hidden / 128 > kMaxSsChunks) return false;
+    if (2 * c->intermediate / 128 > kCntStride || (c->n_q_heads + 2 * c->n_kv_heads) > kCntStride) return false;
+    const int rb = (kMaxT * (c->n_q_heads / c->n_kv_heads) + 63) / 64;
+    if (c->n_kv_heads * rb > kAttnCnt) return false;
+  }
   return true;
 }
 
@@ -140,22 +147,19 @@ static int enqueue_verify(Model& m, const oos_kv_cache* kv, int ctx, const int32
   const int L = c.n_layers;
   const int qd = c.n_q_heads * c.head_dim, kvd = c.n_kv_heads * c.head_dim;
   OOS_TRY(launch_tree_prep(m, tokens, parent, T, ctx, st));
-  OOS_TRY(launch_embed_norm(m, tokens, T, st));
-  const int bi = bn_index(T);
+  if (c.dtype == OOS_DTYPE_BF16) OOS_TRY(launch_embed_tc(m, tokens, T, st));
+  else OOS_TRY(launch_embed_norm(m, tokens, T, st));
   for (int l = 0; l < L; ++l) {
     const oos_layer_weights& W = m.layers[l];
     const void* next_gain = (l + 1 < L) ? m.layers[l + 1].attn_norm : m.w.final_norm;
     float* hid = (l + 1 < L) ? nullptr : hidden;
     if (c.dtype == OOS_DTYPE_BF16) {
-      OOS_TRY(launch_gemm_tc(m, m.g_qkv[l], m.amap_xn[bi], T, st));
-      OOS_TRY(launch_qkv_post(m, l, m.g_qkv[l].plan, kv->k[l], kv->v[l], ctx, T, st));
+      // five kernels per layer; every elementwise step runs in a GEMM epilogue
+      OOS_TRY(launch_gemm_qkv(m, l, kv->k[l], kv->v[l], ctx, T, st));
       OOS_TRY(launch_attention(m, kv->k[l], kv->v[l], ctx, T, st));
-      OOS_TRY(launch_gemm_tc(m, m.g_o[l], m.amap_attn[bi], T, st));
-      OOS_TRY(launch_resid_norm(m, m.g_o[l].plan, W.mlp_norm, nullptr, T, st));
-      OOS_TRY(launch_gemm_tc(m, m.g_gu[l], m.amap_xn[bi], T, st));
-      OOS_TRY(launch_silu_mul(m, m.g_gu[l].plan, T, st));
-      OOS_TRY(launch_gemm_tc(m, m.g_down[l], m.amap_act[bi], T, st));
-      OOS_TRY(launch_resid_norm(m, m.g_down[l].plan, next_gain, hid, T, st));
+      OOS_TRY(launch_gemm_o(m, l, T, st));
+      OOS_TRY(launch_gemm_gu(m, l, T, st));
+      OOS_TRY(launch_gemm_down(m, l, T, st));
     } else {
       OOS_TRY(launch_gemm_f32(m, W.w_q, W.w_k, W.w_v, qd, kvd, kvd, c.hidden, m.ws.xn, T, st));
       OOS_TRY(launch_qkv_post(m, l, m.p_qkv, kv->k[l], kv->v[l], ctx, T, st));
@@ -169,8 +173,12 @@ static int enqueue_verify(Model& m, const oos_kv_cache* kv, int ctx, const int32
       OOS_TRY(launch_resid_norm(m, m.p_down, next_gain, hid, T, st));
     }
   }
-  if (c.dtype == OOS_DTYPE_BF16) OOS_TRY(launch_lm_head_tc(m, T, st));
-  else OOS_TRY(launch_lm_head_f32(m, T, st));
+  if (c.dtype == OOS_DTYPE_BF16) {
+    if (hidden) OOS_TRY(launch_final_hidden(m, hidden, T, st));
+    OOS_TRY(launch_lm_head_tc(m, T, st));
+  } else {
+    OOS_TRY(launch_lm_head_f32(m, T, st));
+  }
   OOS_TRY(launch_argmax_accept(m, tokens, parent, T, m.lm_grid, len, nodes, toks, bonus, dbg_arg, dbg_t1, dbg_t2, st));
   return OOS_OK;
 }
@@ -293,8 +301,9 @@ int oos_model_create(const oos_model_config* cfg, const oos_weights* w, void* wo
     const int H = c.hidden, I = c.intermediate, qd = c.n_q_heads * c.head_dim, kvd = c.n_kv_heads * c.head_dim;
     m->lm_grid = lm_grid_for(c, n_sms);
     if (c.dtype == OOS_DTYPE_BF16) {
-      auto mk = [&](GemmW& g, const void* const* ptrs, const int* rows, int nseg, int K) -> bool {
+      auto mk = [&](GemmW& g, const void* const* ptrs, const int* rows, int nseg, int K, int interleave) -> bool {
         memset(&g, 0, sizeof(g));
+        g.interleave2 = interleave;
         int tiles = 0, N = 0;
         for (int s = 0; s < nseg; ++s) {
           if (!encode_weight_map(&g.map[s], ptrs[s], rows[s], K)) return false;
@@ -325,12 +334,12 @@ int oos_model_create(const oos_model_config* cfg, const oos_weights* w, void* wo
         const int rg[2] = {I, I};
         const void* pd[1] = {L.w_down};
         const int rd[1] = {H};
-        ok = mk(m->g_qkv[l], pq, rq, 3, H) && mk(m->g_o[l], po, ro, 1, qd) && mk(m->g_gu[l], pg, rg, 2, H) &&
-             mk(m->g_down[l], pd, rd, 1, I);
+        ok = mk(m->g_qkv[l], pq, rq, 3, H, 0) && mk(m->g_o[l], po, ro, 1, qd, 0) && mk(m->g_gu[l], pg, rg, 2, H, 1) &&
+             mk(m->g_down[l], pd, rd, 1, I, 0);
       }
       const void* pl[1] = {c.vocab ? w->lm_head : nullptr};
       const int rl[1] = {c.vocab};
-      ok = ok && mk(m->g_lm, pl, rl, 1, H);
+      ok = ok && mk(m->g_lm, pl, rl, 1, H, 0);
       const int boxes[4] = {16, 32, 64, 128};
       for (int b = 0; b < 4 && ok; ++b)
         ok = encode_act_map(&m->amap_xn[b], m->ws.xn, H, boxes[b]) &&
@@ -418,12 +427,11 @@ int oos_launch_stage(oos_model* m, int32_t layer, int32_t stage, int32_t T, void
   const int qd = c.n_q_heads * c.head_dim, kvd = c.n_kv_heads * c.head_dim;
   cudaError_t e;
   if (c.dtype == OOS_DTYPE_BF16) {
-    const int bi = bn_index(T);
     switch (stage) {
-      case OOS_STAGE_QKV: e = launch_gemm_tc(*m, m->g_qkv[layer], m->amap_xn[bi], T, st); break;
-      case OOS_STAGE_O: e = launch_gemm_tc(*m, m->g_o[layer], m->amap_attn[bi], T, st); break;
-      case OOS_STAGE_GATE_UP: e = launch_gemm_tc(*m, m->g_gu[layer], m->amap_xn[bi], T, st); break;
-      case OOS_STAGE_DOWN: e = launch_gemm_tc(*m, m->g_down[layer], m->amap_act[bi], T, st); break;
+      case OOS_STAGE_QKV: return OOS_EINVAL;   // its epilogue writes the KV cache
+      case OOS_STAGE_O: e = launch_gemm_o(*m, layer, T, st); break;
+      case OOS_STAGE_GATE_UP: e = launch_gemm_gu(*m, layer, T, st); break;
+      case OOS_STAGE_DOWN: e = launch_gemm_down(*m, layer, T, st); break;
       default: e = launch_lm_head_tc(*m, T, st); break;
     }
   } else {

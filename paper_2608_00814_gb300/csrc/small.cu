@@ -18,6 +18,7 @@ __global__ void __launch_bounds__(kMaxT) k_tree_prep(const int32_t* __restrict__
                                                      int32_t* pos_out, unsigned long long* anc_out) {
   __shared__ int s_parent[kMaxT];
   __shared__ int s_bad;
+  pdl_trigger();
   pdl_wait();
   const int i = threadIdx.x;
   if (i == 0) s_bad = 0;
@@ -47,7 +48,6 @@ __global__ void __launch_bounds__(kMaxT) k_tree_prep(const int32_t* __restrict__
     anc_out[2 * i] = lo;
     anc_out[2 * i + 1] = hi;
   }
-  pdl_trigger();
 }
 
 cudaError_t launch_tree_prep(Model& m, const int32_t* tokens, const int32_t* parent, int T, int ctx,
@@ -63,6 +63,7 @@ __global__ void __launch_bounds__(256) k_embed_norm(const int32_t* __restrict__ 
                                                     const E* __restrict__ gain, int H, int vocab, float eps,
                                                     float* __restrict__ x, E* __restrict__ xn) {
   __shared__ float red[32];
+  pdl_trigger();
   pdl_wait();
   const int t = blockIdx.x;
   int tok = tokens[t];
@@ -78,7 +79,6 @@ __global__ void __launch_bounds__(256) k_embed_norm(const int32_t* __restrict__ 
   const float r = rsqrtf(ss / (float)H + eps);
   for (int f = threadIdx.x; f < H; f += blockDim.x)
     store_act(xn, (size_t)t * H + f, (size_t)kMaxT * H, x[(size_t)t * H + f] * r * to_f32(gain[f]));
-  pdl_trigger();
 }
 
 cudaError_t launch_embed_norm(Model& m, const int32_t* tokens, int T, cudaStream_t st) {
@@ -89,6 +89,60 @@ cudaError_t launch_embed_norm(Model& m, const int32_t* tokens, int T, cudaStream
                   c.vocab, c.rms_eps, m.ws.x, (__nv_bfloat16*)m.ws.xn);
   return launch(m.pdl, k_embed_norm<float>, dim3(T), dim3(256), 0, st, tokens, (const float*)m.w.embed,
                 (const float*)m.layers[0].attn_norm, c.hidden, c.vocab, c.rms_eps, m.ws.x, (float*)m.ws.xn);
+}
+
+// bf16 path: the first RMSNorm is folded into the QKV GEMM.  Block (t, chunk)
+// writes x = E[token] (fp32 residual), y = g (.) x (hi/lo bf16 GEMM input) and
+// the chunk's sum of x^2 (the GEMM epilogue turns the chunk sums into
+// rsqrt(mean(x^2) + eps)).
+__global__ void __launch_bounds__(128) k_embed_tc(const int32_t* __restrict__ tokens, const __nv_bfloat16* __restrict__ emb,
+                                                  const __nv_bfloat16* __restrict__ gain, int H, int vocab,
+                                                  float* __restrict__ x, __nv_bfloat16* __restrict__ y,
+                                                  float* __restrict__ ss) {
+  __shared__ float red[32];
+  pdl_trigger();
+  pdl_trigger();
+  pdl_wait();
+  const int t = blockIdx.x, f = blockIdx.y * 128 + threadIdx.x;
+  int tok = tokens[t];
+  tok = tok < 0 ? 0 : (tok >= vocab ? vocab - 1 : tok);   // invalid trees are flagged by tree_prep
+  float v = 0.f;
+  if (f < H) {
+    v = __bfloat162float(emb[(size_t)tok * H + f]);
+    x[(size_t)t * H + f] = v;
+    store_act(y, (size_t)t * H + f, (size_t)kMaxT * H, v * __bfloat162float(gain[f]));
+  }
+  const float s = block_sum(v * v, red);
+  if (threadIdx.x == 0) ss[(size_t)blockIdx.y * kMaxT + t] = s;
+}
+
+cudaError_t launch_embed_tc(Model& m, const int32_t* tokens, int T, cudaStream_t st) {
+  const auto& c = m.cfg;
+  return launch(m.pdl, k_embed_tc, dim3(T, (c.hidden + 127) / 128), dim3(128), 0, st, tokens,
+                (const __nv_bfloat16*)m.w.embed, (const __nv_bfloat16*)m.layers[0].attn_norm, c.hidden, c.vocab,
+                m.ws.x, (__nv_bfloat16*)m.ws.xn, m.ws.ss);
+}
+
+// bf16 path, checking output only: the final RMSNorm output in fp32,
+// hidden[t] = x[t] * rsqrt(mean(x[t]^2) + eps) * g.
+__global__ void __launch_bounds__(256) k_final_hidden(const float* __restrict__ x, const float* __restrict__ ss,
+                                                      int chunks, const __nv_bfloat16* __restrict__ gain, int H,
+                                                      float eps, float* __restrict__ hidden) {
+  pdl_trigger();
+  pdl_trigger();
+  pdl_wait();
+  const int t = blockIdx.x;
+  float s = 0.f;
+  for (int c = 0; c < chunks; ++c) s += ss[(size_t)c * kMaxT + t];
+  const float r = rsqrtf(s / (float)H + eps);
+  for (int f = threadIdx.x; f < H; f += blockDim.x)
+    hidden[(size_t)t * H + f] = x[(size_t)t * H + f] * r * __bfloat162float(gain[f]);
+}
+
+cudaError_t launch_final_hidden(Model& m, float* hidden, int T, cudaStream_t st) {
+  const auto& c = m.cfg;
+  return launch(m.pdl, k_final_hidden, dim3(T), dim3(256), 0, st, (const float*)m.ws.x, (const float*)m.ws.ss,
+                (c.hidden + 127) / 128, (const __nv_bfloat16*)m.w.final_norm, c.hidden, c.rms_eps, hidden);
 }
 
 // sum of the fp32 partial slices of GEMM output (t, f)
@@ -126,6 +180,7 @@ struct QkvPostArgs {
 template <typename E>
 __global__ void k_qkv_post(QkvPostArgs a) {
   __shared__ float red[32];
+  pdl_trigger();
   pdl_wait();
   const int t = blockIdx.x, hs = blockIdx.y, j = threadIdx.x, half = a.d / 2;
   const int f0 = hs * a.d + j, f1 = f0 + half;
@@ -164,7 +219,6 @@ __global__ void k_qkv_post(QkvPostArgs a) {
   else dst = (E*)(kind == 1 ? a.kc : a.vc) + ((size_t)(a.ctx + t) * a.nkv + h) * a.d;
   dst[j] = from_f32<E>(v0);
   dst[j + half] = from_f32<E>(v1);
-  pdl_trigger();
 }
 
 cudaError_t launch_qkv_post(Model& m, int layer, const StreamK& plan, void* kc, void* vc, int ctx, int T,
@@ -204,6 +258,7 @@ __global__ void __launch_bounds__(256) k_resid_norm(const float* __restrict__ pa
                                                     const E* __restrict__ gain, float eps, float* __restrict__ x,
                                                     E* __restrict__ xn, float* __restrict__ hidden_out) {
   __shared__ float red[32];
+  pdl_trigger();
   pdl_wait();
   const int t = blockIdx.x;
   float* xr = x + (size_t)t * H;
@@ -220,7 +275,6 @@ __global__ void __launch_bounds__(256) k_resid_norm(const float* __restrict__ pa
     store_act(xn, (size_t)t * H + f, (size_t)kMaxT * H, y);
     if (hidden_out) hidden_out[(size_t)t * H + f] = y;
   }
-  pdl_trigger();
 }
 
 cudaError_t launch_resid_norm(Model& m, const StreamK& plan, const void* gain, float* hidden_out, int T,
@@ -238,6 +292,7 @@ cudaError_t launch_resid_norm(Model& m, const StreamK& plan, const void* gain, f
 template <typename E>
 __global__ void __launch_bounds__(256) k_silu_mul(const float* __restrict__ part, StreamK plan, int I,
                                                   E* __restrict__ act) {
+  pdl_trigger();
   pdl_wait();
   const int t = blockIdx.y;
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
@@ -246,7 +301,6 @@ __global__ void __launch_bounds__(256) k_silu_mul(const float* __restrict__ part
     const float u = gather_partial(part, plan, 2 * I, t, I + i);
     store_act(act, (size_t)t * I + i, (size_t)kMaxT * I, g / (1.f + expf(-g)) * u);
   }
-  pdl_trigger();
 }
 
 cudaError_t launch_silu_mul(Model& m, const StreamK& plan, int T, cudaStream_t st) {
@@ -343,28 +397,41 @@ __global__ void __launch_bounds__(kMaxT) k_argmax_accept(const float* __restrict
                                                          int32_t* len, int32_t* nodes, int32_t* toks, int32_t* bonus,
                                                          int32_t* dbg_argmax, float* dbg_top1, float* dbg_top2) {
   __shared__ int32_t s_tok[kMaxT], s_par[kMaxT], s_dep[kMaxT], s_arg[kMaxT];
+  pdl_trigger();
   pdl_wait();
-  const int t = threadIdx.x;
-  if (t < T) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
+  // the merge is order independent (max with lowest-id ties, multiset second max)
+  for (int t = warp; t < T; t += nw) {
     Top2 r{-INFINITY, 0x7fffffff, -INFINITY};
-    for (int c = 0; c < n_parts; ++c) {
+    for (int c = lane; c < n_parts; c += 32) {
       const size_t k = (size_t)c * kMaxT + t;
       r = top2_merge(r, Top2{v1[k], i1[k], v2[k]});
     }
-    argmax_ws[t] = r.i1;
-    top1_ws[t] = r.v1;
-    top2_ws[t] = r.v2;
-    if (dbg_argmax) dbg_argmax[t] = r.i1;
-    if (dbg_top1) dbg_top1[t] = r.v1;
-    if (dbg_top2) dbg_top2[t] = r.v2;
-    s_arg[t] = r.i1;
-    s_tok[t] = tokens[t];
-    s_par[t] = parent[t];
-    s_dep[t] = depth[t];
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      Top2 y{__shfl_xor_sync(0xffffffffu, r.v1, o), __shfl_xor_sync(0xffffffffu, r.i1, o),
+             __shfl_xor_sync(0xffffffffu, r.v2, o)};
+      r = top2_merge(r, y);
+    }
+    if (lane == 0) {
+      argmax_ws[t] = r.i1;
+      top1_ws[t] = r.v1;
+      top2_ws[t] = r.v2;
+      if (dbg_argmax) dbg_argmax[t] = r.i1;
+      if (dbg_top1) dbg_top1[t] = r.v1;
+      if (dbg_top2) dbg_top2[t] = r.v2;
+      s_arg[t] = r.i1;
+    }
+  }
+  const int i = threadIdx.x;
+  if (i < T) {
+    s_tok[i] = tokens[i];
+    s_par[i] = parent[i];
+    s_dep[i] = depth[i];
   }
   __syncthreads();
-  if (t < 32) accept_walk_warp(s_tok, s_par, s_dep, s_arg, T, (*status & ST_TREE) != 0, len, nodes, toks, bonus);
-  pdl_trigger();
+  if (threadIdx.x < 32)
+    accept_walk_warp(s_tok, s_par, s_dep, s_arg, T, (*status & ST_TREE) != 0, len, nodes, toks, bonus);
 }
 
 cudaError_t launch_argmax_accept(Model& m, const int32_t* tokens, const int32_t* parent, int T, int n_parts,
@@ -425,6 +492,7 @@ __global__ void k_kv_compact(KvPtrs p, int nkv, int d, int ctx, const int32_t* _
                              const int32_t* __restrict__ len_ptr, int max_len) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   E* buf = reinterpret_cast<E*>(smem_raw);
+  pdl_trigger();
   pdl_wait();
   const int layer = blockIdx.x, which = blockIdx.y, g = blockIdx.z;
   E* base = (E*)(which == 0 ? p.k[layer] : p.v[layer]);
@@ -441,7 +509,6 @@ __global__ void k_kv_compact(KvPtrs p, int nkv, int d, int ctx, const int32_t* _
     const int src = nodes[j];
     if (src >= 0 && src < max_len) base[((size_t)(ctx + j) * nkv + g) * d + c] = buf[e];
   }
-  pdl_trigger();
 }
 
 cudaError_t compact_setup() {
