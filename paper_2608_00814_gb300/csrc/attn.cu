@@ -90,6 +90,7 @@ __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __nv_bfloat16* ring = reinterpret_cast<__nv_bfloat16*>(smem_raw);   // [stage][K | V][64][ld]
   __shared__ int s_last;
+  __shared__ float s_w[kAttnRows][kMaxAttnSplits];   // merge weights (last split only)
   pdl_trigger();
   pdl_wait();
   const int rb = blockIdx.x, g = blockIdx.y, split = blockIdx.z;
@@ -295,22 +296,67 @@ __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
   __syncthreads();
   if (!s_last) return;
   __threadfence();
-  for (int idx = threadIdx.x; idx < kAttnRows * kAttnD; idx += blockDim.x) {
-    const int r = rb * kAttnRows + idx / kAttnD, c = idx % kAttnD;
-    if (r >= R) break;
-    const int node = r / a.group, hq = g * a.group + r % a.group;
-    const size_t grow = (size_t)node * a.nq + hq;
-    float M = -INFINITY;
-    for (int sp = 0; sp < a.splits; ++sp) M = fmaxf(M, __ldcg(a.ml_part + ((size_t)sp * rows_total + grow) * 2));
-    float num = 0.f, den = 0.f;
-    for (int sp = 0; sp < a.splits; ++sp) {
-      const float ms = __ldcg(a.ml_part + ((size_t)sp * rows_total + grow) * 2);
-      if (ms == -INFINITY) continue;
-      const float w = exp2f(ms - M);
-      den += w * __ldcg(a.ml_part + ((size_t)sp * rows_total + grow) * 2 + 1);
-      num += w * __ldcg(a.o_part + ((size_t)sp * rows_total + grow) * kAttnD + c);
+  // per-row split weights w_s = 2^(m_s - M) / sum_s 2^(m_s - M) l_s
+  if (threadIdx.x < kAttnRows) {
+    const int r = rb * kAttnRows + threadIdx.x;
+    if (r < R) {
+      const size_t grow = (size_t)(r / a.group) * a.nq + g * a.group + r % a.group;
+      float ms[kMaxAttnSplits], ls[kMaxAttnSplits];
+      float M = -INFINITY;
+#pragma unroll
+      for (int sp = 0; sp < kMaxAttnSplits; ++sp) {
+        if (sp < a.splits) {
+          const float2 v = __ldcg(reinterpret_cast<const float2*>(a.ml_part + ((size_t)sp * rows_total + grow) * 2));
+          ms[sp] = v.x;
+          ls[sp] = v.y;
+          M = fmaxf(M, v.x);
+        }
+      }
+      float den = 0.f;
+#pragma unroll
+      for (int sp = 0; sp < kMaxAttnSplits; ++sp) {
+        if (sp < a.splits) {
+          const float wgt = ms[sp] == -INFINITY ? 0.f : exp2f(ms[sp] - M);
+          ms[sp] = wgt;
+          den += wgt * ls[sp];
+        }
+      }
+#pragma unroll
+      for (int sp = 0; sp < kMaxAttnSplits; ++sp)
+        if (sp < a.splits) s_w[threadIdx.x][sp] = ms[sp] / den;
     }
-    store_act(a.out, grow * kAttnD + c, a.out_lo_off, num / den);
+  }
+  __syncthreads();
+  // warp w: rows w, w+4, ...; lane: four head dims
+  {
+    constexpr int RW = kAttnRows / 4;
+    float4 acc[RW];
+#pragma unroll
+    for (int i = 0; i < RW; ++i) acc[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int sp = 0; sp < a.splits; ++sp) {
+#pragma unroll
+      for (int i = 0; i < RW; ++i) {
+        const int rr = warp + 4 * i, r = rb * kAttnRows + rr;
+        if (r < R) {
+          const size_t grow = (size_t)(r / a.group) * a.nq + g * a.group + r % a.group;
+          const float4 v = __ldcg(reinterpret_cast<const float4*>(a.o_part + ((size_t)sp * rows_total + grow) * kAttnD + 4 * lane));
+          const float wgt = s_w[rr][sp];
+          acc[i].x += wgt * v.x;
+          acc[i].y += wgt * v.y;
+          acc[i].z += wgt * v.z;
+          acc[i].w += wgt * v.w;
+        }
+      }
+    }
+#pragma unroll
+    for (int i = 0; i < RW; ++i) {
+      const int rr = warp + 4 * i, r = rb * kAttnRows + rr;
+      if (r >= R) break;
+      const size_t grow = (size_t)(r / a.group) * a.nq + g * a.group + r % a.group;
+      const float vals[4] = {acc[i].x, acc[i].y, acc[i].z, acc[i].w};
+#pragma unroll
+      for (int c = 0; c < 4; ++c) store_act(a.out, grow * kAttnD + 4 * lane + c, a.out_lo_off, vals[c]);
+    }
   }
 }
 

@@ -81,7 +81,7 @@ struct TcCfg {
   static constexpr int S = S_RAW > 8 ? 8 : S_RAW;
   static constexpr int NCOLS = (2 * BN) < 32 ? 32 : 2 * BN;    // two accumulators, power of two
   static constexpr int BAR_BYTES = 256;
-  static constexpr int EPI_BYTES = 4 * kMaxT * 4 + kMaxT * 4 + 64;   // column sums, rms, flags
+  static constexpr int EPI_BYTES = kMaxT * 4 + 64;             // input RMSNorm factors, flags
   static constexpr int RED_BYTES = 4 * BN * 12 + BN * 12;      // argmax cross-warp scratch + running state
   static constexpr int SMEM = 1024 /*align slack*/ + S * STAGE + BAR_BYTES + EPI_BYTES + RED_BYTES;
 };
@@ -106,102 +106,155 @@ OOS_DEV Top2s t2_merge(Top2s a, Top2s b) {
 
 OOS_DEV void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
-// sum of the stream-K slices of element (t, n) of a partial tile
-OOS_DEV float slice_sum(const float* part, int nc, size_t slice, size_t idx) {
-  float v = 0.f;
-  for (int s = 0; s < nc; ++s) v += __ldcg(part + (size_t)s * slice + idx);
-  return v;
+// Finishing a tile: warp w of the four epilogue warps owns token rows
+// t = t0 + 4k + w, lane l owns the four features 4l..4l+3 of the tile, so a
+// token's 128 features sit in one warp (RMSNorm sums, q/k norm and the RoPE
+// pair exchange are warp shuffles) and every slice load is a coalesced float4.
+// All loads of a pass are issued before any result is stored.
+constexpr int kFinRows = 16;   // token rows per warp per pass (64 tokens per pass)
+
+OOS_DEV float4 f4_add(float4 a, float4 b) { return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w); }
+OOS_DEV float4 f4_ldcg(const float* p) { return __ldcg(reinterpret_cast<const float4*>(p)); }
+
+// acc[k] = (init ? init row : 0) + sum over nc slices of the partial tile rows
+OOS_DEV void load_tile_rows(float4 (&acc)[kFinRows], const float* __restrict__ part, int nc, size_t slice, int n_part,
+                            int col, int t0, int T, const float* __restrict__ init, int init_ld) {
+  const int w = (threadIdx.x - 64) >> 5;
+#pragma unroll
+  for (int k = 0; k < kFinRows; ++k) {
+    const int t = t0 + 4 * k + w;
+    acc[k] = (init && t < T) ? *reinterpret_cast<const float4*>(init + (size_t)t * init_ld + col)
+                             : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
+  for (int sl = 0; sl < nc; ++sl) {
+    const float* base = part + (size_t)sl * slice + col;
+#pragma unroll
+    for (int k = 0; k < kFinRows; ++k) {
+      const int t = t0 + 4 * k + w;
+      if (t < T) acc[k] = f4_add(acc[k], f4_ldcg(base + (size_t)t * n_part));
+    }
+  }
+}
+
+OOS_DEV void store_act4(__nv_bfloat16* p, size_t i, size_t lo_off, float4 v) {
+  const float a[4] = {v.x, v.y, v.z, v.w};
+  __nv_bfloat16 hi[4], lo[4];
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    hi[c] = __float2bfloat16_rn(a[c]);
+    lo[c] = __float2bfloat16_rn(a[c] - __bfloat162float(hi[c]));
+  }
+  *reinterpret_cast<uint2*>(p + i) = *reinterpret_cast<const uint2*>(hi);
+  *reinterpret_cast<uint2*>(p + i + lo_off) = *reinterpret_cast<const uint2*>(lo);
+}
+
+OOS_DEV float4 bf16x4(const __nv_bfloat16* p) {
+  const uint2 u = *reinterpret_cast<const uint2*>(p);
+  const __nv_bfloat16* h = reinterpret_cast<const __nv_bfloat16*>(&u);
+  return make_float4(__bfloat162float(h[0]), __bfloat162float(h[1]), __bfloat162float(h[2]), __bfloat162float(h[3]));
 }
 
 template <int EPI>
-OOS_DEV void finish_tile(const GemmArgs& a, int tile, const float* rms, float* col_red, float* pair_red) {
+OOS_DEV void finish_tile(const GemmArgs& a, int tile, const float* rms) {
   const int e = threadIdx.x - 64;     // 0..127
-  const int warp = e >> 5, lane = e & 31;
+  const int w = e >> 5, l = e & 31;
   const int n_part = a.n_tiles * kTile;
   const size_t slice = (size_t)kMaxT * n_part;
   StreamK sk{a.n_tiles, a.kbt, a.total, (int)gridDim.x};
   int c0, c1;
   if (EPI == EPI_RESID) {
+    // x += W.a; y = g (.) x (next RMSNorm input); per-tile sums of x^2
     sk.contributors(tile, c0, c1);
-    const int nc = c1 - c0 + 1;
-    const int f = tile * kTile + e;
-    const bool fv = f < a.N;
-    const float g = fv ? __bfloat162float(a.gain[f]) : 0.f;
-    for (int t = 0; t < a.T; ++t) {
-      float sq = 0.f;
-      if (fv) {
-        const float xv = a.x[(size_t)t * a.N + f] + slice_sum(a.part, nc, slice, (size_t)t * n_part + f);
-        a.x[(size_t)t * a.N + f] = xv;
-        store_act(a.y_out, (size_t)t * a.N + f, (size_t)kMaxT * a.N, g * xv);
-        sq = xv * xv;
+    const int f = tile * kTile + 4 * l;
+    const float4 g = bf16x4(a.gain + f);
+    for (int t0 = 0; t0 < a.T; t0 += 4 * kFinRows) {
+      float4 acc[kFinRows];
+      load_tile_rows(acc, a.part, c1 - c0 + 1, slice, n_part, f, t0, a.T, a.x, a.N);   // x + sum of slices
+#pragma unroll
+      for (int k = 0; k < kFinRows; ++k) {
+        const int t = t0 + 4 * k + w;
+        if (t >= a.T) break;
+        const float4 xv = acc[k];
+        *reinterpret_cast<float4*>(a.x + (size_t)t * a.N + f) = xv;
+        store_act4(a.y_out, (size_t)t * a.N + f, (size_t)kMaxT * a.N,
+                   make_float4(g.x * xv.x, g.y * xv.y, g.z * xv.z, g.w * xv.w));
+        const float sq = warp_sum(xv.x * xv.x + xv.y * xv.y + xv.z * xv.z + xv.w * xv.w);
+        if (l == 0) a.ss_out[(size_t)tile * kMaxT + t] = sq;
       }
-      sq = warp_sum(sq);
-      if (lane == 0) col_red[warp * kMaxT + t] = sq;
     }
-    epi_bar();
-    if (e < a.T) a.ss_out[(size_t)tile * kMaxT + e] = col_red[e] + col_red[kMaxT + e] + col_red[2 * kMaxT + e] + col_red[3 * kMaxT + e];
-    epi_bar();
   } else if (EPI == EPI_SILU) {
-    int g0, g1, u0, u1;
-    sk.contributors(2 * (tile >> 1), g0, g1);
-    sk.contributors(2 * (tile >> 1) + 1, u0, u1);
-    const int i = (tile >> 1) * kTile + e;        // feature of the SwiGLU output
-    if (i < a.I) {
-      const int fg = 2 * (tile >> 1) * kTile + e, fu = fg + kTile;
-      for (int t = 0; t < a.T; ++t) {
-        const float gv = slice_sum(a.part, g1 - g0 + 1, slice, (size_t)t * n_part + fg) * rms[t];
-        const float uv = slice_sum(a.part, u1 - u0 + 1, slice, (size_t)t * n_part + fu) * rms[t];
-        store_act(a.act_out, (size_t)t * a.I + i, (size_t)kMaxT * a.I, gv / (1.f + expf(-gv)) * uv);
+    // act = silu(r g) * (r u) for the 128 features of gate/up pair tile/2
+    const int pr = tile >> 1;
+    int u0, u1;
+    sk.contributors(2 * pr, c0, c1);
+    sk.contributors(2 * pr + 1, u0, u1);
+    const int i = pr * kTile + 4 * l;
+    for (int t0 = 0; t0 < a.T; t0 += 4 * kFinRows) {
+      float4 gv[kFinRows], uv[kFinRows];
+      load_tile_rows(gv, a.part, c1 - c0 + 1, slice, n_part, 2 * pr * kTile + 4 * l, t0, a.T, nullptr, 0);
+      load_tile_rows(uv, a.part, u1 - u0 + 1, slice, n_part, (2 * pr + 1) * kTile + 4 * l, t0, a.T, nullptr, 0);
+#pragma unroll
+      for (int k = 0; k < kFinRows; ++k) {
+        const int t = t0 + 4 * k + w;
+        if (t >= a.T) break;
+        const float r = rms[t];
+        const float g4[4] = {gv[k].x * r, gv[k].y * r, gv[k].z * r, gv[k].w * r};
+        const float u4[4] = {uv[k].x * r, uv[k].y * r, uv[k].z * r, uv[k].w * r};
+        float o4[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) o4[c] = g4[c] / (1.f + expf(-g4[c])) * u4[c];
+        store_act4(a.act_out, (size_t)t * a.I + i, (size_t)kMaxT * a.I, make_float4(o4[0], o4[1], o4[2], o4[3]));
       }
     }
-  } else {  // EPI_QKV: tile = one head of 128 features (q heads, then k heads, then v heads)
+  } else {
+    // EPI_QKV: tile = one head of 128 features (q heads, then k heads, then v heads)
     sk.contributors(tile, c0, c1);
-    const int nc = c1 - c0 + 1;
     int kind, h;
     if (tile < a.nq) { kind = 0; h = tile; }
     else if (tile < a.nq + a.nkv) { kind = 1; h = tile - a.nq; }
     else { kind = 2; h = tile - a.nq - a.nkv; }
     const __nv_bfloat16* bias = kind == 0 ? a.bq : kind == 1 ? a.bk : a.bv;
     const __nv_bfloat16* gn = kind == 0 ? a.gq : kind == 1 ? a.gk : nullptr;
-    const int j = e & 63;
+    const float4 b4 = bias ? bf16x4(bias + h * kTile + 4 * l) : make_float4(0.f, 0.f, 0.f, 0.f);
+    const float4 g4 = gn ? bf16x4(gn + 4 * l) : make_float4(1.f, 1.f, 1.f, 1.f);
+    const int m0 = 4 * (l & 15);      // rotary frequency index of this lane's first feature
+    const bool first_half = l < 16;   // features 0..63 pair with 64..127 held by lane ^ 16
     const double two_pi = 6.283185307179586476925286766559;
-    for (int t0 = 0; t0 < a.T; t0 += 2) {
-      const int t = t0 + (e >> 6);
-      const bool tv = t < a.T;
-      float v0 = 0.f, v1 = 0.f;
-      if (tv) {
-        const size_t base = (size_t)t * n_part + (size_t)tile * kTile + j;
-        v0 = slice_sum(a.part, nc, slice, base) * rms[t];
-        v1 = slice_sum(a.part, nc, slice, base + 64) * rms[t];
-        if (bias) {
-          v0 += __bfloat162float(bias[h * kTile + j]);
-          v1 += __bfloat162float(bias[h * kTile + j + 64]);
+    for (int t0 = 0; t0 < a.T; t0 += 4 * kFinRows) {
+      float4 acc[kFinRows];
+      load_tile_rows(acc, a.part, c1 - c0 + 1, slice, n_part, tile * kTile + 4 * l, t0, a.T, nullptr, 0);
+#pragma unroll
+      for (int k = 0; k < kFinRows; ++k) {
+        const int t = t0 + 4 * k + w;
+        if (t >= a.T) break;
+        const float r = rms[t];
+        float v[4] = {acc[k].x * r + b4.x, acc[k].y * r + b4.y, acc[k].z * r + b4.z, acc[k].w * r + b4.w};
+        if (gn) {   // per-head RMSNorm over the head's 128 features
+          const float ss = warp_sum(v[0] * v[0] + v[1] * v[1] + v[2] * v[2] + v[3] * v[3]);
+          const float rn = rsqrtf(ss * (1.f / kTile) + a.eps);
+          v[0] *= rn * g4.x;
+          v[1] *= rn * g4.y;
+          v[2] *= rn * g4.z;
+          v[3] *= rn * g4.w;
         }
+        if (kind < 2) {   // rotate-half RoPE at position ctx + depth(t)
+          const double p = (double)a.pos[t];
+#pragma unroll
+          for (int c = 0; c < 4; ++c) {
+            const float other = __shfl_xor_sync(0xffffffffu, v[c], 16);
+            const double ang = p * a.inv_freq[m0 + c];
+            float sn, cs;
+            sincosf((float)(ang - two_pi * rint(ang / two_pi)), &sn, &cs);
+            v[c] = first_half ? v[c] * cs - other * sn : v[c] * cs + other * sn;
+          }
+        }
+        __nv_bfloat16* dst = kind == 0 ? a.q_out + ((size_t)t * a.nq + h) * kTile
+                                       : (kind == 1 ? a.kc : a.vc) + ((size_t)(a.ctx + t) * a.nkv + h) * kTile;
+        __nv_bfloat16 o[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) o[c] = __float2bfloat16_rn(v[c]);
+        *reinterpret_cast<uint2*>(dst + 4 * l) = *reinterpret_cast<const uint2*>(o);
       }
-      if (gn) {   // per-head RMSNorm over the 128 features of this token
-        const float ss = warp_sum(v0 * v0 + v1 * v1);
-        if (lane == 0) pair_red[warp] = ss;
-        epi_bar();
-        const float tot = pair_red[warp & 2] + pair_red[(warp & 2) + 1];
-        epi_bar();
-        const float r = rsqrtf(tot * (1.f / kTile) + a.eps);
-        v0 = v0 * r * __bfloat162float(gn[j]);
-        v1 = v1 * r * __bfloat162float(gn[j + 64]);
-      }
-      if (!tv) continue;
-      if (kind < 2) {   // rotate-half RoPE at position ctx + depth(t)
-        const double ang = (double)a.pos[t] * a.inv_freq[j];
-        const float ra = (float)(ang - two_pi * rint(ang / two_pi));
-        float sn, cs;
-        sincosf(ra, &sn, &cs);
-        const float o0 = v0 * cs - v1 * sn, o1 = v1 * cs + v0 * sn;
-        v0 = o0;
-        v1 = o1;
-      }
-      __nv_bfloat16* dst = kind == 0 ? a.q_out + ((size_t)t * a.nq + h) * kTile
-                                     : (kind == 1 ? a.kc : a.vc) + ((size_t)(a.ctx + t) * a.nkv + h) * kTile;
-      dst[j] = __float2bfloat16_rn(v0);
-      dst[j + 64] = __float2bfloat16_rn(v1);
     }
   }
 }
@@ -224,10 +277,8 @@ __global__ void __launch_bounds__(192, 1)
   uint64_t* drain = acce + 2;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  float* col_red = reinterpret_cast<float*>(smem + S * C::STAGE + C::BAR_BYTES);   // [4][kMaxT]
-  float* rms = col_red + 4 * kMaxT;                                                 // [kMaxT]
-  float* pair_red = rms + kMaxT;                                                    // [4]
-  volatile int* s_last = reinterpret_cast<volatile int*>(pair_red + 4);
+  float* rms = reinterpret_cast<float*>(smem + S * C::STAGE + C::BAR_BYTES);       // [kMaxT]
+  volatile int* s_last = reinterpret_cast<volatile int*>(rms + kMaxT);
   Top2s* red = reinterpret_cast<Top2s*>(smem + S * C::STAGE + C::BAR_BYTES + C::EPI_BYTES);   // [4][BN]
   Top2s* run = red + 4 * BN;                                                                   // [BN]
 
@@ -460,7 +511,7 @@ __global__ void __launch_bounds__(192, 1)
         epi_bar();
         if (*s_last) {
           __threadfence();
-          finish_tile<EPI>(a, tile, rms, col_red, pair_red);
+          finish_tile<EPI>(a, tile, rms);
         }
         epi_bar();
       } else {
