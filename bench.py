@@ -220,7 +220,7 @@ def run_ours(args):
     torch.cuda.set_device(local)
     dev = torch.cuda.current_device()
     w = WORKLOADS[args.workload]
-    cfg = w.model
+    cfg = w.model if not args.layers else dataclasses.replace(w.model, n_layers=args.layers)
     T, ctx = w.T, w.ctx_len
     seed, tokens_np, parent_np, path = workload_tree(args.workload)
 
@@ -342,7 +342,9 @@ def run_ours(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16" if cfg.dtype == "bf16" else "f32", "data": "synthetic",
-            "config": {"workload": "%s T=%d ctx_len=%d" % (args.workload, T, ctx), "T": T, "ctx_len": ctx,
+            "config": {"workload": "%s T=%d ctx_len=%d%s" % (args.workload, T, ctx,
+                                                               " layers=%d" % cfg.n_layers if args.layers else ""),
+                       "T": T, "ctx_len": ctx,
                        "accepted_len": acc_len, "l2": "inputs larger than L2 (weights streamed once per step)",
                        "parallelism": "replicas" if world > 1 else "single GPU"},
             "us_per_step": ms * 1e3,
@@ -371,6 +373,8 @@ def main():
                                                                       if w.model.dtype == "bf16"))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--layers", type=int, default=0,
+                    help="profiling captures only: keep the first N layers of the workload's model")
     args = ap.parse_args()
     if args.impl == "reference":
         run_reference(args)

@@ -54,8 +54,7 @@ struct GemmArgs {
   // EPI_QKV
   int nq, nkv;
   const __nv_bfloat16 *bq, *bk, *bv, *gq, *gk;
-  const int32_t* pos;
-  const double* inv_freq;
+  const float2* rope;   // [kMaxT][64] (cos, sin) of the step's positions
   __nv_bfloat16 *q_out, *kc, *vc;
   int ctx;
   // EPI_RESID
@@ -219,7 +218,6 @@ OOS_DEV void finish_tile(const GemmArgs& a, int tile, const float* rms) {
     const float4 g4 = gn ? bf16x4(gn + 4 * l) : make_float4(1.f, 1.f, 1.f, 1.f);
     const int m0 = 4 * (l & 15);      // rotary frequency index of this lane's first feature
     const bool first_half = l < 16;   // features 0..63 pair with 64..127 held by lane ^ 16
-    const double two_pi = 6.283185307179586476925286766559;
     for (int t0 = 0; t0 < a.T; t0 += 4 * kFinRows) {
       float4 acc[kFinRows];
       load_tile_rows(acc, a.part, c1 - c0 + 1, slice, n_part, tile * kTile + 4 * l, t0, a.T, nullptr, 0);
@@ -238,14 +236,11 @@ OOS_DEV void finish_tile(const GemmArgs& a, int tile, const float* rms) {
           v[3] *= rn * g4.w;
         }
         if (kind < 2) {   // rotate-half RoPE at position ctx + depth(t)
-          const double p = (double)a.pos[t];
 #pragma unroll
           for (int c = 0; c < 4; ++c) {
             const float other = __shfl_xor_sync(0xffffffffu, v[c], 16);
-            const double ang = p * a.inv_freq[m0 + c];
-            float sn, cs;
-            sincosf((float)(ang - two_pi * rint(ang / two_pi)), &sn, &cs);
-            v[c] = first_half ? v[c] * cs - other * sn : v[c] * cs + other * sn;
+            const float2 cs = a.rope[t * (kTile / 2) + m0 + c];
+            v[c] = first_half ? v[c] * cs.x - other * cs.y : v[c] * cs.x + other * cs.y;
           }
         }
         __nv_bfloat16* dst = kind == 0 ? a.q_out + ((size_t)t * a.nq + h) * kTile
@@ -681,8 +676,7 @@ cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int ctx, in
   a.bv = (const __nv_bfloat16*)(c.qkv_bias ? L.b_v : nullptr);
   a.gq = (const __nv_bfloat16*)(c.qk_norm ? L.q_norm : nullptr);
   a.gk = (const __nv_bfloat16*)(c.qk_norm ? L.k_norm : nullptr);
-  a.pos = m.ws.pos;
-  a.inv_freq = m.ws.inv_freq;
+  a.rope = m.ws.rope;
   a.q_out = (__nv_bfloat16*)m.ws.q;
   a.kc = (__nv_bfloat16*)kc;
   a.vc = (__nv_bfloat16*)vc;

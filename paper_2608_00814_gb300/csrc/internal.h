@@ -88,6 +88,7 @@ struct Workspace {
   float* top1;
   float* top2;
   float* ss;                 // sum of x^2 per 128-feature chunk [kMaxSsChunks][kMaxT] (bf16 path)
+  float2* rope;              // (cos, sin) per node and rotary pair [kMaxT][d/2] (bf16 path)
   int* cnt;                  // GEMM arrival counters [4][kCntStride]
   int* attn_cnt;             // attention split arrival counters [kAttnCnt]
 };

@@ -86,6 +86,7 @@ size_t carve_workspace(const oos_model_config& c, int n_sms, uint8_t* base, Work
   w.top1 = (float*)take(kMaxT * 4);
   w.top2 = (float*)take(kMaxT * 4);
   w.ss = (float*)take((size_t)kMaxSsChunks * kMaxT * 4);
+  w.rope = (float2*)take((size_t)kMaxT * (c.head_dim / 2) * 8);
   w.cnt = (int*)take((size_t)4 * kCntStride * 4);
   w.attn_cnt = (int*)take((size_t)kAttnCnt * 4);
   if (ws) *ws = w;

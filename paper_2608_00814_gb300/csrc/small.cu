@@ -95,15 +95,26 @@ cudaError_t launch_embed_norm(Model& m, const int32_t* tokens, int T, cudaStream
 // writes x = E[token] (fp32 residual), y = g (.) x (hi/lo bf16 GEMM input) and
 // the chunk's sum of x^2 (the GEMM epilogue turns the chunk sums into
 // rsqrt(mean(x^2) + eps)).
+// Block (t, 0) also fills the step's RoPE table: cos/sin of pos[t] * theta^(-2m/d)
+// for m < d/2, the angle formed and reduced to [-pi, pi] in fp64 once per step
+// (every layer reuses it).
 __global__ void __launch_bounds__(128) k_embed_tc(const int32_t* __restrict__ tokens, const __nv_bfloat16* __restrict__ emb,
                                                   const __nv_bfloat16* __restrict__ gain, int H, int vocab,
                                                   float* __restrict__ x, __nv_bfloat16* __restrict__ y,
-                                                  float* __restrict__ ss) {
+                                                  float* __restrict__ ss, const int32_t* __restrict__ pos,
+                                                  const double* __restrict__ inv_freq, int half_d,
+                                                  float2* __restrict__ rope) {
   __shared__ float red[32];
-  pdl_trigger();
   pdl_trigger();
   pdl_wait();
   const int t = blockIdx.x, f = blockIdx.y * 128 + threadIdx.x;
+  if (blockIdx.y == 0 && threadIdx.x < half_d) {
+    const double two_pi = 6.283185307179586476925286766559;
+    const double ang = (double)pos[t] * inv_freq[threadIdx.x];
+    float sn, cs;
+    sincosf((float)(ang - two_pi * rint(ang / two_pi)), &sn, &cs);
+    rope[t * half_d + threadIdx.x] = make_float2(cs, sn);
+  }
   int tok = tokens[t];
   tok = tok < 0 ? 0 : (tok >= vocab ? vocab - 1 : tok);   // invalid trees are flagged by tree_prep
   float v = 0.f;
@@ -120,7 +131,8 @@ cudaError_t launch_embed_tc(Model& m, const int32_t* tokens, int T, cudaStream_t
   const auto& c = m.cfg;
   return launch(m.pdl, k_embed_tc, dim3(T, (c.hidden + 127) / 128), dim3(128), 0, st, tokens,
                 (const __nv_bfloat16*)m.w.embed, (const __nv_bfloat16*)m.layers[0].attn_norm, c.hidden, c.vocab,
-                m.ws.x, (__nv_bfloat16*)m.ws.xn, m.ws.ss);
+                m.ws.x, (__nv_bfloat16*)m.ws.xn, m.ws.ss, (const int32_t*)m.ws.pos, (const double*)m.ws.inv_freq,
+                c.head_dim / 2, m.ws.rope);
 }
 
 // bf16 path, checking output only: the final RMSNorm output in fp32,
@@ -128,7 +140,6 @@ cudaError_t launch_embed_tc(Model& m, const int32_t* tokens, int T, cudaStream_t
 __global__ void __launch_bounds__(256) k_final_hidden(const float* __restrict__ x, const float* __restrict__ ss,
                                                       int chunks, const __nv_bfloat16* __restrict__ gain, int H,
                                                       float eps, float* __restrict__ hidden) {
-  pdl_trigger();
   pdl_trigger();
   pdl_wait();
   const int t = blockIdx.x;
