@@ -62,8 +62,10 @@ OOS_DEV void ldsm_x4_t(uint32_t (&r)[4], const void* p) {
                : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
                : "r"(smem_addr(p)));
 }
+// pure register operation: not volatile, so the compiler may interleave
+// independent MMAs with loads and each other
 OOS_DEV void mma_bf16(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
-  asm volatile(
+  asm(
       "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
       "{%0,%1,%2,%3};"
       : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
@@ -174,18 +176,21 @@ __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
     bool tree;
     tile_keys(ti, key0, key_end, tree);
 
-    // S = Q K^T  (16 rows x 64 keys per warp)
+    // S = Q K^T  (16 rows x 64 keys per warp); k-steps outer, key groups inner,
+    // so consecutive MMAs write different accumulators
     float s[8][4];
 #pragma unroll
-    for (int nt = 0; nt < 8; ++nt) {
-      s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
+    for (int nt = 0; nt < 8; ++nt) s[nt][0] = s[nt][1] = s[nt][2] = s[nt][3] = 0.f;
 #pragma unroll
-      for (int ks = 0; ks < 8; ks += 2) {
-        uint32_t b[4];
-        ldsm_x4(b, kt + (nt * 8 + (lane & 7)) * kAttnLd + ks * 16 + (lane >> 3) * 8);
-        mma_bf16(s[nt], qf[ks], b[0], b[1]);
-        mma_bf16(s[nt], qf[ks + 1], b[2], b[3]);
-      }
+    for (int ks = 0; ks < 8; ks += 2) {
+      uint32_t b[8][4];
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt)
+        ldsm_x4(b[nt], kt + (nt * 8 + (lane & 7)) * kAttnLd + ks * 16 + (lane >> 3) * 8);
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt) mma_bf16(s[nt], qf[ks], b[nt][0], b[nt][1]);
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt) mma_bf16(s[nt], qf[ks + 1], b[nt][2], b[nt][3]);
     }
     // mask + scale, tile row maxima
     float tmax_lo = -INFINITY, tmax_hi = -INFINITY;
@@ -244,13 +249,15 @@ __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
       pa[1] = pack_bf16(s[2 * kk][2], s[2 * kk][3]);
       pa[2] = pack_bf16(s[2 * kk + 1][0], s[2 * kk + 1][1]);
       pa[3] = pack_bf16(s[2 * kk + 1][2], s[2 * kk + 1][3]);
+      uint32_t b[8][4];
+      const int mi = lane >> 3;
+#pragma unroll
+      for (int n2 = 0; n2 < 16; n2 += 2)
+        ldsm_x4_t(b[n2 / 2], vt + (kk * 16 + (mi & 1) * 8 + (lane & 7)) * kAttnLd + (n2 + (mi >> 1)) * 8);
 #pragma unroll
       for (int n2 = 0; n2 < 16; n2 += 2) {
-        uint32_t b[4];
-        const int mi = lane >> 3;
-        ldsm_x4_t(b, vt + (kk * 16 + (mi & 1) * 8 + (lane & 7)) * kAttnLd + (n2 + (mi >> 1)) * 8);
-        mma_bf16(o[n2], pa, b[0], b[1]);
-        mma_bf16(o[n2 + 1], pa, b[2], b[3]);
+        mma_bf16(o[n2], pa, b[n2 / 2][0], b[n2 / 2][1]);
+        mma_bf16(o[n2 + 1], pa, b[n2 / 2][2], b[n2 / 2][3]);
       }
     }
     __syncthreads();
