@@ -15,6 +15,7 @@
 //
 // fp32 path: one block per (node, head), CUDA cores (small models only).
 #include <math.h>
+#include <stdlib.h>
 
 #include "common.cuh"
 #include "internal.h"
@@ -192,23 +193,33 @@ __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
 #pragma unroll
       for (int nt = 0; nt < 8; ++nt) mma_bf16(s[nt], qf[ks + 1], b[nt][2], b[nt][3]);
     }
-    // mask + scale, tile row maxima
+    // scale (+ mask on the tree tail and a partial last cache tile), tile row maxima
     float tmax_lo = -INFINITY, tmax_hi = -INFINITY;
+    if (tree || key_end < key0 + kAttnKeys) {
 #pragma unroll
-    for (int nt = 0; nt < 8; ++nt) {
+      for (int nt = 0; nt < 8; ++nt) {
 #pragma unroll
-      for (int e = 0; e < 4; ++e) {
-        const int key = key0 + nt * 8 + (lane & 3) * 2 + (e & 1);
-        bool valid = key < key_end;
-        if (tree && valid) {
-          const int j = key - a.ctx;
-          const unsigned long long w0 = (e < 2) ? anc_lo0 : anc_hi0;
-          const unsigned long long w1 = (e < 2) ? anc_lo1 : anc_hi1;
-          valid = ((j < 64 ? (w0 >> j) : (w1 >> (j - 64))) & 1ull) != 0;
+        for (int e = 0; e < 4; ++e) {
+          const int key = key0 + nt * 8 + (lane & 3) * 2 + (e & 1);
+          bool valid = key < key_end;
+          if (tree && valid) {
+            const int j = key - a.ctx;
+            const unsigned long long w0 = (e < 2) ? anc_lo0 : anc_hi0;
+            const unsigned long long w1 = (e < 2) ? anc_lo1 : anc_hi1;
+            valid = ((j < 64 ? (w0 >> j) : (w1 >> (j - 64))) & 1ull) != 0;
+          }
+          const float v = valid ? s[nt][e] * a.scale_log2 : -INFINITY;
+          s[nt][e] = v;
+          if (e < 2) tmax_lo = fmaxf(tmax_lo, v); else tmax_hi = fmaxf(tmax_hi, v);
         }
-        const float v = valid ? s[nt][e] * a.scale_log2 : -INFINITY;
-        s[nt][e] = v;
-        if (e < 2) tmax_lo = fmaxf(tmax_lo, v); else tmax_hi = fmaxf(tmax_hi, v);
+      }
+    } else {
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt) {
+#pragma unroll
+        for (int e = 0; e < 4; ++e) s[nt][e] *= a.scale_log2;
+        tmax_lo = fmaxf(tmax_lo, fmaxf(s[nt][0], s[nt][1]));
+        tmax_hi = fmaxf(tmax_hi, fmaxf(s[nt][2], s[nt][3]));
       }
     }
 #pragma unroll
@@ -338,16 +349,20 @@ __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
   {
     constexpr int RW = kAttnRows / 4;
     float4 acc[RW];
+    int grow[RW];   // output row (node * nq + head) of each handled query row, -1 past R
 #pragma unroll
-    for (int i = 0; i < RW; ++i) acc[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int i = 0; i < RW; ++i) {
+      acc[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+      const int r = rb * kAttnRows + warp + 4 * i;
+      grow[i] = r < R ? (r / a.group) * a.nq + g * a.group + r % a.group : -1;
+    }
     for (int sp = 0; sp < a.splits; ++sp) {
+      const float* src = a.o_part + (size_t)sp * rows_total * kAttnD + 4 * lane;
 #pragma unroll
       for (int i = 0; i < RW; ++i) {
-        const int rr = warp + 4 * i, r = rb * kAttnRows + rr;
-        if (r < R) {
-          const size_t grow = (size_t)(r / a.group) * a.nq + g * a.group + r % a.group;
-          const float4 v = __ldcg(reinterpret_cast<const float4*>(a.o_part + ((size_t)sp * rows_total + grow) * kAttnD + 4 * lane));
-          const float wgt = s_w[rr][sp];
+        if (grow[i] >= 0) {
+          const float4 v = __ldcg(reinterpret_cast<const float4*>(src + (size_t)grow[i] * kAttnD));
+          const float wgt = s_w[warp + 4 * i][sp];
           acc[i].x += wgt * v.x;
           acc[i].y += wgt * v.y;
           acc[i].z += wgt * v.z;
@@ -356,14 +371,8 @@ __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
       }
     }
 #pragma unroll
-    for (int i = 0; i < RW; ++i) {
-      const int rr = warp + 4 * i, r = rb * kAttnRows + rr;
-      if (r >= R) break;
-      const size_t grow = (size_t)(r / a.group) * a.nq + g * a.group + r % a.group;
-      const float vals[4] = {acc[i].x, acc[i].y, acc[i].z, acc[i].w};
-#pragma unroll
-      for (int c = 0; c < 4; ++c) store_act(a.out, grow * kAttnD + 4 * lane + c, a.out_lo_off, vals[c]);
-    }
+    for (int i = 0; i < RW; ++i)
+      if (grow[i] >= 0) store_act4(a.out, (size_t)grow[i] * kAttnD + 4 * lane, a.out_lo_off, acc[i]);
   }
 }
 
@@ -444,8 +453,9 @@ cudaError_t launch_attention(Model& m, const void* kc, const void* vc, int ctx, 
   const int R = T * a.group;
   const int RB = (R + kAttnRows - 1) / kAttnRows;
   a.row_blocks = RB;
-  // one wave at two blocks per SM
+  // one wave at two blocks per SM (OOS_ATTN_SPLITS overrides, for tuning)
   int splits = (2 * m.num_sms) / (a.nkv * RB);
+  if (const char* e = getenv("OOS_ATTN_SPLITS")) splits = atoi(e);
   const int max_splits = a.cache_blocks > 0 ? (a.cache_blocks < kMaxAttnSplits ? a.cache_blocks : kMaxAttnSplits) : 1;
   splits = splits < 1 ? 1 : (splits > max_splits ? max_splits : splits);
   a.splits = splits;

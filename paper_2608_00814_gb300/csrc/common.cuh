@@ -41,6 +41,18 @@ OOS_DEV void store_act(__nv_bfloat16* p, size_t i, size_t lo_off, float v) {
   p[i + lo_off] = __float2bfloat16_rn(v - __bfloat162float(hi));
 }
 
+OOS_DEV void store_act4(__nv_bfloat16* p, size_t i, size_t lo_off, float4 v) {
+  const float a[4] = {v.x, v.y, v.z, v.w};
+  __nv_bfloat16 hi[4], lo[4];
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    hi[c] = __float2bfloat16_rn(a[c]);
+    lo[c] = __float2bfloat16_rn(a[c] - __bfloat162float(hi[c]));
+  }
+  *reinterpret_cast<uint2*>(p + i) = *reinterpret_cast<const uint2*>(hi);
+  *reinterpret_cast<uint2*>(p + i + lo_off) = *reinterpret_cast<const uint2*>(lo);
+}
+
 // ---- block reductions (deterministic order)
 OOS_DEV float warp_sum(float v) {
 #pragma unroll
