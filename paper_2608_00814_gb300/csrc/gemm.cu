@@ -38,14 +38,21 @@ namespace oos {
 // multiplies column t by r_t = rsqrt(sum x_t^2 / H + eps) in its epilogue.
 enum { EPI_QKV = 0, EPI_RESID = 1, EPI_SILU = 2, EPI_ARGMAX = 3 };
 
+// A work tile is kSub = 2 weight subtiles of 128 rows (the MMA's M) that share
+// every staged activation slice: per weight byte, half the activation traffic
+// and more weight bytes in flight than single 128-row tiles.  Subtile s of
+// work tile w is the 128-row tile 2w + s of the stacked weight.
+constexpr int kSub = 2;
+
 struct GemmArgs {
-  int seg_tiles[3];   // cumulative tile counts per weight segment
-  int interleave2;    // tile 2i -> segment 0 block i, tile 2i+1 -> segment 1 block i
-  int n_tiles, kbt, total;
+  int seg_tiles[3];   // cumulative 128-row tile counts per weight segment
+  int interleave2;    // 128-row tile 2i -> segment 0 block i, tile 2i+1 -> segment 1 block i
+  int n_tiles;        // 128-row tiles of the stacked weight
+  int n_work, kbt, total;   // work tiles (kSub subtiles each), k-blocks per tile, n_work * kbt
   int N;              // output rows (features / vocab) of the stacked weight
   int T;              // valid columns (tree nodes)
-  float* part;        // partial tiles [slice][kMaxT][n_tiles * 128]
-  int* cnt;           // arrival counters (per tile, per gate/up pair); zero between launches
+  float* part;        // partial tiles [slice][kMaxT][n_work * kSub * 128]
+  int* cnt;           // arrival counters per work tile; zero between launches
   uint32_t* status;
   // RMSNorm scale of the GEMM input (EPI_QKV, EPI_SILU, EPI_ARGMAX)
   const float* ss_in;   // [chunk][kMaxT]
@@ -73,16 +80,17 @@ struct GemmArgs {
 
 template <int BN>
 struct TcCfg {
-  static constexpr int A_BYTES = kTile * kBK * 2;              // 16 KB weight tile
+  static constexpr int A_BYTES = kTile * kBK * 2;              // 16 KB per 128-row weight subtile
   static constexpr int B_BYTES = BN * kBK * 2;                 // one activation half (hi or lo)
-  static constexpr int STAGE = A_BYTES + 2 * B_BYTES;
-  static constexpr int S_RAW = (200 * 1024) / STAGE;
-  static constexpr int S = S_RAW > 8 ? 8 : S_RAW;
-  static constexpr int NCOLS = (2 * BN) < 32 ? 32 : 2 * BN;    // two accumulators, power of two
+  static constexpr int STAGE = kSub * A_BYTES + 2 * B_BYTES;
   static constexpr int BAR_BYTES = 256;
   static constexpr int EPI_BYTES = kMaxT * 4 + 64;             // input RMSNorm factors, flags
   static constexpr int RED_BYTES = 4 * BN * 12 + BN * 12;      // argmax cross-warp scratch + running state
-  static constexpr int SMEM = 1024 /*align slack*/ + S * STAGE + BAR_BYTES + EPI_BYTES + RED_BYTES;
+  static constexpr int FIXED = 1024 /*align slack*/ + BAR_BYTES + EPI_BYTES + RED_BYTES;
+  static constexpr int S_RAW = (227 * 1024 - FIXED) / STAGE;
+  static constexpr int S = S_RAW > 8 ? 8 : S_RAW;
+  static constexpr int NCOLS = (2 * kSub * BN) < 32 ? 32 : 2 * kSub * BN;   // 2 buffers x kSub accumulators
+  static constexpr int SMEM = FIXED + S * STAGE;
 };
 
 struct Top2s {
@@ -105,8 +113,8 @@ OOS_DEV Top2s t2_merge(Top2s a, Top2s b) {
 
 OOS_DEV void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
-// Finishing a tile: warp w of the four epilogue warps owns token rows
-// t = t0 + 4k + w, lane l owns the four features 4l..4l+3 of the tile, so a
+// Finishing a subtile: warp w of the four epilogue warps owns token rows
+// t = t0 + 4k + w, lane l owns the four features 4l..4l+3 of the subtile, so a
 // token's 128 features sit in one warp (RMSNorm sums, q/k norm and the RoPE
 // pair exchange are warp shuffles) and every slice load is a coalesced float4.
 // All loads of a pass are issued before any result is stored.
@@ -116,19 +124,20 @@ OOS_DEV float4 f4_add(float4 a, float4 b) { return make_float4(a.x + b.x, a.y + 
 OOS_DEV float4 f4_ldcg(const float* p) { return __ldcg(reinterpret_cast<const float4*>(p)); }
 
 // acc[k] = (init ? init row : 0) + sum over nc slices of the partial tile rows
-OOS_DEV void load_tile_rows(float4 (&acc)[kFinRows], const float* __restrict__ part, int nc, size_t slice, int n_part,
-                            int col, int t0, int T, const float* __restrict__ init, int init_ld) {
+template <int R>
+OOS_DEV void load_tile_rows(float4 (&acc)[R], const float* __restrict__ part, int nc, size_t slice, int n_part,
+                            int col, int t0, int T, const float* __restrict__ init, int init_ld, int init_col) {
   const int w = (threadIdx.x - 64) >> 5;
 #pragma unroll
-  for (int k = 0; k < kFinRows; ++k) {
+  for (int k = 0; k < R; ++k) {
     const int t = t0 + 4 * k + w;
-    acc[k] = (init && t < T) ? *reinterpret_cast<const float4*>(init + (size_t)t * init_ld + col)
+    acc[k] = (init && t < T) ? *reinterpret_cast<const float4*>(init + (size_t)t * init_ld + init_col)
                              : make_float4(0.f, 0.f, 0.f, 0.f);
   }
   for (int sl = 0; sl < nc; ++sl) {
     const float* base = part + (size_t)sl * slice + col;
 #pragma unroll
-    for (int k = 0; k < kFinRows; ++k) {
+    for (int k = 0; k < R; ++k) {
       const int t = t0 + 4 * k + w;
       if (t < T) acc[k] = f4_add(acc[k], f4_ldcg(base + (size_t)t * n_part));
     }
@@ -141,103 +150,102 @@ OOS_DEV float4 bf16x4(const __nv_bfloat16* p) {
   return make_float4(__bfloat162float(h[0]), __bfloat162float(h[1]), __bfloat162float(h[2]), __bfloat162float(h[3]));
 }
 
-template <int EPI>
-OOS_DEV void finish_tile(const GemmArgs& a, int tile, const float* rms) {
-  const int e = threadIdx.x - 64;     // 0..127
-  const int w = e >> 5, l = e & 31;
-  const int n_part = a.n_tiles * kTile;
+// EPI_RESID on 128-row tile `tile`: x += W.a; y = g (.) x; per-tile sums of x^2
+OOS_DEV void finish_resid(const GemmArgs& a, int tile, int nc) {
+  const int e = threadIdx.x - 64, w = e >> 5, l = e & 31;
+  const int n_part = a.n_work * kSub * kTile;
   const size_t slice = (size_t)kMaxT * n_part;
-  StreamK sk{a.n_tiles, a.kbt, a.total, (int)gridDim.x};
-  int c0, c1;
-  if (EPI == EPI_RESID) {
-    // x += W.a; y = g (.) x (next RMSNorm input); per-tile sums of x^2
-    sk.contributors(tile, c0, c1);
-    const int f = tile * kTile + 4 * l;
-    const float4 g = bf16x4(a.gain + f);
-    for (int t0 = 0; t0 < a.T; t0 += 4 * kFinRows) {
-      float4 acc[kFinRows];
-      load_tile_rows(acc, a.part, c1 - c0 + 1, slice, n_part, f, t0, a.T, a.x, a.N);   // x + sum of slices
+  const int f = tile * kTile + 4 * l;
+  const float4 g = bf16x4(a.gain + f);
+  for (int t0 = 0; t0 < a.T; t0 += 4 * kFinRows) {
+    float4 acc[kFinRows];
+    load_tile_rows(acc, a.part, nc, slice, n_part, f, t0, a.T, a.x, a.N, f);   // x + sum of slices
 #pragma unroll
-      for (int k = 0; k < kFinRows; ++k) {
-        const int t = t0 + 4 * k + w;
-        if (t >= a.T) break;
-        const float4 xv = acc[k];
-        *reinterpret_cast<float4*>(a.x + (size_t)t * a.N + f) = xv;
-        store_act4(a.y_out, (size_t)t * a.N + f, (size_t)kMaxT * a.N,
-                   make_float4(g.x * xv.x, g.y * xv.y, g.z * xv.z, g.w * xv.w));
-        const float sq = warp_sum(xv.x * xv.x + xv.y * xv.y + xv.z * xv.z + xv.w * xv.w);
-        if (l == 0) a.ss_out[(size_t)tile * kMaxT + t] = sq;
-      }
+    for (int k = 0; k < kFinRows; ++k) {
+      const int t = t0 + 4 * k + w;
+      if (t >= a.T) break;
+      const float4 xv = acc[k];
+      *reinterpret_cast<float4*>(a.x + (size_t)t * a.N + f) = xv;
+      store_act4(a.y_out, (size_t)t * a.N + f, (size_t)kMaxT * a.N,
+                 make_float4(g.x * xv.x, g.y * xv.y, g.z * xv.z, g.w * xv.w));
+      const float sq = warp_sum(xv.x * xv.x + xv.y * xv.y + xv.z * xv.z + xv.w * xv.w);
+      if (l == 0) a.ss_out[(size_t)tile * kMaxT + t] = sq;
     }
-  } else if (EPI == EPI_SILU) {
-    // act = silu(r g) * (r u) for the 128 features of gate/up pair tile/2
-    const int pr = tile >> 1;
-    int u0, u1;
-    sk.contributors(2 * pr, c0, c1);
-    sk.contributors(2 * pr + 1, u0, u1);
-    const int i = pr * kTile + 4 * l;
-    for (int t0 = 0; t0 < a.T; t0 += 4 * kFinRows) {
-      float4 gv[kFinRows], uv[kFinRows];
-      load_tile_rows(gv, a.part, c1 - c0 + 1, slice, n_part, 2 * pr * kTile + 4 * l, t0, a.T, nullptr, 0);
-      load_tile_rows(uv, a.part, u1 - u0 + 1, slice, n_part, (2 * pr + 1) * kTile + 4 * l, t0, a.T, nullptr, 0);
+  }
+}
+
+// EPI_SILU on work tile wt: subtile 0 = gate rows of block wt, subtile 1 = up rows
+OOS_DEV void finish_silu(const GemmArgs& a, int wt, int nc, const float* rms) {
+  const int e = threadIdx.x - 64, w = e >> 5, l = e & 31;
+  const int n_part = a.n_work * kSub * kTile;
+  const size_t slice = (size_t)kMaxT * n_part;
+  const int i = wt * kTile + 4 * l;
+  constexpr int R = kFinRows / 2;   // two row sets live at once: half the rows per pass
+  for (int t0 = 0; t0 < a.T; t0 += 4 * R) {
+    float4 gv[R], uv[R];
+    load_tile_rows(gv, a.part, nc, slice, n_part, 2 * wt * kTile + 4 * l, t0, a.T, nullptr, 0, 0);
+    load_tile_rows(uv, a.part, nc, slice, n_part, (2 * wt + 1) * kTile + 4 * l, t0, a.T, nullptr, 0, 0);
 #pragma unroll
-      for (int k = 0; k < kFinRows; ++k) {
-        const int t = t0 + 4 * k + w;
-        if (t >= a.T) break;
-        const float r = rms[t];
-        const float g4[4] = {gv[k].x * r, gv[k].y * r, gv[k].z * r, gv[k].w * r};
-        const float u4[4] = {uv[k].x * r, uv[k].y * r, uv[k].z * r, uv[k].w * r};
-        float o4[4];
+    for (int k = 0; k < R; ++k) {
+      const int t = t0 + 4 * k + w;
+      if (t >= a.T) break;
+      const float r = rms[t];
+      const float g4[4] = {gv[k].x * r, gv[k].y * r, gv[k].z * r, gv[k].w * r};
+      const float u4[4] = {uv[k].x * r, uv[k].y * r, uv[k].z * r, uv[k].w * r};
+      float o4[4];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) o4[c] = g4[c] / (1.f + expf(-g4[c])) * u4[c];
-        store_act4(a.act_out, (size_t)t * a.I + i, (size_t)kMaxT * a.I, make_float4(o4[0], o4[1], o4[2], o4[3]));
-      }
+      for (int c = 0; c < 4; ++c) o4[c] = g4[c] / (1.f + expf(-g4[c])) * u4[c];
+      store_act4(a.act_out, (size_t)t * a.I + i, (size_t)kMaxT * a.I, make_float4(o4[0], o4[1], o4[2], o4[3]));
     }
-  } else {
-    // EPI_QKV: tile = one head of 128 features (q heads, then k heads, then v heads)
-    sk.contributors(tile, c0, c1);
-    int kind, h;
-    if (tile < a.nq) { kind = 0; h = tile; }
-    else if (tile < a.nq + a.nkv) { kind = 1; h = tile - a.nq; }
-    else { kind = 2; h = tile - a.nq - a.nkv; }
-    const __nv_bfloat16* bias = kind == 0 ? a.bq : kind == 1 ? a.bk : a.bv;
-    const __nv_bfloat16* gn = kind == 0 ? a.gq : kind == 1 ? a.gk : nullptr;
-    const float4 b4 = bias ? bf16x4(bias + h * kTile + 4 * l) : make_float4(0.f, 0.f, 0.f, 0.f);
-    const float4 g4 = gn ? bf16x4(gn + 4 * l) : make_float4(1.f, 1.f, 1.f, 1.f);
-    const int m0 = 4 * (l & 15);      // rotary frequency index of this lane's first feature
-    const bool first_half = l < 16;   // features 0..63 pair with 64..127 held by lane ^ 16
-    for (int t0 = 0; t0 < a.T; t0 += 4 * kFinRows) {
-      float4 acc[kFinRows];
-      load_tile_rows(acc, a.part, c1 - c0 + 1, slice, n_part, tile * kTile + 4 * l, t0, a.T, nullptr, 0);
+  }
+}
+
+// EPI_QKV on 128-row tile `tile` = one head (q heads, then k heads, then v heads)
+OOS_DEV void finish_qkv(const GemmArgs& a, int tile, int nc, const float* rms) {
+  const int e = threadIdx.x - 64, w = e >> 5, l = e & 31;
+  const int n_part = a.n_work * kSub * kTile;
+  const size_t slice = (size_t)kMaxT * n_part;
+  int kind, h;
+  if (tile < a.nq) { kind = 0; h = tile; }
+  else if (tile < a.nq + a.nkv) { kind = 1; h = tile - a.nq; }
+  else { kind = 2; h = tile - a.nq - a.nkv; }
+  const __nv_bfloat16* bias = kind == 0 ? a.bq : kind == 1 ? a.bk : a.bv;
+  const __nv_bfloat16* gn = kind == 0 ? a.gq : kind == 1 ? a.gk : nullptr;
+  const float4 b4 = bias ? bf16x4(bias + h * kTile + 4 * l) : make_float4(0.f, 0.f, 0.f, 0.f);
+  const float4 g4 = gn ? bf16x4(gn + 4 * l) : make_float4(1.f, 1.f, 1.f, 1.f);
+  const int m0 = 4 * (l & 15);      // rotary frequency index of this lane's first feature
+  const bool first_half = l < 16;   // features 0..63 pair with 64..127 held by lane ^ 16
+  for (int t0 = 0; t0 < a.T; t0 += 4 * kFinRows) {
+    float4 acc[kFinRows];
+    load_tile_rows(acc, a.part, nc, slice, n_part, tile * kTile + 4 * l, t0, a.T, nullptr, 0, 0);
 #pragma unroll
-      for (int k = 0; k < kFinRows; ++k) {
-        const int t = t0 + 4 * k + w;
-        if (t >= a.T) break;
-        const float r = rms[t];
-        float v[4] = {acc[k].x * r + b4.x, acc[k].y * r + b4.y, acc[k].z * r + b4.z, acc[k].w * r + b4.w};
-        if (gn) {   // per-head RMSNorm over the head's 128 features
-          const float ss = warp_sum(v[0] * v[0] + v[1] * v[1] + v[2] * v[2] + v[3] * v[3]);
-          const float rn = rsqrtf(ss * (1.f / kTile) + a.eps);
-          v[0] *= rn * g4.x;
-          v[1] *= rn * g4.y;
-          v[2] *= rn * g4.z;
-          v[3] *= rn * g4.w;
-        }
-        if (kind < 2) {   // rotate-half RoPE at position ctx + depth(t)
-#pragma unroll
-          for (int c = 0; c < 4; ++c) {
-            const float other = __shfl_xor_sync(0xffffffffu, v[c], 16);
-            const float2 cs = a.rope[t * (kTile / 2) + m0 + c];
-            v[c] = first_half ? v[c] * cs.x - other * cs.y : v[c] * cs.x + other * cs.y;
-          }
-        }
-        __nv_bfloat16* dst = kind == 0 ? a.q_out + ((size_t)t * a.nq + h) * kTile
-                                       : (kind == 1 ? a.kc : a.vc) + ((size_t)(a.ctx + t) * a.nkv + h) * kTile;
-        __nv_bfloat16 o[4];
-#pragma unroll
-        for (int c = 0; c < 4; ++c) o[c] = __float2bfloat16_rn(v[c]);
-        *reinterpret_cast<uint2*>(dst + 4 * l) = *reinterpret_cast<const uint2*>(o);
+    for (int k = 0; k < kFinRows; ++k) {
+      const int t = t0 + 4 * k + w;
+      if (t >= a.T) break;
+      const float r = rms[t];
+      float v[4] = {acc[k].x * r + b4.x, acc[k].y * r + b4.y, acc[k].z * r + b4.z, acc[k].w * r + b4.w};
+      if (gn) {   // per-head RMSNorm over the head's 128 features
+        const float ss = warp_sum(v[0] * v[0] + v[1] * v[1] + v[2] * v[2] + v[3] * v[3]);
+        const float rn = rsqrtf(ss * (1.f / kTile) + a.eps);
+        v[0] *= rn * g4.x;
+        v[1] *= rn * g4.y;
+        v[2] *= rn * g4.z;
+        v[3] *= rn * g4.w;
       }
+      if (kind < 2) {   // rotate-half RoPE at position ctx + depth(t)
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const float other = __shfl_xor_sync(0xffffffffu, v[c], 16);
+          const float2 cs = a.rope[t * (kTile / 2) + m0 + c];
+          v[c] = first_half ? v[c] * cs.x - other * cs.y : v[c] * cs.x + other * cs.y;
+        }
+      }
+      __nv_bfloat16* dst = kind == 0 ? a.q_out + ((size_t)t * a.nq + h) * kTile
+                                     : (kind == 1 ? a.kc : a.vc) + ((size_t)(a.ctx + t) * a.nkv + h) * kTile;
+      __nv_bfloat16 o[4];
+#pragma unroll
+      for (int c = 0; c < 4; ++c) o[c] = __float2bfloat16_rn(v[c]);
+      *reinterpret_cast<uint2*>(dst + 4 * l) = *reinterpret_cast<const uint2*>(o);
     }
   }
 }
@@ -251,8 +259,7 @@ __global__ void __launch_bounds__(192, 1)
   constexpr bool ARGMAX = EPI == EPI_ARGMAX;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* smem = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-  unsigned char* sA = smem;
-  unsigned char* sB = smem + S * C::A_BYTES;      // [stage][hi|lo][BN rows x 128 B]
+  // stage layout: [A subtile 0 | A subtile 1 | B hi | B lo]
   uint64_t* full = reinterpret_cast<uint64_t*>(smem + S * C::STAGE);
   uint64_t* empty = full + S;
   uint64_t* accf = empty + S;
@@ -268,24 +275,24 @@ __global__ void __launch_bounds__(192, 1)
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = gridDim.x, cta = blockIdx.x;
 
-  // this CTA's work: units [u0, u1) (stream-K) or tiles cta, cta+G, ... (LM head)
+  // this CTA's work: units [u0, u1) (stream-K) or work tiles cta, cta+G, ... (LM head)
   long long u0, u1;
   if (!ARGMAX) {
     u0 = (long long)cta * a.total / G;
     u1 = (long long)(cta + 1) * a.total / G;
   } else {
-    const int my_tiles = cta < a.n_tiles ? (a.n_tiles - cta + G - 1) / G : 0;
+    const int my_tiles = cta < a.n_work ? (a.n_work - cta + G - 1) / G : 0;
     u0 = 0;
     u1 = (long long)my_tiles * a.kbt;
   }
   const int n_units = (int)(u1 - u0);
-  auto unit_tile = [&](int j, int& tile, int& kb) {
+  auto unit_tile = [&](int j, int& wt, int& kb) {
     if (!ARGMAX) {
       const long long u = u0 + j;
-      tile = (int)(u / a.kbt);
+      wt = (int)(u / a.kbt);
       kb = (int)(u % a.kbt);
     } else {
-      tile = cta + (j / a.kbt) * G;
+      wt = cta + (j / a.kbt) * G;
       kb = j % a.kbt;
     }
   };
@@ -321,28 +328,33 @@ __global__ void __launch_bounds__(192, 1)
       const uint64_t pol_w = policy_evict_first();
       const uint64_t pol_a = policy_evict_last();
       auto load_w = [&](int j, int stage) {
-        int tile, kb;
-        unit_tile(j, tile, kb);
-        const CUtensorMap* wm = &wm0;
-        int row = tile * kTile;
-        if (a.interleave2) {
-          wm = (tile & 1) ? &wm1 : &wm0;
-          row = (tile >> 1) * kTile;
-        } else if (tile >= a.seg_tiles[0]) {
-          if (tile >= a.seg_tiles[1]) {
-            wm = &wm2;
-            row = (tile - a.seg_tiles[1]) * kTile;
-          } else {
-            wm = &wm1;
-            row = (tile - a.seg_tiles[0]) * kTile;
+        int wt, kb;
+        unit_tile(j, wt, kb);
+#pragma unroll
+        for (int sub = 0; sub < kSub; ++sub) {
+          const int tile = wt * kSub + sub;          // 128-row tile of the stacked weight
+          const CUtensorMap* wm = &wm0;
+          int row = tile * kTile;
+          if (a.interleave2) {
+            wm = (tile & 1) ? &wm1 : &wm0;
+            row = (tile >> 1) * kTile;
+          } else if (tile >= a.seg_tiles[0]) {
+            if (tile >= a.seg_tiles[1]) {
+              wm = &wm2;
+              row = (tile - a.seg_tiles[1]) * kTile;
+            } else {
+              wm = &wm1;
+              row = (tile - a.seg_tiles[0]) * kTile;
+            }
           }
+          // a subtile past the last weight row reads zeros (TMA out-of-bounds fill)
+          tma_load_2d(smem + stage * C::STAGE + sub * C::A_BYTES, wm, &full[stage], kb * kBK, row, pol_w);
         }
-        tma_load_2d(sA + stage * C::A_BYTES, wm, &full[stage], kb * kBK, row, pol_w);
       };
       auto load_x = [&](int j, int stage) {
-        int tile, kb;
-        unit_tile(j, tile, kb);
-        unsigned char* dst = sB + stage * 2 * C::B_BYTES;
+        int wt, kb;
+        unit_tile(j, wt, kb);
+        unsigned char* dst = smem + stage * C::STAGE + kSub * C::A_BYTES;
         tma_load_2d(dst, &am, &full[stage], kb * kBK, 0, pol_a);                   // hi rows
         tma_load_2d(dst + C::B_BYTES, &am, &full[stage], kb * kBK, kMaxT, pol_a);  // lo rows
       };
@@ -390,26 +402,31 @@ __global__ void __launch_bounds__(192, 1)
       int j = 0;
       bool ok = true;
       while (j < n_units && ok) {
-        int tile, kb;
-        unit_tile(j, tile, kb);
-        int seg_end = j + (a.kbt - kb);       // units of this tile owned here
+        int wt, kb;
+        unit_tile(j, wt, kb);
+        int seg_end = j + (a.kbt - kb);       // units of this work tile owned here
         if (seg_end > n_units) seg_end = n_units;
         if (!mbar_wait(&acce[acc], (acc_use[acc] & 1u) ^ 1u, abort_flag, a.status)) break;
         tc_fence_after();
-        const uint32_t d_tmem = tmem_base + (uint32_t)(acc * BN);
+        const uint32_t d0 = tmem_base + (uint32_t)(acc * kSub * BN);
         for (int jj = j; jj < seg_end; ++jj) {
           if (!mbar_wait(&full[stage], phase, abort_flag, a.status)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint64_t ad = smem_desc_sw128(smem_addr(sA + stage * C::A_BYTES));
-          const uint64_t bh = smem_desc_sw128(smem_addr(sB + stage * 2 * C::B_BYTES));
-          const uint64_t bl = smem_desc_sw128(smem_addr(sB + stage * 2 * C::B_BYTES + C::B_BYTES));
+          const uint32_t sbase = smem_addr(smem + stage * C::STAGE);
+          const uint64_t bh = smem_desc_sw128(sbase + kSub * C::A_BYTES);
+          const uint64_t bl = smem_desc_sw128(sbase + kSub * C::A_BYTES + C::B_BYTES);
 #pragma unroll
           for (int k = 0; k < kBK / 16; ++k) {
-            tc_mma_bf16(d_tmem, ad + 2 * k, bh + 2 * k, idesc, (jj > j || k > 0) ? 1u : 0u);
-            tc_mma_bf16(d_tmem, ad + 2 * k, bl + 2 * k, idesc, 1u);
+#pragma unroll
+            for (int sub = 0; sub < kSub; ++sub) {
+              const uint64_t ad = smem_desc_sw128(sbase + sub * C::A_BYTES);
+              const uint32_t d = d0 + (uint32_t)(sub * BN);
+              tc_mma_bf16(d, ad + 2 * k, bh + 2 * k, idesc, (jj > j || k > 0) ? 1u : 0u);
+              tc_mma_bf16(d, ad + 2 * k, bl + 2 * k, idesc, 1u);
+            }
           }
           tc_commit(&empty[stage]);
           if (++stage == S) {
@@ -443,79 +460,91 @@ __global__ void __launch_bounds__(192, 1)
       }
       epi_bar();
     }
-    const int n_part = a.n_tiles * kTile;
+    const int n_part = a.n_work * kSub * kTile;
     int acc = 0;
     uint32_t acc_use[2] = {0, 0};
     int j = 0;
     while (j < n_units) {
-      int tile, kb;
-      unit_tile(j, tile, kb);
+      int wt, kb;
+      unit_tile(j, wt, kb);
       int seg_end = j + (a.kbt - kb);
       if (seg_end > n_units) seg_end = n_units;
       if (!mbar_wait(&accf[acc], acc_use[acc] & 1u, abort_flag, a.status)) break;
       tc_fence_after();
-      const uint32_t taddr = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * BN);
+      const uint32_t taddr0 = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kSub * BN);
       if (!ARGMAX) {
         int c0, c1;
-        StreamK sk{a.n_tiles, a.kbt, a.total, G};
-        sk.contributors(tile, c0, c1);
-        float* dst = a.part + (size_t)(cta - c0) * kMaxT * n_part + (size_t)tile * kTile + row;
+        StreamK sk{a.n_work, a.kbt, a.total, G};
+        sk.contributors(wt, c0, c1);
 #pragma unroll 1
-        for (int cc = 0; cc < BN / 16; ++cc) {
-          if (cc * 16 >= a.T) break;
-          float v[16];
-          tmem_ld16(taddr + cc * 16, v);
+        for (int sub = 0; sub < kSub; ++sub) {
+          float* dst = a.part + (size_t)(cta - c0) * kMaxT * n_part + (size_t)(wt * kSub + sub) * kTile + row;
+#pragma unroll 1
+          for (int cc = 0; cc < BN / 16; ++cc) {
+            if (cc * 16 >= a.T) break;
+            float v[16];
+            tmem_ld16(taddr0 + sub * BN + cc * 16, v);
 #pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            const int t = cc * 16 + i;
-            if (t < a.T) dst[(size_t)t * n_part] = v[i];
+            for (int i = 0; i < 16; ++i) {
+              const int t = cc * 16 + i;
+              if (t < a.T) dst[(size_t)t * n_part] = v[i];
+            }
           }
         }
-        // accumulator drained: hand the TMEM buffer back to the MMA issuer
+        // accumulators drained: hand the TMEM buffer back to the MMA issuer
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&acce[acc]);
-        // arrival: the last contributor of the tile (or gate/up pair) finishes it
+        // arrival: the last contributor of the work tile finishes it
         __threadfence();
         epi_bar();
         if (e == 0) {
-          int expected = c1 - c0 + 1;
-          int ci = tile;
-          if (EPI == EPI_SILU) {
-            int o0, o1;
-            sk.contributors(tile ^ 1, o0, o1);
-            expected += o1 - o0 + 1;
-            ci = tile >> 1;
-          }
-          const int old = atomicAdd(&a.cnt[ci], 1);
-          *s_last = (old == expected - 1);
-          if (old == expected - 1) a.cnt[ci] = 0;   // ready for the next launch
+          const int old = atomicAdd(&a.cnt[wt], 1);
+          *s_last = (old == c1 - c0);
+          if (old == c1 - c0) a.cnt[wt] = 0;   // ready for the next launch
         }
         epi_bar();
         if (*s_last) {
           __threadfence();
-          finish_tile<EPI>(a, tile, rms);
+          const int nc = c1 - c0 + 1;
+          if (EPI == EPI_SILU) {
+            finish_silu(a, wt, nc, rms);
+          } else {
+#pragma unroll 1
+            for (int sub = 0; sub < kSub; ++sub) {
+              const int tile = wt * kSub + sub;
+              if (tile >= a.n_tiles) break;
+              if (EPI == EPI_RESID) finish_resid(a, tile, nc);
+              else finish_qkv(a, tile, nc, rms);
+            }
+          }
         }
         epi_bar();
       } else {
-        const int f = tile * kTile + row;
 #pragma unroll 1
-        for (int cc = 0; cc < BN / 16; ++cc) {
-          if (cc * 16 >= a.T) break;
-          float v[16];
-          tmem_ld16(taddr + cc * 16, v);
+        for (int sub = 0; sub < kSub; ++sub) {
+          const int f = (wt * kSub + sub) * kTile + row;
+#pragma unroll 1
+          for (int cc = 0; cc < BN / 16; ++cc) {
+            if (cc * 16 >= a.T) break;
+            float v[16];
+            tmem_ld16(taddr0 + sub * BN + cc * 16, v);
 #pragma unroll
-          for (int i = 0; i < 16; ++i) {
-            Top2s s{f < a.N ? v[i] * rms[cc * 16 + i] : -INFINITY, f, -INFINITY};
+            for (int i = 0; i < 16; ++i) {
+              Top2s s{f < a.N ? v[i] * rms[cc * 16 + i] : -INFINITY, f, -INFINITY};
 #pragma unroll
-            for (int o = 16; o > 0; o >>= 1) {
-              Top2s y;
-              y.v1 = __shfl_xor_sync(0xffffffffu, s.v1, o);
-              y.i1 = __shfl_xor_sync(0xffffffffu, s.i1, o);
-              y.v2 = __shfl_xor_sync(0xffffffffu, s.v2, o);
-              s = t2_merge(s, y);
+              for (int o = 16; o > 0; o >>= 1) {
+                Top2s y;
+                y.v1 = __shfl_xor_sync(0xffffffffu, s.v1, o);
+                y.i1 = __shfl_xor_sync(0xffffffffu, s.i1, o);
+                y.v2 = __shfl_xor_sync(0xffffffffu, s.v2, o);
+                s = t2_merge(s, y);
+              }
+              if (lane == 0) {
+                Top2s* slot = &red[q * BN + cc * 16 + i];
+                *slot = sub == 0 ? s : t2_merge(*slot, s);
+              }
             }
-            if (lane == 0) red[q * BN + cc * 16 + i] = s;
           }
         }
         tc_fence_before();
@@ -638,7 +667,8 @@ static GemmArgs base_args(Model& m, const GemmW& g, int T, int* cnt) {
   memset(&a, 0, sizeof(a));
   for (int s = 0; s < 3; ++s) a.seg_tiles[s] = g.seg_tiles[s < g.n_seg ? s : g.n_seg - 1];
   a.interleave2 = g.interleave2;
-  a.n_tiles = g.plan.n_tiles;
+  a.n_tiles = (g.N + kTile - 1) / kTile;
+  a.n_work = g.plan.n_tiles;
   a.kbt = g.plan.kbt;
   a.total = g.plan.total;
   a.N = g.N;

@@ -13,7 +13,8 @@
 namespace oos {
 
 constexpr int kMaxT = 128;          // largest tree (ancestor sets are 128-bit masks)
-constexpr int kTile = 128;          // output features per GEMM tile (tcgen05 M)
+constexpr int kTile = 128;          // weight rows per MMA (tcgen05 M)
+constexpr int kWorkRows = 256;      // weight rows per stream-K work tile (two MMA subtiles)
 constexpr int kBK = 64;             // reduction elements per pipeline stage (128 bytes of bf16)
 constexpr int kMaxLayers = 128;
 constexpr int kMaxAttnSplits = 16;  // cache splits of the attention kernel
@@ -51,7 +52,7 @@ struct StreamK {
   }
 };
 
-StreamK make_streamk(int n_rows, int K, int n_sms);
+StreamK make_streamk(int n_rows, int K, int n_sms, int tile_rows);
 StreamK make_single_slice(int n_rows);   // one contributor per tile (CUDA-core GEMM)
 
 // One weight GEMM of the bf16 path: up to three row-stacked segments (q|k|v,

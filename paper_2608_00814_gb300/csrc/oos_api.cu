@@ -17,9 +17,9 @@ namespace oos {
 
 static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
-StreamK make_streamk(int n_rows, int K, int n_sms) {
+StreamK make_streamk(int n_rows, int K, int n_sms, int tile_rows) {
   StreamK p;
-  p.n_tiles = (n_rows + kTile - 1) / kTile;
+  p.n_tiles = (n_rows + tile_rows - 1) / tile_rows;
   p.kbt = K / kBK;
   p.total = p.n_tiles * p.kbt;
   p.grid = std::min(std::min(n_sms, p.total), kMaxGridCTAs);
@@ -36,7 +36,7 @@ StreamK make_single_slice(int n_rows) {
 }
 
 static int lm_grid_for(const oos_model_config& c, int n_sms) {
-  if (c.dtype == OOS_DTYPE_BF16) return std::min(std::min(n_sms, (c.vocab + kTile - 1) / kTile), kMaxGridCTAs);
+  if (c.dtype == OOS_DTYPE_BF16) return std::min(std::min(n_sms, (c.vocab + kWorkRows - 1) / kWorkRows), kMaxGridCTAs);
   return std::max(1, std::min(std::min(2 * n_sms, (c.vocab + 15) / 16), kMaxGridCTAs));
 }
 
@@ -65,9 +65,10 @@ size_t carve_workspace(const oos_model_config& c, int n_sms, uint8_t* base, Work
   size_t pf = 0;
   const int Nq = (int)(qd + 2 * kvd);
   if (c.dtype == OOS_DTYPE_BF16) {
-    const StreamK ps[4] = {make_streamk(Nq, (int)H, n_sms), make_streamk((int)H, (int)qd, n_sms),
-                           make_streamk((int)(2 * I), (int)H, n_sms), make_streamk((int)H, (int)I, n_sms)};
-    for (int i = 0; i < 4; ++i) pf = std::max(pf, (size_t)ps[i].max_slices() * kMaxT * ps[i].n_tiles * kTile);
+    const StreamK ps[4] = {make_streamk(Nq, (int)H, n_sms, kWorkRows), make_streamk((int)H, (int)qd, n_sms, kWorkRows),
+                           make_streamk((int)(2 * I), (int)H, n_sms, kWorkRows),
+                           make_streamk((int)H, (int)I, n_sms, kWorkRows)};
+    for (int i = 0; i < 4; ++i) pf = std::max(pf, (size_t)ps[i].max_slices() * kMaxT * ps[i].n_tiles * kWorkRows);
   } else {
     pf = (size_t)kMaxT * std::max(std::max((size_t)Nq, H), 2 * I);
   }
@@ -109,7 +110,7 @@ static bool shape_supported(const oos_model_config* c) {
   if (c->dtype == OOS_DTYPE_BF16) {
     if (c->head_dim != 128 || c->hidden % 128 || c->intermediate % 128) return false;
     if (c->hidden / 128 > kMaxSsChunks) return false;
-    if (2 * c->intermediate / 128 > kCntStride || (c->n_q_heads + 2 * c->n_kv_heads) > kCntStride) return false;
+    if (2 * c->intermediate / kWorkRows > kCntStride || (c->n_q_heads + 2 * c->n_kv_heads) > kCntStride) return false;
     const int rb = (kMaxT * (c->n_q_heads / c->n_kv_heads) + 63) / 64;
     if (c->n_kv_heads * rb > kAttnCnt) return false;
   }
@@ -317,7 +318,7 @@ int oos_model_create(const oos_model_config* cfg, const oos_weights* w, void* wo
         g.n_seg = nseg;
         g.N = N;
         g.K = K;
-        g.plan = make_streamk(N, K, n_sms);
+        g.plan = make_streamk(N, K, n_sms, kWorkRows);
         return true;
       };
       bool ok = true;
