@@ -66,7 +66,8 @@ extern "C" {
 #define OOS_ECAPACITY (-2)     /* ctx_len + T exceeds the KV cache capacity */
 #define OOS_ECUDA (-3)         /* a CUDA runtime or driver call failed */
 #define OOS_ETREE (-4)         /* parent[] is not a parents-first tree, or a token is outside [0, vocab) */
-#define OOS_ETIMEOUT (-5)      /* a device pipeline wait exceeded its limit; outputs are not valid */
+#define OOS_ETIMEOUT (-5)      /* a device wait exceeded its limit; outputs are not valid and the handle
+                                  must be destroyed and created again */
 #define OOS_EUNSUPPORTED (-6)  /* shape outside what the kernels handle (see oos_model_create) */
 #define OOS_EWORKSPACE (-7)    /* workspace NULL, misaligned (256 B) or smaller than oos_workspace_bytes */
 

@@ -38,21 +38,26 @@ namespace oos {
 // multiplies column t by r_t = rsqrt(sum x_t^2 / H + eps) in its epilogue.
 enum { EPI_QKV = 0, EPI_RESID = 1, EPI_SILU = 2, EPI_ARGMAX = 3 };
 
-// A work tile is kSub = 2 weight subtiles of 128 rows (the MMA's M) that share
-// every staged activation slice: per weight byte, half the activation traffic
-// and more weight bytes in flight than single 128-row tiles.  Subtile s of
-// work tile w is the 128-row tile 2w + s of the stacked weight.
-constexpr int kSub = 2;
+// A work tile is SUB weight subtiles of 128 rows (the MMA's M) that share every
+// staged activation slice.  The gate/up GEMM and the LM head use SUB = 2 (per
+// weight byte half the activation traffic, more weight bytes in flight, and
+// gate + up rows of one block in one CTA); the smaller QKV, O and down GEMMs
+// use SUB = 1 so each tile has fewer stream-K contributors.  Subtile s of work
+// tile w is the 128-row tile SUB*w + s of the stacked weight.
+template <int EPI>
+struct SubOf {
+  static constexpr int v = (EPI == 2 || EPI == 3) ? 2 : 1;
+};
 
 struct GemmArgs {
   int seg_tiles[3];   // cumulative 128-row tile counts per weight segment
   int interleave2;    // 128-row tile 2i -> segment 0 block i, tile 2i+1 -> segment 1 block i
   int n_tiles;        // 128-row tiles of the stacked weight
-  int n_work, kbt, total;   // work tiles (kSub subtiles each), k-blocks per tile, n_work * kbt
+  int n_work, kbt, total;   // work tiles (SUB subtiles each), k-blocks per tile, n_work * kbt
   int N;              // output rows (features / vocab) of the stacked weight
   int T;              // valid columns (tree nodes)
-  float* part;        // partial tiles [slice][kMaxT][n_work * kSub * 128]
-  int* cnt;           // arrival counters per work tile; zero between launches
+  float* part;        // partial tiles [slice][kMaxT][n_work * SUB * 128]
+  int* cnt;           // per work tile: contributions arrived [0, n_work), shares finished [kCntStride, ...)
   uint32_t* status;
   // RMSNorm scale of the GEMM input (EPI_QKV, EPI_SILU, EPI_ARGMAX)
   const float* ss_in;   // [chunk][kMaxT]
@@ -78,7 +83,7 @@ struct GemmArgs {
   float* am_v2;
 };
 
-template <int BN>
+template <int BN, int kSub>
 struct TcCfg {
   static constexpr int A_BYTES = kTile * kBK * 2;              // 16 KB per 128-row weight subtile
   static constexpr int B_BYTES = BN * kBK * 2;                 // one activation half (hi or lo)
@@ -127,6 +132,7 @@ OOS_DEV float4 f4_ldcg(const float* p) { return __ldcg(reinterpret_cast<const fl
 template <int R>
 OOS_DEV void load_tile_rows(float4 (&acc)[R], const float* __restrict__ part, int nc, size_t slice, int n_part,
                             int col, int t0, int T, const float* __restrict__ init, int init_ld, int init_col) {
+  // rows t = t0 + 4k + w, t < T (T here is the end of the token range)
   const int w = (threadIdx.x - 64) >> 5;
 #pragma unroll
   for (int k = 0; k < R; ++k) {
@@ -150,20 +156,20 @@ OOS_DEV float4 bf16x4(const __nv_bfloat16* p) {
   return make_float4(__bfloat162float(h[0]), __bfloat162float(h[1]), __bfloat162float(h[2]), __bfloat162float(h[3]));
 }
 
-// EPI_RESID on 128-row tile `tile`: x += W.a; y = g (.) x; per-tile sums of x^2
-OOS_DEV void finish_resid(const GemmArgs& a, int tile, int nc) {
+// EPI_RESID on 128-row tile `tile`, tokens [tb, te): x += W.a; y = g (.) x;
+// per-tile sums of x^2
+OOS_DEV void finish_resid(const GemmArgs& a, int n_part, int tile, int nc, int tb, int te) {
   const int e = threadIdx.x - 64, w = e >> 5, l = e & 31;
-  const int n_part = a.n_work * kSub * kTile;
   const size_t slice = (size_t)kMaxT * n_part;
   const int f = tile * kTile + 4 * l;
   const float4 g = bf16x4(a.gain + f);
-  for (int t0 = 0; t0 < a.T; t0 += 4 * kFinRows) {
+  for (int t0 = tb; t0 < te; t0 += 4 * kFinRows) {
     float4 acc[kFinRows];
-    load_tile_rows(acc, a.part, nc, slice, n_part, f, t0, a.T, a.x, a.N, f);   // x + sum of slices
+    load_tile_rows(acc, a.part, nc, slice, n_part, f, t0, te, a.x, a.N, f);   // x + sum of slices
 #pragma unroll
     for (int k = 0; k < kFinRows; ++k) {
       const int t = t0 + 4 * k + w;
-      if (t >= a.T) break;
+      if (t >= te) break;
       const float4 xv = acc[k];
       *reinterpret_cast<float4*>(a.x + (size_t)t * a.N + f) = xv;
       store_act4(a.y_out, (size_t)t * a.N + f, (size_t)kMaxT * a.N,
@@ -174,21 +180,21 @@ OOS_DEV void finish_resid(const GemmArgs& a, int tile, int nc) {
   }
 }
 
-// EPI_SILU on work tile wt: subtile 0 = gate rows of block wt, subtile 1 = up rows
-OOS_DEV void finish_silu(const GemmArgs& a, int wt, int nc, const float* rms) {
+// EPI_SILU on work tile wt (subtile 0 = gate rows of block wt, subtile 1 = up
+// rows), tokens [tb, te)
+OOS_DEV void finish_silu(const GemmArgs& a, int n_part, int wt, int nc, const float* rms, int tb, int te) {
   const int e = threadIdx.x - 64, w = e >> 5, l = e & 31;
-  const int n_part = a.n_work * kSub * kTile;
   const size_t slice = (size_t)kMaxT * n_part;
   const int i = wt * kTile + 4 * l;
   constexpr int R = kFinRows / 2;   // two row sets live at once: half the rows per pass
-  for (int t0 = 0; t0 < a.T; t0 += 4 * R) {
+  for (int t0 = tb; t0 < te; t0 += 4 * R) {
     float4 gv[R], uv[R];
-    load_tile_rows(gv, a.part, nc, slice, n_part, 2 * wt * kTile + 4 * l, t0, a.T, nullptr, 0, 0);
-    load_tile_rows(uv, a.part, nc, slice, n_part, (2 * wt + 1) * kTile + 4 * l, t0, a.T, nullptr, 0, 0);
+    load_tile_rows(gv, a.part, nc, slice, n_part, 2 * wt * kTile + 4 * l, t0, te, nullptr, 0, 0);
+    load_tile_rows(uv, a.part, nc, slice, n_part, (2 * wt + 1) * kTile + 4 * l, t0, te, nullptr, 0, 0);
 #pragma unroll
     for (int k = 0; k < R; ++k) {
       const int t = t0 + 4 * k + w;
-      if (t >= a.T) break;
+      if (t >= te) break;
       const float r = rms[t];
       const float g4[4] = {gv[k].x * r, gv[k].y * r, gv[k].z * r, gv[k].w * r};
       const float u4[4] = {uv[k].x * r, uv[k].y * r, uv[k].z * r, uv[k].w * r};
@@ -200,10 +206,10 @@ OOS_DEV void finish_silu(const GemmArgs& a, int wt, int nc, const float* rms) {
   }
 }
 
-// EPI_QKV on 128-row tile `tile` = one head (q heads, then k heads, then v heads)
-OOS_DEV void finish_qkv(const GemmArgs& a, int tile, int nc, const float* rms) {
+// EPI_QKV on 128-row tile `tile` = one head (q heads, then k heads, then v
+// heads), tokens [tb, te)
+OOS_DEV void finish_qkv(const GemmArgs& a, int n_part, int tile, int nc, const float* rms, int tb, int te) {
   const int e = threadIdx.x - 64, w = e >> 5, l = e & 31;
-  const int n_part = a.n_work * kSub * kTile;
   const size_t slice = (size_t)kMaxT * n_part;
   int kind, h;
   if (tile < a.nq) { kind = 0; h = tile; }
@@ -215,13 +221,13 @@ OOS_DEV void finish_qkv(const GemmArgs& a, int tile, int nc, const float* rms) {
   const float4 g4 = gn ? bf16x4(gn + 4 * l) : make_float4(1.f, 1.f, 1.f, 1.f);
   const int m0 = 4 * (l & 15);      // rotary frequency index of this lane's first feature
   const bool first_half = l < 16;   // features 0..63 pair with 64..127 held by lane ^ 16
-  for (int t0 = 0; t0 < a.T; t0 += 4 * kFinRows) {
+  for (int t0 = tb; t0 < te; t0 += 4 * kFinRows) {
     float4 acc[kFinRows];
-    load_tile_rows(acc, a.part, nc, slice, n_part, tile * kTile + 4 * l, t0, a.T, nullptr, 0, 0);
+    load_tile_rows(acc, a.part, nc, slice, n_part, tile * kTile + 4 * l, t0, te, nullptr, 0, 0);
 #pragma unroll
     for (int k = 0; k < kFinRows; ++k) {
       const int t = t0 + 4 * k + w;
-      if (t >= a.T) break;
+      if (t >= te) break;
       const float r = rms[t];
       float v[4] = {acc[k].x * r + b4.x, acc[k].y * r + b4.y, acc[k].z * r + b4.z, acc[k].w * r + b4.w};
       if (gn) {   // per-head RMSNorm over the head's 128 features
@@ -254,7 +260,8 @@ template <int BN, int EPI>
 __global__ void __launch_bounds__(192, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap wm0, const __grid_constant__ CUtensorMap wm1,
               const __grid_constant__ CUtensorMap wm2, const __grid_constant__ CUtensorMap am, GemmArgs a) {
-  using C = TcCfg<BN>;
+  constexpr int kSub = SubOf<EPI>::v;
+  using C = TcCfg<BN, kSub>;
   constexpr int S = C::S;
   constexpr bool ARGMAX = EPI == EPI_ARGMAX;
   extern __shared__ __align__(1024) unsigned char smem_raw[];
@@ -495,31 +502,10 @@ __global__ void __launch_bounds__(192, 1)
         tc_fence_before();
         __syncwarp();
         if (lane == 0) mbar_arrive(&acce[acc]);
-        // arrival: the last contributor of the work tile finishes it
+        // publish this contribution (finished at the end of the range)
         __threadfence();
         epi_bar();
-        if (e == 0) {
-          const int old = atomicAdd(&a.cnt[wt], 1);
-          *s_last = (old == c1 - c0);
-          if (old == c1 - c0) a.cnt[wt] = 0;   // ready for the next launch
-        }
-        epi_bar();
-        if (*s_last) {
-          __threadfence();
-          const int nc = c1 - c0 + 1;
-          if (EPI == EPI_SILU) {
-            finish_silu(a, wt, nc, rms);
-          } else {
-#pragma unroll 1
-            for (int sub = 0; sub < kSub; ++sub) {
-              const int tile = wt * kSub + sub;
-              if (tile >= a.n_tiles) break;
-              if (EPI == EPI_RESID) finish_resid(a, tile, nc);
-              else finish_qkv(a, tile, nc, rms);
-            }
-          }
-        }
-        epi_bar();
+        if (e == 0) atomicAdd(&a.cnt[wt], 1);
       } else {
 #pragma unroll 1
         for (int sub = 0; sub < kSub; ++sub) {
@@ -562,6 +548,63 @@ __global__ void __launch_bounds__(192, 1)
       ++acc_use[acc];
       acc ^= 1;
       j = seg_end;
+    }
+    if (!ARGMAX && !*abort_flag) {
+      // Finish every work tile this CTA touched: once all nc contributions of
+      // the tile have arrived, contributor i (in CTA order) finishes token rows
+      // [T*i/nc, T*(i+1)/nc) -- slices are still added in slice order, so the
+      // result does not depend on who finishes.  All contributors end their
+      // ranges at about the same time (balanced stream-K), and the grid never
+      // exceeds one CTA per SM, so every awaited CTA is resident.
+      StreamK sk{a.n_work, a.kbt, a.total, G};
+      int jj = 0;
+      while (jj < n_units) {
+        int wt, kb;
+        unit_tile(jj, wt, kb);
+        int seg_end = jj + (a.kbt - kb);
+        if (seg_end > n_units) seg_end = n_units;
+        jj = seg_end;
+        int c0, c1;
+        sk.contributors(wt, c0, c1);
+        const int nc = c1 - c0 + 1;
+        if (e == 0) {
+          const unsigned long long t0 = globaltimer();
+          while (atomicAdd(&a.cnt[wt], 0) < nc) {
+            if (globaltimer() - t0 > kWaitLimitNs) {
+              atomicOr(a.status, ST_TIMEOUT);
+              *abort_flag = 1;
+              break;
+            }
+          }
+        }
+        epi_bar();
+        if (*abort_flag) break;
+        __threadfence();
+        const int share = cta - c0;
+        const int tb = (int)((long long)a.T * share / nc), te = (int)((long long)a.T * (share + 1) / nc);
+        if (tb < te) {
+          if (EPI == EPI_SILU) {
+            finish_silu(a, n_part, wt, nc, rms, tb, te);
+          } else {
+#pragma unroll 1
+            for (int sub = 0; sub < kSub; ++sub) {
+              const int tile = wt * kSub + sub;
+              if (tile >= a.n_tiles) break;
+              if (EPI == EPI_RESID) finish_resid(a, n_part, tile, nc, tb, te);
+              else finish_qkv(a, n_part, tile, nc, rms, tb, te);
+            }
+          }
+        }
+        __threadfence();
+        epi_bar();
+        if (e == 0) {
+          // the last share resets both counters of the tile for the next launch
+          if (atomicAdd(&a.cnt[kCntStride + wt], 1) == nc - 1) {
+            a.cnt[wt] = 0;
+            a.cnt[kCntStride + wt] = 0;
+          }
+        }
+      }
     }
     if (ARGMAX && e < a.T) {
       const Top2s r = run[e];
@@ -621,7 +664,8 @@ int bn_index(int T) { return T <= 16 ? 0 : T <= 32 ? 1 : T <= 64 ? 2 : 3; }
 
 template <int BN, int EPI>
 static cudaError_t set_smem() {
-  return cudaFuncSetAttribute(k_gemm_tc<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<BN>::SMEM);
+  return cudaFuncSetAttribute(k_gemm_tc<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                              TcCfg<BN, SubOf<EPI>::v>::SMEM);
 }
 
 template <int BN>
@@ -646,8 +690,8 @@ static cudaError_t launch_tc(Model& m, const GemmW& g, const CUtensorMap& amap, 
                              cudaStream_t st) {
   const CUtensorMap& w1 = g.n_seg > 1 ? g.map[1] : g.map[0];
   const CUtensorMap& w2 = g.n_seg > 2 ? g.map[2] : g.map[0];
-  return launch(m.pdl, k_gemm_tc<BN, EPI>, dim3(grid), dim3(192), (size_t)TcCfg<BN>::SMEM, st, g.map[0], w1, w2,
-                amap, a);
+  return launch(m.pdl, k_gemm_tc<BN, EPI>, dim3(grid), dim3(192), (size_t)TcCfg<BN, SubOf<EPI>::v>::SMEM, st,
+                g.map[0], w1, w2, amap, a);
 }
 
 template <int EPI>
@@ -686,7 +730,7 @@ static GemmArgs base_args(Model& m, const GemmW& g, int T, int* cnt) {
 cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int ctx, int T, cudaStream_t st) {
   const auto& c = m.cfg;
   const oos_layer_weights& L = m.layers[layer];
-  GemmArgs a = base_args(m, m.g_qkv[layer], T, m.ws.cnt + 0 * kCntStride);
+  GemmArgs a = base_args(m, m.g_qkv[layer], T, m.ws.cnt + 0 * 2 * kCntStride);
   a.nq = c.n_q_heads;
   a.nkv = c.n_kv_heads;
   a.bq = (const __nv_bfloat16*)(c.qkv_bias ? L.b_q : nullptr);
@@ -713,16 +757,16 @@ static cudaError_t launch_resid(Model& m, const GemmW& g, const CUtensorMap* ama
 }
 
 cudaError_t launch_gemm_o(Model& m, int layer, int T, cudaStream_t st) {
-  return launch_resid(m, m.g_o[layer], m.amap_attn, m.layers[layer].mlp_norm, m.ws.cnt + 1 * kCntStride, T, st);
+  return launch_resid(m, m.g_o[layer], m.amap_attn, m.layers[layer].mlp_norm, m.ws.cnt + 1 * 2 * kCntStride, T, st);
 }
 
 cudaError_t launch_gemm_down(Model& m, int layer, int T, cudaStream_t st) {
   const void* gain = layer + 1 < m.cfg.n_layers ? m.layers[layer + 1].attn_norm : m.w.final_norm;
-  return launch_resid(m, m.g_down[layer], m.amap_act, gain, m.ws.cnt + 3 * kCntStride, T, st);
+  return launch_resid(m, m.g_down[layer], m.amap_act, gain, m.ws.cnt + 3 * 2 * kCntStride, T, st);
 }
 
 cudaError_t launch_gemm_gu(Model& m, int layer, int T, cudaStream_t st) {
-  GemmArgs a = base_args(m, m.g_gu[layer], T, m.ws.cnt + 2 * kCntStride);
+  GemmArgs a = base_args(m, m.g_gu[layer], T, m.ws.cnt + 2 * 2 * kCntStride);
   a.act_out = (__nv_bfloat16*)m.ws.act;
   a.I = m.cfg.intermediate;
   return dispatch_tc<EPI_SILU>(m, m.g_gu[layer], m.amap_xn, T, m.g_gu[layer].plan.grid, a, st);

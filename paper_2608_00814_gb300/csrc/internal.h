@@ -14,7 +14,7 @@ namespace oos {
 
 constexpr int kMaxT = 128;          // largest tree (ancestor sets are 128-bit masks)
 constexpr int kTile = 128;          // weight rows per MMA (tcgen05 M)
-constexpr int kWorkRows = 256;      // weight rows per stream-K work tile (two MMA subtiles)
+constexpr int kWorkRowsWide = 256;  // weight rows per work tile of the gate/up GEMM and LM head
 constexpr int kBK = 64;             // reduction elements per pipeline stage (128 bytes of bf16)
 constexpr int kMaxLayers = 128;
 constexpr int kMaxAttnSplits = 16;  // cache splits of the attention kernel
@@ -90,7 +90,7 @@ struct Workspace {
   float* top2;
   float* ss;                 // sum of x^2 per 128-feature chunk [kMaxSsChunks][kMaxT] (bf16 path)
   float2* rope;              // (cos, sin) per node and rotary pair [kMaxT][d/2] (bf16 path)
-  int* cnt;                  // GEMM arrival counters [4][kCntStride]
+  int* cnt;                  // GEMM counters [4 kinds][arrived | finished][kCntStride]
   int* attn_cnt;             // attention split arrival counters [kAttnCnt]
 };
 

@@ -36,7 +36,8 @@ StreamK make_single_slice(int n_rows) {
 }
 
 static int lm_grid_for(const oos_model_config& c, int n_sms) {
-  if (c.dtype == OOS_DTYPE_BF16) return std::min(std::min(n_sms, (c.vocab + kWorkRows - 1) / kWorkRows), kMaxGridCTAs);
+  if (c.dtype == OOS_DTYPE_BF16)
+    return std::min(std::min(n_sms, (c.vocab + kWorkRowsWide - 1) / kWorkRowsWide), kMaxGridCTAs);
   return std::max(1, std::min(std::min(2 * n_sms, (c.vocab + 15) / 16), kMaxGridCTAs));
 }
 
@@ -65,10 +66,11 @@ size_t carve_workspace(const oos_model_config& c, int n_sms, uint8_t* base, Work
   size_t pf = 0;
   const int Nq = (int)(qd + 2 * kvd);
   if (c.dtype == OOS_DTYPE_BF16) {
-    const StreamK ps[4] = {make_streamk(Nq, (int)H, n_sms, kWorkRows), make_streamk((int)H, (int)qd, n_sms, kWorkRows),
-                           make_streamk((int)(2 * I), (int)H, n_sms, kWorkRows),
-                           make_streamk((int)H, (int)I, n_sms, kWorkRows)};
-    for (int i = 0; i < 4; ++i) pf = std::max(pf, (size_t)ps[i].max_slices() * kMaxT * ps[i].n_tiles * kWorkRows);
+    const int rows[4] = {kTile, kTile, kWorkRowsWide, kTile};
+    const StreamK ps[4] = {make_streamk(Nq, (int)H, n_sms, rows[0]), make_streamk((int)H, (int)qd, n_sms, rows[1]),
+                           make_streamk((int)(2 * I), (int)H, n_sms, rows[2]),
+                           make_streamk((int)H, (int)I, n_sms, rows[3])};
+    for (int i = 0; i < 4; ++i) pf = std::max(pf, (size_t)ps[i].max_slices() * kMaxT * ps[i].n_tiles * rows[i]);
   } else {
     pf = (size_t)kMaxT * std::max(std::max((size_t)Nq, H), 2 * I);
   }
@@ -88,7 +90,7 @@ size_t carve_workspace(const oos_model_config& c, int n_sms, uint8_t* base, Work
   w.top2 = (float*)take(kMaxT * 4);
   w.ss = (float*)take((size_t)kMaxSsChunks * kMaxT * 4);
   w.rope = (float2*)take((size_t)kMaxT * (c.head_dim / 2) * 8);
-  w.cnt = (int*)take((size_t)4 * kCntStride * 4);
+  w.cnt = (int*)take((size_t)4 * 2 * kCntStride * 4);
   w.attn_cnt = (int*)take((size_t)kAttnCnt * 4);
   if (ws) *ws = w;
   return align_up(off, 256);
@@ -110,7 +112,9 @@ static bool shape_supported(const oos_model_config* c) {
   if (c->dtype == OOS_DTYPE_BF16) {
     if (c->head_dim != 128 || c->hidden % 128 || c->intermediate % 128) return false;
     if (c->hidden / 128 > kMaxSsChunks) return false;
-    if (2 * c->intermediate / kWorkRows > kCntStride || (c->n_q_heads + 2 * c->n_kv_heads) > kCntStride) return false;
+    if (2 * c->intermediate / kWorkRowsWide > kCntStride || (c->n_q_heads + 2 * c->n_kv_heads) > kCntStride ||
+        c->hidden / kTile > kCntStride)
+      return false;
     const int rb = (kMaxT * (c->n_q_heads / c->n_kv_heads) + 63) / 64;
     if (c->n_kv_heads * rb > kAttnCnt) return false;
   }
@@ -303,7 +307,8 @@ int oos_model_create(const oos_model_config* cfg, const oos_weights* w, void* wo
     const int H = c.hidden, I = c.intermediate, qd = c.n_q_heads * c.head_dim, kvd = c.n_kv_heads * c.head_dim;
     m->lm_grid = lm_grid_for(c, n_sms);
     if (c.dtype == OOS_DTYPE_BF16) {
-      auto mk = [&](GemmW& g, const void* const* ptrs, const int* rows, int nseg, int K, int interleave) -> bool {
+      auto mk = [&](GemmW& g, const void* const* ptrs, const int* rows, int nseg, int K, int interleave,
+                    int tile_rows) -> bool {
         memset(&g, 0, sizeof(g));
         g.interleave2 = interleave;
         int tiles = 0, N = 0;
@@ -318,7 +323,7 @@ int oos_model_create(const oos_model_config* cfg, const oos_weights* w, void* wo
         g.n_seg = nseg;
         g.N = N;
         g.K = K;
-        g.plan = make_streamk(N, K, n_sms, kWorkRows);
+        g.plan = make_streamk(N, K, n_sms, tile_rows);
         return true;
       };
       bool ok = true;
@@ -336,12 +341,12 @@ int oos_model_create(const oos_model_config* cfg, const oos_weights* w, void* wo
         const int rg[2] = {I, I};
         const void* pd[1] = {L.w_down};
         const int rd[1] = {H};
-        ok = mk(m->g_qkv[l], pq, rq, 3, H, 0) && mk(m->g_o[l], po, ro, 1, qd, 0) && mk(m->g_gu[l], pg, rg, 2, H, 1) &&
-             mk(m->g_down[l], pd, rd, 1, I, 0);
+        ok = mk(m->g_qkv[l], pq, rq, 3, H, 0, kTile) && mk(m->g_o[l], po, ro, 1, qd, 0, kTile) &&
+             mk(m->g_gu[l], pg, rg, 2, H, 1, kWorkRowsWide) && mk(m->g_down[l], pd, rd, 1, I, 0, kTile);
       }
       const void* pl[1] = {c.vocab ? w->lm_head : nullptr};
       const int rl[1] = {c.vocab};
-      ok = ok && mk(m->g_lm, pl, rl, 1, H, 0);
+      ok = ok && mk(m->g_lm, pl, rl, 1, H, 0, kWorkRowsWide);
       const int boxes[4] = {16, 32, 64, 128};
       for (int b = 0; b < 4 && ok; ++b)
         ok = encode_act_map(&m->amap_xn[b], m->ws.xn, H, boxes[b]) &&
