@@ -21,7 +21,16 @@ from synth import gen, trees
 from synth.configs import TINY
 from synth.model import SynthModel
 
-torch.set_default_dtype(torch.float64)
+
+
+@pytest.fixture(autouse=True)
+def _float64_default():
+    """fp64 torch defaults for these pins only (restored afterwards, so other
+    test modules keep torch's float32 default)."""
+    prev = torch.get_default_dtype()
+    torch.set_default_dtype(torch.float64)
+    yield
+    torch.set_default_dtype(prev)
 
 
 # ------------------------------------------------------------------ tree shape
