@@ -216,6 +216,30 @@ int oos_accept_walk(const int32_t* tree_tokens, const int32_t* tree_parent, cons
 #define OOS_STAGE_LM_HEAD 4
 int oos_launch_stage(oos_model* m, int32_t layer, int32_t stage, int32_t T, void* stream);
 
+/* LM-head greedy argmax that allocates nothing.  The paper has no counterpart:
+ * this entry point exists for callers that cannot allocate device memory at
+ * all -- code running inside someone else's CUDA-graph capture, under a memory
+ * pool or allocator it does not own, or in a process whose allocator is locked
+ * -- and so cannot provide the workspace oos_model_create needs.
+ *   hidden      DEVICE float [T, hidden_dim]: final-RMSNorm rows (for example
+ *               out_final_hidden of oos_tree_verify_debug).
+ *   lm_head     DEVICE [vocab, hidden_dim], element type `dtype`.
+ *   out_argmax  DEVICE int32 [T]: argmax_v hidden[t] . lm_head[v] (Eq. 1; ties
+ *               to the lowest id); out_top1 / out_top2 DEVICE float [T]: the
+ *               largest and second-largest logit.
+ * Scratch: a fixed 0.8 MB array in the library's device memory (allocated when
+ * the library is loaded, held on every GPU that loads it until exit) holds the
+ * per-block partial results; T must be <= 128, larger T returns OOS_EINVAL.
+ * The first call on a device looks up that array's address (a one-time set-up
+ * per device): make it before any stream capture.  Every call shares the
+ * array, so calls that may overlap on the GPU (different streams, different
+ * host threads) race and must be serialised by the caller.  CUDA cores only; a
+ * correctness and portability path, not the fused tensor-core LM head of
+ * oos_tree_verify. */
+int oos_lm_head_argmax_static(int32_t dtype, int32_t vocab, int32_t hidden_dim, const void* lm_head,
+                              const float* hidden, int32_t T, int32_t* out_argmax, float* out_top1,
+                              float* out_top2, void* stream);
+
 /* Synchronise `stream` and return the device status of the last verify on
  * this handle: OOS_OK, OOS_ETREE or OOS_ETIMEOUT (or OOS_ECUDA). */
 int oos_last_status(oos_model* m, void* stream);

@@ -79,6 +79,8 @@ def lib():
         L.oos_last_status.argtypes = [c_vp, c_vp]
         L.oos_launch_stage.argtypes = [c_vp, c_i32, c_i32, c_i32, c_vp]
         L.oos_launch_stage.restype = ctypes.c_int
+        L.oos_lm_head_argmax_static.argtypes = [c_i32, c_i32, c_i32, c_vp, c_vp, c_i32, c_vp, c_vp, c_vp, c_vp]
+        L.oos_lm_head_argmax_static.restype = ctypes.c_int
         L.oos_status_string.argtypes = [ctypes.c_int]
         L.oos_status_string.restype = ctypes.c_char_p
         for fn in ("oos_model_create", "oos_model_destroy", "oos_tree_verify", "oos_tree_verify_debug",
@@ -220,6 +222,14 @@ OOS_STAGE_QKV, OOS_STAGE_O, OOS_STAGE_GATE_UP, OOS_STAGE_DOWN, OOS_STAGE_LM_HEAD
 
 def oos_launch_stage(model, layer, stage, T, stream=None):
     _check(lib().oos_launch_stage(model.handle, layer, stage, T, _stream(stream)), "oos_launch_stage")
+
+
+def oos_lm_head_argmax_static(dtype, vocab, hidden_dim, lm_head, hidden, T, out_argmax, out_top1, out_top2,
+                              stream=None):
+    """LM-head greedy argmax that allocates no device memory (see include/oos.h)."""
+    _check(lib().oos_lm_head_argmax_static(dtype, vocab, hidden_dim, _ptr(lm_head), _ptr(hidden), T, _ptr(out_argmax),
+                                           _ptr(out_top1), _ptr(out_top2), _stream(stream)),
+           "oos_lm_head_argmax_static")
 
 
 def oos_last_status(model, stream=None):
