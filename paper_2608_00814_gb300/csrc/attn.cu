@@ -356,17 +356,28 @@ __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
       const int r = rb * kAttnRows + warp + 4 * i;
       grow[i] = r < R ? (r / a.group) * a.nq + g * a.group + r % a.group : -1;
     }
-    for (int sp = 0; sp < a.splits; ++sp) {
-      const float* src = a.o_part + (size_t)sp * rows_total * kAttnD + 4 * lane;
+    // splits two at a time: all loads of a pair are issued before any is used
+    for (int sp0 = 0; sp0 < a.splits; sp0 += 2) {
+      float4 v[2][RW];
 #pragma unroll
-      for (int i = 0; i < RW; ++i) {
-        if (grow[i] >= 0) {
-          const float4 v = __ldcg(reinterpret_cast<const float4*>(src + (size_t)grow[i] * kAttnD));
-          const float wgt = s_w[warp + 4 * i][sp];
-          acc[i].x += wgt * v.x;
-          acc[i].y += wgt * v.y;
-          acc[i].z += wgt * v.z;
-          acc[i].w += wgt * v.w;
+      for (int q = 0; q < 2; ++q) {
+        const float* src = a.o_part + (size_t)(sp0 + q) * rows_total * kAttnD + 4 * lane;
+#pragma unroll
+        for (int i = 0; i < RW; ++i)
+          v[q][i] = (sp0 + q < a.splits && grow[i] >= 0)
+                        ? __ldcg(reinterpret_cast<const float4*>(src + (size_t)grow[i] * kAttnD))
+                        : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int q = 0; q < 2; ++q) {
+        if (sp0 + q >= a.splits) break;
+#pragma unroll
+        for (int i = 0; i < RW; ++i) {
+          const float wgt = s_w[warp + 4 * i][sp0 + q];
+          acc[i].x += wgt * v[q][i].x;
+          acc[i].y += wgt * v[q][i].y;
+          acc[i].z += wgt * v[q][i].z;
+          acc[i].w += wgt * v[q][i].w;
         }
       }
     }

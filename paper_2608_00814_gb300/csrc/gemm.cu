@@ -123,16 +123,18 @@ OOS_DEV void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 // token's 128 features sit in one warp (RMSNorm sums, q/k norm and the RoPE
 // pair exchange are warp shuffles) and every slice load is a coalesced float4.
 // All loads of a pass are issued before any result is stored.
-constexpr int kFinRows = 16;   // token rows per warp per pass (64 tokens per pass)
+constexpr int kFinRows = 8;    // token rows per warp per pass (32 tokens per pass)
 
 OOS_DEV float4 f4_add(float4 a, float4 b) { return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w); }
 OOS_DEV float4 f4_ldcg(const float* p) { return __ldcg(reinterpret_cast<const float4*>(p)); }
 
-// acc[k] = (init ? init row : 0) + sum over nc slices of the partial tile rows
+// acc[k] = (init ? init row : 0) + sum over nc slices of the partial tile rows,
+// rows t = t0 + 4k + w below T (the end of the token range).  Slices are
+// fetched four at a time -- every load of a group is issued before any is
+// added -- and added in slice order, so the sum is the same for every finisher.
 template <int R>
 OOS_DEV void load_tile_rows(float4 (&acc)[R], const float* __restrict__ part, int nc, size_t slice, int n_part,
                             int col, int t0, int T, const float* __restrict__ init, int init_ld, int init_col) {
-  // rows t = t0 + 4k + w, t < T (T here is the end of the token range)
   const int w = (threadIdx.x - 64) >> 5;
 #pragma unroll
   for (int k = 0; k < R; ++k) {
@@ -140,13 +142,21 @@ OOS_DEV void load_tile_rows(float4 (&acc)[R], const float* __restrict__ part, in
     acc[k] = (init && t < T) ? *reinterpret_cast<const float4*>(init + (size_t)t * init_ld + init_col)
                              : make_float4(0.f, 0.f, 0.f, 0.f);
   }
-  for (int sl = 0; sl < nc; ++sl) {
-    const float* base = part + (size_t)sl * slice + col;
+  for (int s0 = 0; s0 < nc; s0 += 4) {
+    float4 v[4][R];
 #pragma unroll
-    for (int k = 0; k < R; ++k) {
-      const int t = t0 + 4 * k + w;
-      if (t < T) acc[k] = f4_add(acc[k], f4_ldcg(base + (size_t)t * n_part));
+    for (int q = 0; q < 4; ++q) {
+      const float* base = part + (size_t)(s0 + q) * slice + col;
+#pragma unroll
+      for (int k = 0; k < R; ++k) {
+        const int t = t0 + 4 * k + w;
+        v[q][k] = (s0 + q < nc && t < T) ? f4_ldcg(base + (size_t)t * n_part) : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
     }
+#pragma unroll
+    for (int q = 0; q < 4; ++q)
+#pragma unroll
+      for (int k = 0; k < R; ++k) acc[k] = f4_add(acc[k], v[q][k]);
   }
 }
 
@@ -186,7 +196,7 @@ OOS_DEV void finish_silu(const GemmArgs& a, int n_part, int wt, int nc, const fl
   const int e = threadIdx.x - 64, w = e >> 5, l = e & 31;
   const size_t slice = (size_t)kMaxT * n_part;
   const int i = wt * kTile + 4 * l;
-  constexpr int R = kFinRows / 2;   // two row sets live at once: half the rows per pass
+  constexpr int R = kFinRows / 2;   // two row sets (gate, up) live at once: half the rows per pass
   for (int t0 = tb; t0 < te; t0 += 4 * R) {
     float4 gv[R], uv[R];
     load_tile_rows(gv, a.part, nc, slice, n_part, 2 * wt * kTile + 4 * l, t0, te, nullptr, 0, 0);
@@ -275,7 +285,6 @@ __global__ void __launch_bounds__(192, 1)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(drain + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   float* rms = reinterpret_cast<float*>(smem + S * C::STAGE + C::BAR_BYTES);       // [kMaxT]
-  volatile int* s_last = reinterpret_cast<volatile int*>(rms + kMaxT);
   Top2s* red = reinterpret_cast<Top2s*>(smem + S * C::STAGE + C::BAR_BYTES + C::EPI_BYTES);   // [4][BN]
   Top2s* run = red + 4 * BN;                                                                   // [BN]
 
