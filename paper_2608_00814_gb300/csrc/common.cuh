@@ -159,6 +159,13 @@ OOS_DEV void tma_load_2d(void* smem_dst, const void* tmap, uint64_t* bar, int x,
       : "memory");
 }
 
+// L2 prefetch of one 2-D box (no shared-memory destination, no completion)
+OOS_DEV void tma_prefetch_l2(const void* tmap, int x, int y) {
+  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(reinterpret_cast<uint64_t>(tmap)),
+               "r"(x), "r"(y)
+               : "memory");
+}
+
 // ---- tcgen05 (5th-generation tensor cores, accumulators in TMEM)
 OOS_DEV void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
 OOS_DEV void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }

@@ -57,7 +57,7 @@ struct GemmArgs {
   int N;              // output rows (features / vocab) of the stacked weight
   int T;              // valid columns (tree nodes)
   float* part;        // partial tiles [slice][kMaxT][n_work * SUB * 128]
-  int* cnt;           // per work tile: contributions arrived [0, n_work), shares finished [kCntStride, ...)
+  int* cnt;           // arrival counter per work tile (zeroed at every step start)
   uint32_t* status;
   // RMSNorm scale of the GEMM input (EPI_QKV, EPI_SILU, EPI_ARGMAX)
   const float* ss_in;   // [chunk][kMaxT]
@@ -81,6 +81,10 @@ struct GemmArgs {
   float* am_v1;
   int32_t* am_i;
   float* am_v2;
+  // L2 prefetch, during this GEMM's tail, of the next weight GEMM's first units
+  int pf_units;       // units per CTA of the next GEMM (0: no prefetch)
+  int pf_n_tiles, pf_n_work, pf_kbt, pf_total, pf_grid, pf_sub, pf_interleave, pf_round_robin;
+  int pf_seg_tiles[3];
 };
 
 template <int BN, int kSub>
@@ -123,16 +127,16 @@ OOS_DEV void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 // token's 128 features sit in one warp (RMSNorm sums, q/k norm and the RoPE
 // pair exchange are warp shuffles) and every slice load is a coalesced float4.
 // All loads of a pass are issued before any result is stored.
-constexpr int kFinRows = 8;    // token rows per warp per pass (32 tokens per pass)
+constexpr int kFinRows = 4;    // token rows per warp per pass (16 tokens per pass)
 
 OOS_DEV float4 f4_add(float4 a, float4 b) { return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w); }
 OOS_DEV float4 f4_ldcg(const float* p) { return __ldcg(reinterpret_cast<const float4*>(p)); }
 
 // acc[k] = (init ? init row : 0) + sum over nc slices of the partial tile rows,
 // rows t = t0 + 4k + w below T (the end of the token range).  Slices are
-// fetched four at a time -- every load of a group is issued before any is
+// fetched BATCH at a time -- every load of a group is issued before any is
 // added -- and added in slice order, so the sum is the same for every finisher.
-template <int R>
+template <int R, int BATCH>
 OOS_DEV void load_tile_rows(float4 (&acc)[R], const float* __restrict__ part, int nc, size_t slice, int n_part,
                             int col, int t0, int T, const float* __restrict__ init, int init_ld, int init_col) {
   const int w = (threadIdx.x - 64) >> 5;
@@ -142,10 +146,10 @@ OOS_DEV void load_tile_rows(float4 (&acc)[R], const float* __restrict__ part, in
     acc[k] = (init && t < T) ? *reinterpret_cast<const float4*>(init + (size_t)t * init_ld + init_col)
                              : make_float4(0.f, 0.f, 0.f, 0.f);
   }
-  for (int s0 = 0; s0 < nc; s0 += 4) {
-    float4 v[4][R];
+  for (int s0 = 0; s0 < nc; s0 += BATCH) {
+    float4 v[BATCH][R];
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
+    for (int q = 0; q < BATCH; ++q) {
       const float* base = part + (size_t)(s0 + q) * slice + col;
 #pragma unroll
       for (int k = 0; k < R; ++k) {
@@ -154,7 +158,7 @@ OOS_DEV void load_tile_rows(float4 (&acc)[R], const float* __restrict__ part, in
       }
     }
 #pragma unroll
-    for (int q = 0; q < 4; ++q)
+    for (int q = 0; q < BATCH; ++q)
 #pragma unroll
       for (int k = 0; k < R; ++k) acc[k] = f4_add(acc[k], v[q][k]);
   }
@@ -175,7 +179,7 @@ OOS_DEV void finish_resid(const GemmArgs& a, int n_part, int tile, int nc, int t
   const float4 g = bf16x4(a.gain + f);
   for (int t0 = tb; t0 < te; t0 += 4 * kFinRows) {
     float4 acc[kFinRows];
-    load_tile_rows(acc, a.part, nc, slice, n_part, f, t0, te, a.x, a.N, f);   // x + sum of slices
+    load_tile_rows<kFinRows, 8>(acc, a.part, nc, slice, n_part, f, t0, te, a.x, a.N, f);   // x + sum of slices
 #pragma unroll
     for (int k = 0; k < kFinRows; ++k) {
       const int t = t0 + 4 * k + w;
@@ -196,11 +200,11 @@ OOS_DEV void finish_silu(const GemmArgs& a, int n_part, int wt, int nc, const fl
   const int e = threadIdx.x - 64, w = e >> 5, l = e & 31;
   const size_t slice = (size_t)kMaxT * n_part;
   const int i = wt * kTile + 4 * l;
-  constexpr int R = kFinRows / 2;   // two row sets (gate, up) live at once: half the rows per pass
+  constexpr int R = 8;   // gate and up row sets, 32 tokens per pass, slices four at a time
   for (int t0 = tb; t0 < te; t0 += 4 * R) {
     float4 gv[R], uv[R];
-    load_tile_rows(gv, a.part, nc, slice, n_part, 2 * wt * kTile + 4 * l, t0, te, nullptr, 0, 0);
-    load_tile_rows(uv, a.part, nc, slice, n_part, (2 * wt + 1) * kTile + 4 * l, t0, te, nullptr, 0, 0);
+    load_tile_rows<R, 4>(gv, a.part, nc, slice, n_part, 2 * wt * kTile + 4 * l, t0, te, nullptr, 0, 0);
+    load_tile_rows<R, 4>(uv, a.part, nc, slice, n_part, (2 * wt + 1) * kTile + 4 * l, t0, te, nullptr, 0, 0);
 #pragma unroll
     for (int k = 0; k < R; ++k) {
       const int t = t0 + 4 * k + w;
@@ -233,7 +237,7 @@ OOS_DEV void finish_qkv(const GemmArgs& a, int n_part, int tile, int nc, const f
   const bool first_half = l < 16;   // features 0..63 pair with 64..127 held by lane ^ 16
   for (int t0 = tb; t0 < te; t0 += 4 * kFinRows) {
     float4 acc[kFinRows];
-    load_tile_rows(acc, a.part, nc, slice, n_part, tile * kTile + 4 * l, t0, te, nullptr, 0, 0);
+    load_tile_rows<kFinRows, 8>(acc, a.part, nc, slice, n_part, tile * kTile + 4 * l, t0, te, nullptr, 0, 0);
 #pragma unroll
     for (int k = 0; k < kFinRows; ++k) {
       const int t = t0 + 4 * k + w;
@@ -269,7 +273,9 @@ OOS_DEV void finish_qkv(const GemmArgs& a, int n_part, int tile, int nc, const f
 template <int BN, int EPI>
 __global__ void __launch_bounds__(192, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap wm0, const __grid_constant__ CUtensorMap wm1,
-              const __grid_constant__ CUtensorMap wm2, const __grid_constant__ CUtensorMap am, GemmArgs a) {
+              const __grid_constant__ CUtensorMap wm2, const __grid_constant__ CUtensorMap am,
+              const __grid_constant__ CUtensorMap pm0, const __grid_constant__ CUtensorMap pm1,
+              const __grid_constant__ CUtensorMap pm2, GemmArgs a) {
   constexpr int kSub = SubOf<EPI>::v;
   using C = TcCfg<BN, kSub>;
   constexpr int S = C::S;
@@ -395,6 +401,38 @@ __global__ void __launch_bounds__(192, 1)
         if (++stage == S) {
           stage = 0;
           phase ^= 1u;
+        }
+      }
+      if (!*abort_flag && a.pf_units > 0) {
+        // HBM goes idle during this GEMM's tail (reductions in L2): warm L2
+        // with the first units the next weight GEMM's CTAs will stream
+        for (int c2 = cta; c2 < a.pf_grid; c2 += G) {
+          const long long v0 = a.pf_round_robin ? 0 : (long long)c2 * a.pf_total / a.pf_grid;
+          const long long v1 = a.pf_round_robin ? (long long)a.pf_units : (long long)(c2 + 1) * a.pf_total / a.pf_grid;
+          for (long long v = v0; v < v1 && v < v0 + a.pf_units; ++v) {
+            const int wt = a.pf_round_robin ? c2 + (int)(v / a.pf_kbt) * a.pf_grid : (int)(v / a.pf_kbt);
+            const int kb = (int)(v % a.pf_kbt);
+            if (wt >= a.pf_n_work) break;
+            for (int sub = 0; sub < a.pf_sub; ++sub) {
+              const int tile = wt * a.pf_sub + sub;
+              if (tile >= a.pf_n_tiles) break;
+              const CUtensorMap* pm = &pm0;
+              int row = tile * kTile;
+              if (a.pf_interleave) {
+                pm = (tile & 1) ? &pm1 : &pm0;
+                row = (tile >> 1) * kTile;
+              } else if (tile >= a.pf_seg_tiles[0]) {
+                if (tile >= a.pf_seg_tiles[1]) {
+                  pm = &pm2;
+                  row = (tile - a.pf_seg_tiles[1]) * kTile;
+                } else {
+                  pm = &pm1;
+                  row = (tile - a.pf_seg_tiles[0]) * kTile;
+                }
+              }
+              tma_prefetch_l2(pm, kb * kBK, row);
+            }
+          }
         }
       }
       if (*abort_flag) {
@@ -578,7 +616,7 @@ __global__ void __launch_bounds__(192, 1)
         const int nc = c1 - c0 + 1;
         if (e == 0) {
           const unsigned long long t0 = globaltimer();
-          while (atomicAdd(&a.cnt[wt], 0) < nc) {
+          while (*(volatile int*)&a.cnt[wt] < nc) {
             if (globaltimer() - t0 > kWaitLimitNs) {
               atomicOr(a.status, ST_TIMEOUT);
               *abort_flag = 1;
@@ -602,15 +640,6 @@ __global__ void __launch_bounds__(192, 1)
               if (EPI == EPI_RESID) finish_resid(a, n_part, tile, nc, tb, te);
               else finish_qkv(a, n_part, tile, nc, rms, tb, te);
             }
-          }
-        }
-        __threadfence();
-        epi_bar();
-        if (e == 0) {
-          // the last share resets both counters of the tile for the next launch
-          if (atomicAdd(&a.cnt[kCntStride + wt], 1) == nc - 1) {
-            a.cnt[wt] = 0;
-            a.cnt[kCntStride + wt] = 0;
           }
         }
       }
@@ -696,24 +725,42 @@ cudaError_t gemm_setup() {
 
 template <int BN, int EPI>
 static cudaError_t launch_tc(Model& m, const GemmW& g, const CUtensorMap& amap, int grid, const GemmArgs& a,
-                             cudaStream_t st) {
+                             const GemmW* next, cudaStream_t st) {
   const CUtensorMap& w1 = g.n_seg > 1 ? g.map[1] : g.map[0];
   const CUtensorMap& w2 = g.n_seg > 2 ? g.map[2] : g.map[0];
+  const GemmW& p = next ? *next : g;
+  const CUtensorMap& p1 = p.n_seg > 1 ? p.map[1] : p.map[0];
+  const CUtensorMap& p2 = p.n_seg > 2 ? p.map[2] : p.map[0];
   return launch(m.pdl, k_gemm_tc<BN, EPI>, dim3(grid), dim3(192), (size_t)TcCfg<BN, SubOf<EPI>::v>::SMEM, st,
-                g.map[0], w1, w2, amap, a);
+                g.map[0], w1, w2, amap, p.map[0], p1, p2, a);
 }
 
 template <int EPI>
-static cudaError_t dispatch_tc(Model& m, const GemmW& g, const CUtensorMap* amaps, int T, int grid, const GemmArgs& a,
-                               cudaStream_t st) {
+static cudaError_t dispatch_tc(Model& m, const GemmW& g, const CUtensorMap* amaps, int T, int grid, GemmArgs& a,
+                               const GemmW* next, cudaStream_t st) {
+  if (next) {
+    // about 128 KB of the next GEMM's weights per CTA index
+    a.pf_units = 8 / next->sub;
+    a.pf_n_tiles = (next->N + kTile - 1) / kTile;
+    a.pf_n_work = next->plan.n_tiles;
+    a.pf_kbt = next->plan.kbt;
+    a.pf_total = next->plan.total;
+    a.pf_grid = next->plan.grid;
+    a.pf_sub = next->sub;
+    a.pf_interleave = next->interleave2;
+    a.pf_round_robin = next->round_robin;
+    for (int s = 0; s < 3; ++s) a.pf_seg_tiles[s] = next->seg_tiles[s < next->n_seg ? s : next->n_seg - 1];
+  }
   const int bi = bn_index(T);
   switch (bi) {
-    case 0: return launch_tc<16, EPI>(m, g, amaps[0], grid, a, st);
-    case 1: return launch_tc<32, EPI>(m, g, amaps[1], grid, a, st);
-    case 2: return launch_tc<64, EPI>(m, g, amaps[2], grid, a, st);
-    default: return launch_tc<128, EPI>(m, g, amaps[3], grid, a, st);
+    case 0: return launch_tc<16, EPI>(m, g, amaps[0], grid, a, next, st);
+    case 1: return launch_tc<32, EPI>(m, g, amaps[1], grid, a, next, st);
+    case 2: return launch_tc<64, EPI>(m, g, amaps[2], grid, a, next, st);
+    default: return launch_tc<128, EPI>(m, g, amaps[3], grid, a, next, st);
   }
 }
+
+int* gemm_counters(Model& m, int layer, int kind) { return m.ws.cnt + ((size_t)layer * 4 + kind) * kCntPer; }
 
 static GemmArgs base_args(Model& m, const GemmW& g, int T, int* cnt) {
   GemmArgs a;
@@ -736,10 +783,11 @@ static GemmArgs base_args(Model& m, const GemmW& g, int T, int* cnt) {
   return a;
 }
 
-cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int ctx, int T, cudaStream_t st) {
+cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int ctx, int T, const GemmW* next,
+                            cudaStream_t st) {
   const auto& c = m.cfg;
   const oos_layer_weights& L = m.layers[layer];
-  GemmArgs a = base_args(m, m.g_qkv[layer], T, m.ws.cnt + 0 * 2 * kCntStride);
+  GemmArgs a = base_args(m, m.g_qkv[layer], T, gemm_counters(m, layer, 0));
   a.nq = c.n_q_heads;
   a.nkv = c.n_kv_heads;
   a.bq = (const __nv_bfloat16*)(c.qkv_bias ? L.b_q : nullptr);
@@ -752,33 +800,34 @@ cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int ctx, in
   a.kc = (__nv_bfloat16*)kc;
   a.vc = (__nv_bfloat16*)vc;
   a.ctx = ctx;
-  return dispatch_tc<EPI_QKV>(m, m.g_qkv[layer], m.amap_xn, T, m.g_qkv[layer].plan.grid, a, st);
+  return dispatch_tc<EPI_QKV>(m, m.g_qkv[layer], m.amap_xn, T, m.g_qkv[layer].plan.grid, a, next, st);
 }
 
 static cudaError_t launch_resid(Model& m, const GemmW& g, const CUtensorMap* amaps, const void* gain, int* cnt, int T,
-                                cudaStream_t st) {
+                                const GemmW* next, cudaStream_t st) {
   GemmArgs a = base_args(m, g, T, cnt);
   a.x = m.ws.x;
   a.gain = (const __nv_bfloat16*)gain;
   a.y_out = (__nv_bfloat16*)m.ws.xn;
   a.ss_out = m.ws.ss;
-  return dispatch_tc<EPI_RESID>(m, g, amaps, T, g.plan.grid, a, st);
+  return dispatch_tc<EPI_RESID>(m, g, amaps, T, g.plan.grid, a, next, st);
 }
 
-cudaError_t launch_gemm_o(Model& m, int layer, int T, cudaStream_t st) {
-  return launch_resid(m, m.g_o[layer], m.amap_attn, m.layers[layer].mlp_norm, m.ws.cnt + 1 * 2 * kCntStride, T, st);
+cudaError_t launch_gemm_o(Model& m, int layer, int T, const GemmW* next, cudaStream_t st) {
+  return launch_resid(m, m.g_o[layer], m.amap_attn, m.layers[layer].mlp_norm, gemm_counters(m, layer, 1), T, next,
+                      st);
 }
 
-cudaError_t launch_gemm_down(Model& m, int layer, int T, cudaStream_t st) {
+cudaError_t launch_gemm_down(Model& m, int layer, int T, const GemmW* next, cudaStream_t st) {
   const void* gain = layer + 1 < m.cfg.n_layers ? m.layers[layer + 1].attn_norm : m.w.final_norm;
-  return launch_resid(m, m.g_down[layer], m.amap_act, gain, m.ws.cnt + 3 * 2 * kCntStride, T, st);
+  return launch_resid(m, m.g_down[layer], m.amap_act, gain, gemm_counters(m, layer, 3), T, next, st);
 }
 
-cudaError_t launch_gemm_gu(Model& m, int layer, int T, cudaStream_t st) {
-  GemmArgs a = base_args(m, m.g_gu[layer], T, m.ws.cnt + 2 * 2 * kCntStride);
+cudaError_t launch_gemm_gu(Model& m, int layer, int T, const GemmW* next, cudaStream_t st) {
+  GemmArgs a = base_args(m, m.g_gu[layer], T, gemm_counters(m, layer, 2));
   a.act_out = (__nv_bfloat16*)m.ws.act;
   a.I = m.cfg.intermediate;
-  return dispatch_tc<EPI_SILU>(m, m.g_gu[layer], m.amap_xn, T, m.g_gu[layer].plan.grid, a, st);
+  return dispatch_tc<EPI_SILU>(m, m.g_gu[layer], m.amap_xn, T, m.g_gu[layer].plan.grid, a, next, st);
 }
 
 cudaError_t launch_lm_head_tc(Model& m, int T, cudaStream_t st) {
@@ -786,7 +835,7 @@ cudaError_t launch_lm_head_tc(Model& m, int T, cudaStream_t st) {
   a.am_v1 = m.ws.lm_v1;
   a.am_i = m.ws.lm_i;
   a.am_v2 = m.ws.lm_v2;
-  return dispatch_tc<EPI_ARGMAX>(m, m.g_lm, m.amap_xn, T, m.lm_grid, a, st);
+  return dispatch_tc<EPI_ARGMAX>(m, m.g_lm, m.amap_xn, T, m.lm_grid, a, nullptr, st);
 }
 
 // ------------------------------------------------------------ fp32 CUDA-core path

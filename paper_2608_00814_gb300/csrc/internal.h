@@ -21,7 +21,7 @@ constexpr int kMaxAttnSplits = 16;  // cache splits of the attention kernel
 constexpr int kAttnCnt = 4096;      // attention arrival counters (kv heads x row blocks)
 constexpr int kMaxGridCTAs = 1024;  // upper bound on CTAs of a stream-K GEMM / LM head
 constexpr int kMaxSsChunks = 64;    // hidden <= 8192: RMSNorm partial sums per 128 features
-constexpr int kCntStride = 1024;    // arrival counters per GEMM kind (tiles or gate/up pairs)
+constexpr int kCntPer = 256;        // arrival counters per (layer, GEMM kind): one per work tile
 
 // Stream-K partition of a weight GEMM: the (tile, k-block) units of all tiles,
 // tile-major, are cut into `grid` contiguous equal ranges, one per CTA.  CTA c
@@ -63,6 +63,8 @@ struct GemmW {
   int seg_tiles[3];   // cumulative tile counts at the end of each segment
   int n_seg;
   int interleave2;    // gate/up: tiles alternate between the two segments
+  int sub;            // 128-row MMA subtiles per stream-K work tile (1 or 2)
+  int round_robin;    // LM head: whole work tiles dealt round-robin instead of stream-K
   int N, K;
   StreamK plan;
 };
@@ -90,7 +92,7 @@ struct Workspace {
   float* top2;
   float* ss;                 // sum of x^2 per 128-feature chunk [kMaxSsChunks][kMaxT] (bf16 path)
   float2* rope;              // (cos, sin) per node and rotary pair [kMaxT][d/2] (bf16 path)
-  int* cnt;                  // GEMM counters [4 kinds][arrived | finished][kCntStride]
+  int* cnt;                  // GEMM arrival counters [layer][4 kinds][kCntPer], zeroed at every step start
   int* attn_cnt;             // attention split arrival counters [kAttnCnt]
 };
 
@@ -175,11 +177,14 @@ bool encode_weight_map(CUtensorMap* map, const void* ptr, int rows, int K);
 bool encode_act_map(CUtensorMap* map, const void* ptr, int K, int box_rows);
 int bn_index(int T);   // N-tile variant for T tree nodes: 0..3 -> 16/32/64/128
 cudaError_t gemm_setup();
-cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int ctx, int T, cudaStream_t st);
-cudaError_t launch_gemm_o(Model& m, int layer, int T, cudaStream_t st);
-cudaError_t launch_gemm_gu(Model& m, int layer, int T, cudaStream_t st);
-cudaError_t launch_gemm_down(Model& m, int layer, int T, cudaStream_t st);
+// `next`: the weight GEMM that follows; its first stages are prefetched into L2
+// during this GEMM's tail (nullptr: none)
+cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int ctx, int T, const GemmW* next, cudaStream_t st);
+cudaError_t launch_gemm_o(Model& m, int layer, int T, const GemmW* next, cudaStream_t st);
+cudaError_t launch_gemm_gu(Model& m, int layer, int T, const GemmW* next, cudaStream_t st);
+cudaError_t launch_gemm_down(Model& m, int layer, int T, const GemmW* next, cudaStream_t st);
 cudaError_t launch_lm_head_tc(Model& m, int T, cudaStream_t st);
+int* gemm_counters(Model& m, int layer, int kind);   // kind 0 qkv, 1 o, 2 gate/up, 3 down
 cudaError_t launch_gemm_f32(Model& m, const void* w0, const void* w1, const void* w2, int rows0, int rows1,
                             int rows2, int K, const void* x, int T, cudaStream_t st);
 cudaError_t launch_lm_head_f32(Model& m, int T, cudaStream_t st);

@@ -90,7 +90,7 @@ size_t carve_workspace(const oos_model_config& c, int n_sms, uint8_t* base, Work
   w.top2 = (float*)take(kMaxT * 4);
   w.ss = (float*)take((size_t)kMaxSsChunks * kMaxT * 4);
   w.rope = (float2*)take((size_t)kMaxT * (c.head_dim / 2) * 8);
-  w.cnt = (int*)take((size_t)4 * 2 * kCntStride * 4);
+  w.cnt = (int*)take((size_t)c.n_layers * 4 * kCntPer * 4);
   w.attn_cnt = (int*)take((size_t)kAttnCnt * 4);
   if (ws) *ws = w;
   return align_up(off, 256);
@@ -112,8 +112,8 @@ static bool shape_supported(const oos_model_config* c) {
   if (c->dtype == OOS_DTYPE_BF16) {
     if (c->head_dim != 128 || c->hidden % 128 || c->intermediate % 128) return false;
     if (c->hidden / 128 > kMaxSsChunks) return false;
-    if (2 * c->intermediate / kWorkRowsWide > kCntStride || (c->n_q_heads + 2 * c->n_kv_heads) > kCntStride ||
-        c->hidden / kTile > kCntStride)
+    if (2 * c->intermediate / kWorkRowsWide > kCntPer || (c->n_q_heads + 2 * c->n_kv_heads) > kCntPer ||
+        c->hidden / kTile > kCntPer)
       return false;
     const int rb = (kMaxT * (c->n_q_heads / c->n_kv_heads) + 63) / 64;
     if (c->n_kv_heads * rb > kAttnCnt) return false;
@@ -161,11 +161,12 @@ static int enqueue_verify(Model& m, const oos_kv_cache* kv, int ctx, const int32
     float* hid = (l + 1 < L) ? nullptr : hidden;
     if (c.dtype == OOS_DTYPE_BF16) {
       // five kernels per layer; every elementwise step runs in a GEMM epilogue
-      OOS_TRY(launch_gemm_qkv(m, l, kv->k[l], kv->v[l], ctx, T, st));
+      const GemmW* after_down = (l + 1 < L) ? &m.g_qkv[l + 1] : &m.g_lm;
+      OOS_TRY(launch_gemm_qkv(m, l, kv->k[l], kv->v[l], ctx, T, &m.g_o[l], st));
       OOS_TRY(launch_attention(m, kv->k[l], kv->v[l], ctx, T, st));
-      OOS_TRY(launch_gemm_o(m, l, T, st));
-      OOS_TRY(launch_gemm_gu(m, l, T, st));
-      OOS_TRY(launch_gemm_down(m, l, T, st));
+      OOS_TRY(launch_gemm_o(m, l, T, &m.g_gu[l], st));
+      OOS_TRY(launch_gemm_gu(m, l, T, &m.g_down[l], st));
+      OOS_TRY(launch_gemm_down(m, l, T, after_down, st));
     } else {
       OOS_TRY(launch_gemm_f32(m, W.w_q, W.w_k, W.w_v, qd, kvd, kvd, c.hidden, m.ws.xn, T, st));
       OOS_TRY(launch_qkv_post(m, l, m.p_qkv, kv->k[l], kv->v[l], ctx, T, st));
@@ -324,6 +325,8 @@ int oos_model_create(const oos_model_config* cfg, const oos_weights* w, void* wo
         g.N = N;
         g.K = K;
         g.plan = make_streamk(N, K, n_sms, tile_rows);
+        g.sub = tile_rows / kTile;
+        g.round_robin = 0;
         return true;
       };
       bool ok = true;
@@ -347,6 +350,8 @@ int oos_model_create(const oos_model_config* cfg, const oos_weights* w, void* wo
       const void* pl[1] = {c.vocab ? w->lm_head : nullptr};
       const int rl[1] = {c.vocab};
       ok = ok && mk(m->g_lm, pl, rl, 1, H, 0, kWorkRowsWide);
+      m->g_lm.round_robin = 1;
+      m->g_lm.plan.grid = m->lm_grid;
       const int boxes[4] = {16, 32, 64, 128};
       for (int b = 0; b < 4 && ok; ++b)
         ok = encode_act_map(&m->amap_xn[b], m->ws.xn, H, boxes[b]) &&
@@ -436,9 +441,18 @@ int oos_launch_stage(oos_model* m, int32_t layer, int32_t stage, int32_t T, void
   if (c.dtype == OOS_DTYPE_BF16) {
     switch (stage) {
       case OOS_STAGE_QKV: return OOS_EINVAL;   // its epilogue writes the KV cache
-      case OOS_STAGE_O: e = launch_gemm_o(*m, layer, T, st); break;
-      case OOS_STAGE_GATE_UP: e = launch_gemm_gu(*m, layer, T, st); break;
-      case OOS_STAGE_DOWN: e = launch_gemm_down(*m, layer, T, st); break;
+      case OOS_STAGE_O:
+      case OOS_STAGE_GATE_UP:
+      case OOS_STAGE_DOWN: {
+        // a lone GEMM: its arrival counters start from zero as in a verify step
+        const int kind = stage == OOS_STAGE_O ? 1 : stage == OOS_STAGE_GATE_UP ? 2 : 3;
+        e = cudaMemsetAsync(gemm_counters(*m, layer, kind), 0, kCntPer * sizeof(int), st);
+        if (e != cudaSuccess) break;
+        e = stage == OOS_STAGE_O ? launch_gemm_o(*m, layer, T, nullptr, st)
+            : stage == OOS_STAGE_GATE_UP ? launch_gemm_gu(*m, layer, T, nullptr, st)
+                                         : launch_gemm_down(*m, layer, T, nullptr, st);
+        break;
+      }
       default: e = launch_lm_head_tc(*m, T, st); break;
     }
   } else {

@@ -103,11 +103,15 @@ __global__ void __launch_bounds__(128) k_embed_tc(const int32_t* __restrict__ to
                                                   float* __restrict__ x, __nv_bfloat16* __restrict__ y,
                                                   float* __restrict__ ss, const int32_t* __restrict__ pos,
                                                   const double* __restrict__ inv_freq, int half_d,
-                                                  float2* __restrict__ rope) {
+                                                  float2* __restrict__ rope, int* __restrict__ cnt, int n_cnt) {
   __shared__ float red[32];
   pdl_trigger();
   pdl_wait();
   const int t = blockIdx.x, f = blockIdx.y * 128 + threadIdx.x;
+  {   // the step's GEMM arrival counters start from zero
+    const int nb = gridDim.x * gridDim.y, b = blockIdx.y * gridDim.x + blockIdx.x;
+    for (int i = b * blockDim.x + threadIdx.x; i < n_cnt; i += nb * blockDim.x) cnt[i] = 0;
+  }
   if (blockIdx.y == 0 && threadIdx.x < half_d) {
     const double two_pi = 6.283185307179586476925286766559;
     const double ang = (double)pos[t] * inv_freq[threadIdx.x];
@@ -132,7 +136,7 @@ cudaError_t launch_embed_tc(Model& m, const int32_t* tokens, int T, cudaStream_t
   return launch(m.pdl, k_embed_tc, dim3(T, (c.hidden + 127) / 128), dim3(128), 0, st, tokens,
                 (const __nv_bfloat16*)m.w.embed, (const __nv_bfloat16*)m.layers[0].attn_norm, c.hidden, c.vocab,
                 m.ws.x, (__nv_bfloat16*)m.ws.xn, m.ws.ss, (const int32_t*)m.ws.pos, (const double*)m.ws.inv_freq,
-                c.head_dim / 2, m.ws.rope);
+                c.head_dim / 2, m.ws.rope, m.ws.cnt, c.n_layers * 4 * kCntPer);
 }
 
 // bf16 path, checking output only: the final RMSNorm output in fp32,
