@@ -164,6 +164,36 @@ OOS_DEV void load_tile_rows(float4 (&acc)[R], const float* __restrict__ part, in
   }
 }
 
+// gate (col) and up (col + up_off) rows of a SwiGLU pair, two slices per batch
+template <int R>
+OOS_DEV void load_pair_rows(float4 (&g)[R], float4 (&u)[R], const float* __restrict__ part, int nc, size_t slice,
+                            int n_part, int col, int up_off, int t0, int T) {
+  const int w = (threadIdx.x - 64) >> 5;
+#pragma unroll
+  for (int k = 0; k < R; ++k) g[k] = u[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+  for (int s0 = 0; s0 < nc; s0 += 2) {
+    float4 vg[2][R], vu[2][R];
+#pragma unroll
+    for (int q = 0; q < 2; ++q) {
+      const float* base = part + (size_t)(s0 + q) * slice + col;
+#pragma unroll
+      for (int k = 0; k < R; ++k) {
+        const int t = t0 + 4 * k + w;
+        const bool ok = s0 + q < nc && t < T;
+        vg[q][k] = ok ? f4_ldcg(base + (size_t)t * n_part) : make_float4(0.f, 0.f, 0.f, 0.f);
+        vu[q][k] = ok ? f4_ldcg(base + (size_t)t * n_part + up_off) : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < 2; ++q)
+#pragma unroll
+      for (int k = 0; k < R; ++k) {
+        g[k] = f4_add(g[k], vg[q][k]);
+        u[k] = f4_add(u[k], vu[q][k]);
+      }
+  }
+}
+
 OOS_DEV float4 bf16x4(const __nv_bfloat16* p) {
   const uint2 u = *reinterpret_cast<const uint2*>(p);
   const __nv_bfloat16* h = reinterpret_cast<const __nv_bfloat16*>(&u);
@@ -200,11 +230,11 @@ OOS_DEV void finish_silu(const GemmArgs& a, int n_part, int wt, int nc, const fl
   const int e = threadIdx.x - 64, w = e >> 5, l = e & 31;
   const size_t slice = (size_t)kMaxT * n_part;
   const int i = wt * kTile + 4 * l;
-  constexpr int R = 8;   // gate and up row sets, 32 tokens per pass, slices four at a time
+  constexpr int R = 8;   // 32 tokens per pass
   for (int t0 = tb; t0 < te; t0 += 4 * R) {
     float4 gv[R], uv[R];
-    load_tile_rows<R, 4>(gv, a.part, nc, slice, n_part, 2 * wt * kTile + 4 * l, t0, te, nullptr, 0, 0);
-    load_tile_rows<R, 4>(uv, a.part, nc, slice, n_part, (2 * wt + 1) * kTile + 4 * l, t0, te, nullptr, 0, 0);
+    // gate and up slices of a pass in one batch of loads
+    load_pair_rows<R>(gv, uv, a.part, nc, slice, n_part, 2 * wt * kTile + 4 * l, kTile, t0, te);
 #pragma unroll
     for (int k = 0; k < R; ++k) {
       const int t = t0 + 4 * k + w;

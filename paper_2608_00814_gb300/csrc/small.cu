@@ -403,7 +403,7 @@ OOS_DEV void accept_walk_warp(const int32_t* tokens, const int32_t* parent, cons
   }
 }
 
-__global__ void __launch_bounds__(kMaxT) k_argmax_accept(const float* __restrict__ v1, const int32_t* __restrict__ i1,
+__global__ void __launch_bounds__(1024) k_argmax_accept(const float* __restrict__ v1, const int32_t* __restrict__ i1,
                                                          const float* __restrict__ v2, int n_parts,
                                                          const int32_t* __restrict__ tokens,
                                                          const int32_t* __restrict__ parent,
@@ -415,9 +415,11 @@ __global__ void __launch_bounds__(kMaxT) k_argmax_accept(const float* __restrict
   pdl_trigger();
   pdl_wait();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
-  // the merge is order independent (max with lowest-id ties, multiset second max)
+  // one warp per node (32 warps); the merge is order independent (max with
+  // lowest-id ties, multiset second max), so lanes take CTA states in any order
   for (int t = warp; t < T; t += nw) {
     Top2 r{-INFINITY, 0x7fffffff, -INFINITY};
+#pragma unroll 4
     for (int c = lane; c < n_parts; c += 32) {
       const size_t k = (size_t)c * kMaxT + t;
       r = top2_merge(r, Top2{v1[k], i1[k], v2[k]});
@@ -452,7 +454,7 @@ __global__ void __launch_bounds__(kMaxT) k_argmax_accept(const float* __restrict
 cudaError_t launch_argmax_accept(Model& m, const int32_t* tokens, const int32_t* parent, int T, int n_parts,
                                  int32_t* len, int32_t* nodes, int32_t* toks, int32_t* bonus, int32_t* dbg_argmax,
                                  float* dbg_top1, float* dbg_top2, cudaStream_t st) {
-  return launch(m.pdl, k_argmax_accept, dim3(1), dim3(kMaxT), 0, st, (const float*)m.ws.lm_v1,
+  return launch(m.pdl, k_argmax_accept, dim3(1), dim3(1024), 0, st, (const float*)m.ws.lm_v1,
                 (const int32_t*)m.ws.lm_i, (const float*)m.ws.lm_v2, n_parts, tokens, parent,
                 (const int32_t*)m.ws.depth, (const uint32_t*)m.ws.status, T, m.ws.argmax, m.ws.top1, m.ws.top2,
                 len, nodes, toks, bonus, dbg_argmax, dbg_top1, dbg_top2);
