@@ -203,6 +203,25 @@ def run_reference(args):
     }), flush=True)
 
 
+# ---------------------------------------------------------------- replicas
+
+def reduce_step_time(ms, world, dist=None, device="cuda"):
+    """Step time of the whole job: the maximum over ranks of each rank's
+    device-timed step (replicas exchange nothing else), then a barrier."""
+    if world <= 1:
+        return ms
+    import torch
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.barrier()
+    return float(t.item())
+
+
+def job_throughput(T, ms, world):
+    """Tree tokens verified per second by all ranks together."""
+    return world * T / (ms * 1e-3)
+
+
 # ---------------------------------------------------------------- GPU arm
 
 def run_ours(args):
@@ -267,12 +286,7 @@ def run_ours(args):
     e1.record(stream)
     torch.cuda.synchronize()
     clk = clocks.stop()
-    ms = e0.elapsed_time(e1) / args.steps
-    if world > 1:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-        dist.barrier()
+    ms = reduce_step_time(e0.elapsed_time(e1) / args.steps, world, dist, "cuda")
 
     # ---- end to end through the C ABI with host buffers (pinned), copies inside the timed region
     h_tok = torch.as_tensor(tokens_np, dtype=torch.int32).pin_memory()
@@ -335,7 +349,7 @@ def run_ours(args):
                          % (cfg.n_layers, T, spent, s_est)}
 
     step_b = step_bytes(cfg, ctx, T)
-    value = world * T / (ms * 1e-3)
+    value = job_throughput(T, ms, world)
     launches_per_step = 2 + cfg.n_layers * 5 + 2 + 1   # prep, embed, 5 per layer, LM head, accept, compact
     if rank == 0:
         print(json.dumps({

@@ -319,3 +319,13 @@ def _sampled_check(name):
 
 def test_bf16_qwen3_8b_bench_shape_sampled():
     _sampled_check("qwen3-8b")
+
+
+def test_bf16_llama31_8b_wide_tree_sampled():
+    """T=128 wide tree over an 8192-position cache (RoPE theta 5e5, no q/k norm)."""
+    _sampled_check("llama3.1-8b")
+
+
+def test_bf16_qwen25_32b_sampled():
+    """64 layers, 40/8 heads, q/k/v bias: about 64 GB of bf16 weights on one GPU."""
+    _sampled_check("qwen2.5-32b")
