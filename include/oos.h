@@ -216,6 +216,15 @@ int oos_accept_walk(const int32_t* tree_tokens, const int32_t* tree_parent, cons
 #define OOS_STAGE_LM_HEAD 4
 int oos_launch_stage(oos_model* m, int32_t layer, int32_t stage, int32_t T, void* stream);
 
+/* Benchmarking aid: enqueue ONE tree-attention kernel of layer `layer`,
+ * launched exactly as oos_tree_verify launches it, over cache positions
+ * [0, ctx_len) of `kv` and the tree K/V in slots ctx_len..ctx_len+T-1 (as the
+ * last verify with this ctx_len and T left them), with the workspace's q and
+ * ancestor sets.  It reads the cache and writes only workspace scratch.
+ * Errors as oos_tree_verify (EINVAL, ECAPACITY, ECUDA). */
+int oos_launch_attention(oos_model* m, const oos_kv_cache* kv, int32_t layer, int32_t ctx_len, int32_t T,
+                         void* stream);
+
 /* LM-head greedy argmax that allocates nothing.  The paper has no counterpart:
  * this entry point exists for callers that cannot allocate device memory at
  * all -- code running inside someone else's CUDA-graph capture, under a memory

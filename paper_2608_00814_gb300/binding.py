@@ -79,6 +79,8 @@ def lib():
         L.oos_last_status.argtypes = [c_vp, c_vp]
         L.oos_launch_stage.argtypes = [c_vp, c_i32, c_i32, c_i32, c_vp]
         L.oos_launch_stage.restype = ctypes.c_int
+        L.oos_launch_attention.argtypes = [c_vp, P(OosKvCache), c_i32, c_i32, c_i32, c_vp]
+        L.oos_launch_attention.restype = ctypes.c_int
         L.oos_lm_head_argmax_static.argtypes = [c_i32, c_i32, c_i32, c_vp, c_vp, c_i32, c_vp, c_vp, c_vp, c_vp]
         L.oos_lm_head_argmax_static.restype = ctypes.c_int
         L.oos_status_string.argtypes = [ctypes.c_int]
@@ -222,6 +224,11 @@ OOS_STAGE_QKV, OOS_STAGE_O, OOS_STAGE_GATE_UP, OOS_STAGE_DOWN, OOS_STAGE_LM_HEAD
 
 def oos_launch_stage(model, layer, stage, T, stream=None):
     _check(lib().oos_launch_stage(model.handle, layer, stage, T, _stream(stream)), "oos_launch_stage")
+
+
+def oos_launch_attention(model, kv, layer, ctx_len, T, stream=None):
+    _check(lib().oos_launch_attention(model.handle, ctypes.byref(kv.c), layer, ctx_len, T, _stream(stream)),
+           "oos_launch_attention")
 
 
 def oos_lm_head_argmax_static(dtype, vocab, hidden_dim, lm_head, hidden, T, out_argmax, out_top1, out_top2,

@@ -4,14 +4,19 @@
 // cache positions [0, ctx) and to the tree slots ctx + a for every ancestor a
 // of i (itself included): softmax(q k / sqrt(d)) v.
 //
-// bf16 path: split-K over the cache (flash-decoding).  A block owns 64 query
-// rows of one kv head -- the (node, q-head) pairs of the group, so GQA reuses
-// every K/V tile for nq/nkv heads -- and one range of cache keys; the last
-// split also takes the tree tail, masked with the 128-bit ancestor sets.  K/V
-// tiles are staged in shared memory by a 3-deep cp.async ring; scores and P.V
-// run on the tensor cores (mma.sync m16n8k16, fp32 accumulate) with an online
-// softmax in fp32.  The last split of a row block to finish merges all splits
-// by log-sum-exp (fixed split order) and writes the hi/lo bf16 GEMM input.
+// bf16 path: split-K over the keys (flash-decoding) inside one thread-block
+// cluster.  A block owns 64 query rows of one kv head -- the (node, q-head)
+// pairs of the group, so GQA reuses every K/V tile for nq/nkv heads -- and one
+// contiguous range of 64-key tiles (cache tiles first, the tree tail last,
+// masked with the 128-bit ancestor sets).  The blocks of the different ranges
+// of the same rows form one cluster.  K/V tiles are staged in shared memory by
+// a 3-deep cp.async ring; scores and P.V run on the tensor cores (mma.sync
+// m16n8k16, fp32 accumulate) with an online softmax in fp32.  Each block then
+// leaves its unnormalised O and (max, sum) in its own shared memory, and after
+// a cluster barrier every block merges a slice of the rows by log-sum-exp,
+// reading the other blocks' shared memory (fixed split order), and writes the
+// hi/lo bf16 GEMM input.  The first cache tiles are fetched before the wait on
+// the producing kernel: no kernel of the step writes cache positions < ctx.
 //
 // fp32 path: one block per (node, head), CUDA cores (small models only).
 #include <math.h>
@@ -36,14 +41,42 @@ struct AttnArgs {
   const __nv_bfloat16* vc;
   const unsigned long long* anc;
   int T, nq, nkv, group, ctx;
-  int splits, cache_blocks, row_blocks;
+  int splits;               // blocks per cluster (key ranges of the same rows)
+  int cache_blocks;         // 64-key tiles of the committed cache
+  int tiles;                // cache_blocks + tree tiles
   float scale_log2;         // log2(e) / sqrt(d)
-  float* o_part;            // [split][T*nq][d]
-  float* ml_part;           // [split][T*nq][2]
-  int* cnt;                 // [nkv * row_blocks] split arrival counters
   __nv_bfloat16* out;       // [T][nq*d] hi rows, lo rows at out_lo_off
   size_t out_lo_off;
 };
+
+// merge staging in the (drained) ring: O rows padded to 136 floats, then (m, l)
+constexpr int kAttnOLd = kAttnD + 8;
+static_assert(kAttnRows * kAttnOLd * 4 + kAttnRows * 8 <= kAttnSmem, "merge staging exceeds the ring");
+
+OOS_DEV uint32_t cluster_rank() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+  return r;
+}
+OOS_DEV void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+// address of the same shared-memory variable in block `rank` of the cluster
+OOS_DEV uint32_t dsmem_addr(const void* p, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr(p)), "r"(rank));
+  return r;
+}
+OOS_DEV float4 dsmem_ld4(uint32_t a) {
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0,%1,%2,%3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(a) : "memory");
+  return v;
+}
+OOS_DEV float2 dsmem_ld2(uint32_t a) {
+  float2 v;
+  asm volatile("ld.shared::cluster.v2.f32 {%0,%1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(a) : "memory");
+  return v;
+}
 
 OOS_DEV void cp_async16(void* smem, const void* gmem, bool valid) {
   const int n = valid ? 16 : 0;
@@ -92,42 +125,49 @@ OOS_DEV void load_kv_tile(__nv_bfloat16* ks, __nv_bfloat16* vs, const AttnArgs& 
 __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   __nv_bfloat16* ring = reinterpret_cast<__nv_bfloat16*>(smem_raw);   // [stage][K | V][64][ld]
-  __shared__ int s_last;
-  __shared__ float s_w[kAttnRows][kMaxAttnSplits];   // merge weights (last split only)
   pdl_trigger();
-  pdl_wait();
   const int rb = blockIdx.x, g = blockIdx.y, split = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int R = a.T * a.group;
 
-  // key tiles of this block: cache blocks [cb0, cb1), then (last split) the tree tail
-  const int cb0 = (int)((long long)split * a.cache_blocks / a.splits);
-  const int cb1 = (int)((long long)(split + 1) * a.cache_blocks / a.splits);
-  const int tree_tiles = (split == a.splits - 1) ? (a.T + kAttnKeys - 1) / kAttnKeys : 0;
-  const int n_tiles = (cb1 - cb0) + tree_tiles;
+  // tiles [t0, t1) of this block: cache tiles, then the tree tail
+  const int t0 = (int)((long long)split * a.tiles / a.splits);
+  const int t1 = (int)((long long)(split + 1) * a.tiles / a.splits);
+  const int n_tiles = t1 - t0;
   auto tile_keys = [&](int ti, int& key0, int& key_end, bool& tree) {
-    if (ti < cb1 - cb0) {
-      key0 = (cb0 + ti) * kAttnKeys;
+    const int t = t0 + ti;
+    if (t < a.cache_blocks) {
+      key0 = t * kAttnKeys;
       key_end = min(a.ctx, key0 + kAttnKeys);
       tree = false;
     } else {
-      const int tt = ti - (cb1 - cb0);
-      key0 = a.ctx + tt * kAttnKeys;
+      key0 = a.ctx + (t - a.cache_blocks) * kAttnKeys;
       key_end = a.ctx + a.T;
       tree = true;
     }
   };
   auto stage_k = [&](int s) { return ring + s * kAttnStageElems; };
   auto stage_v = [&](int s) { return ring + s * kAttnStageElems + kAttnKeys * kAttnLd; };
+  auto load = [&](int ti) {
+    int k0, ke;
+    bool tr;
+    tile_keys(ti, k0, ke, tr);
+    load_kv_tile(stage_k(ti % kAttnStages), stage_v(ti % kAttnStages), a, g, k0, ke);
+  };
   auto issue = [&](int ti) {
-    if (ti < n_tiles) {
-      int k0, ke;
-      bool tr;
-      tile_keys(ti, k0, ke, tr);
-      load_kv_tile(stage_k(ti % kAttnStages), stage_v(ti % kAttnStages), a, g, k0, ke);
-    }
+    if (ti < n_tiles) load(ti);
     cp_async_commit();
   };
+
+  // Cache tiles do not depend on the producing kernel: fetch the first two
+  // before waiting for it.  Tree tiles and Q are read after the wait.
+  const bool pre0 = n_tiles > 0 && t0 < a.cache_blocks;
+  const bool pre1 = n_tiles > 1 && t0 + 1 < a.cache_blocks;
+  if (pre0) load(0);
+  if (pre1) load(1);
+  pdl_wait();
+  if (n_tiles > 0 && !pre0) load(0);
+  if (n_tiles > 1 && !pre1) load(1);
 
   // Q rows (row r -> node r / group, head g*group + r % group), staged through
   // the last ring slot, then kept in registers as mma A fragments
@@ -141,7 +181,7 @@ __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
       cp_async16(Qs + r * kAttnLd + col, a.q + ((size_t)node * a.nq + hq) * kAttnD + col, valid);
     }
     cp_async_commit();
-    cp_async_wait<0>();
+    cp_async_wait<0>();   // Q and tiles 0, 1
     __syncthreads();
   }
   uint32_t qf[8][4];
@@ -152,8 +192,8 @@ __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
     ldsm_x4(qf[ks], stage_k(kAttnStages - 1) + row * kAttnLd + col);
   }
   __syncthreads();
-  issue(0);
-  issue(1);
+  // tiles 0 and 1 have landed; iteration ti commits one group (tile ti + 2),
+  // so wait_group 2 there means tile ti has landed
 
   // per-thread rows: r_lo = warp*16 + lane/4, r_hi = r_lo + 8
   const int r_lo = rb * kAttnRows + warp * 16 + (lane >> 2);
@@ -274,117 +314,80 @@ __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
     __syncthreads();
   }
   cp_async_wait<0>();
+  __syncthreads();   // every warp is done with the ring
 
-  // quad sums of l, then this split's unnormalised O and (m, l)
+  // quad sums of l, then this block's unnormalised O and (m, l) into its own
+  // shared memory
 #pragma unroll
   for (int off = 1; off <= 2; off <<= 1) {
     l_lo += __shfl_xor_sync(0xffffffffu, l_lo, off);
     l_hi += __shfl_xor_sync(0xffffffffu, l_hi, off);
   }
-  const size_t rows_total = (size_t)a.T * a.nq;
-#pragma unroll
-  for (int half = 0; half < 2; ++half) {
-    const int r = half ? r_hi : r_lo;
-    if (r >= R) continue;
-    const int node = r / a.group, hq = g * a.group + r % a.group;
-    const size_t grow = (size_t)node * a.nq + hq;
-    float* dst = a.o_part + ((size_t)split * rows_total + grow) * kAttnD;
+  float* so = reinterpret_cast<float*>(smem_raw);     // [64][kAttnOLd]
+  float* sml = so + kAttnRows * kAttnOLd;             // [64][2]
+  {
+    const int lr = warp * 16 + (lane >> 2);
 #pragma unroll
     for (int n = 0; n < 16; ++n) {
       const int col = n * 8 + (lane & 3) * 2;
-      *reinterpret_cast<float2*>(dst + col) = half ? make_float2(o[n][2], o[n][3]) : make_float2(o[n][0], o[n][1]);
+      *reinterpret_cast<float2*>(so + lr * kAttnOLd + col) = make_float2(o[n][0], o[n][1]);
+      *reinterpret_cast<float2*>(so + (lr + 8) * kAttnOLd + col) = make_float2(o[n][2], o[n][3]);
     }
     if ((lane & 3) == 0) {
-      float* ml = a.ml_part + ((size_t)split * rows_total + grow) * 2;
-      ml[0] = half ? m_hi : m_lo;
-      ml[1] = half ? l_hi : l_lo;
+      *reinterpret_cast<float2*>(sml + 2 * lr) = make_float2(m_lo, l_lo);
+      *reinterpret_cast<float2*>(sml + 2 * (lr + 8)) = make_float2(m_hi, l_hi);
     }
   }
+  cluster_sync();   // every block's partial is in its shared memory
 
-  // the last split of this (row block, kv head) to finish merges all splits:
-  // log-sum-exp weights in base 2, summed in split order
-  __threadfence();
-  __syncthreads();
-  if (threadIdx.x == 0) {
-    const int ci = g * a.row_blocks + rb;
-    const int old = atomicAdd(&a.cnt[ci], 1);
-    s_last = old == a.splits - 1;
-    if (s_last) a.cnt[ci] = 0;
-  }
-  __syncthreads();
-  if (!s_last) return;
-  __threadfence();
-  // per-row split weights w_s = 2^(m_s - M) / sum_s 2^(m_s - M) l_s
-  if (threadIdx.x < kAttnRows) {
-    const int r = rb * kAttnRows + threadIdx.x;
-    if (r < R) {
-      const size_t grow = (size_t)(r / a.group) * a.nq + g * a.group + r % a.group;
-      float ms[kMaxAttnSplits], ls[kMaxAttnSplits];
+  // block of cluster rank c merges local rows [64c/S, 64(c+1)/S): thread ->
+  // (row, four head dims); weights 2^(m_s - M) / sum_s 2^(m_s - M) l_s, summed
+  // in split order
+  {
+    const int S = a.splits;
+    const int c = (int)cluster_rank();
+    const int lr0 = kAttnRows * c / S, lr1 = kAttnRows * (c + 1) / S;
+    for (int idx = threadIdx.x; idx < (lr1 - lr0) * (kAttnD / 4); idx += blockDim.x) {
+      const int lr = lr0 + idx / (kAttnD / 4), d4 = (idx % (kAttnD / 4)) * 4;
+      const int r = rb * kAttnRows + lr;
+      float2 ml[kMaxAttnSplits];
       float M = -INFINITY;
 #pragma unroll
       for (int sp = 0; sp < kMaxAttnSplits; ++sp) {
-        if (sp < a.splits) {
-          const float2 v = __ldcg(reinterpret_cast<const float2*>(a.ml_part + ((size_t)sp * rows_total + grow) * 2));
-          ms[sp] = v.x;
-          ls[sp] = v.y;
-          M = fmaxf(M, v.x);
+        if (sp < S) {
+          ml[sp] = dsmem_ld2(dsmem_addr(sml + 2 * lr, sp));
+          M = fmaxf(M, ml[sp].x);
         }
       }
-      float den = 0.f;
-#pragma unroll
-      for (int sp = 0; sp < kMaxAttnSplits; ++sp) {
-        if (sp < a.splits) {
-          const float wgt = ms[sp] == -INFINITY ? 0.f : exp2f(ms[sp] - M);
-          ms[sp] = wgt;
-          den += wgt * ls[sp];
-        }
-      }
+      float4 v[kMaxAttnSplits];
 #pragma unroll
       for (int sp = 0; sp < kMaxAttnSplits; ++sp)
-        if (sp < a.splits) s_w[threadIdx.x][sp] = ms[sp] / den;
-    }
-  }
-  __syncthreads();
-  // warp w: rows w, w+4, ...; lane: four head dims
-  {
-    constexpr int RW = kAttnRows / 4;
-    float4 acc[RW];
-    int grow[RW];   // output row (node * nq + head) of each handled query row, -1 past R
+        if (sp < S) v[sp] = dsmem_ld4(dsmem_addr(so + lr * kAttnOLd + d4, sp));
+      float den = 0.f;
+      float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-    for (int i = 0; i < RW; ++i) {
-      acc[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-      const int r = rb * kAttnRows + warp + 4 * i;
-      grow[i] = r < R ? (r / a.group) * a.nq + g * a.group + r % a.group : -1;
-    }
-    // splits two at a time: all loads of a pair are issued before any is used
-    for (int sp0 = 0; sp0 < a.splits; sp0 += 2) {
-      float4 v[2][RW];
-#pragma unroll
-      for (int q = 0; q < 2; ++q) {
-        const float* src = a.o_part + (size_t)(sp0 + q) * rows_total * kAttnD + 4 * lane;
-#pragma unroll
-        for (int i = 0; i < RW; ++i)
-          v[q][i] = (sp0 + q < a.splits && grow[i] >= 0)
-                        ? __ldcg(reinterpret_cast<const float4*>(src + (size_t)grow[i] * kAttnD))
-                        : make_float4(0.f, 0.f, 0.f, 0.f);
-      }
-#pragma unroll
-      for (int q = 0; q < 2; ++q) {
-        if (sp0 + q >= a.splits) break;
-#pragma unroll
-        for (int i = 0; i < RW; ++i) {
-          const float wgt = s_w[warp + 4 * i][sp0 + q];
-          acc[i].x += wgt * v[q][i].x;
-          acc[i].y += wgt * v[q][i].y;
-          acc[i].z += wgt * v[q][i].z;
-          acc[i].w += wgt * v[q][i].w;
+      for (int sp = 0; sp < kMaxAttnSplits; ++sp) {
+        if (sp < S) {
+          const float wgt = ml[sp].x == -INFINITY ? 0.f : exp2f(ml[sp].x - M);
+          den += wgt * ml[sp].y;
+          acc.x += wgt * v[sp].x;
+          acc.y += wgt * v[sp].y;
+          acc.z += wgt * v[sp].z;
+          acc.w += wgt * v[sp].w;
         }
       }
+      const float inv = 1.f / den;
+      acc.x *= inv;
+      acc.y *= inv;
+      acc.z *= inv;
+      acc.w *= inv;
+      if (r < R) {
+        const size_t grow = (size_t)(r / a.group) * a.nq + g * a.group + r % a.group;
+        store_act4(a.out, grow * kAttnD + d4, a.out_lo_off, acc);
+      }
     }
-#pragma unroll
-    for (int i = 0; i < RW; ++i)
-      if (grow[i] >= 0) store_act4(a.out, (size_t)grow[i] * kAttnD + 4 * lane, a.out_lo_off, acc[i]);
   }
+  cluster_sync();   // no block leaves while another may still read its shared memory
 }
 
 // ------------------------------------------------------------ fp32 path
@@ -461,22 +464,34 @@ cudaError_t launch_attention(Model& m, const void* kc, const void* vc, int ctx, 
   a.group = c.n_q_heads / c.n_kv_heads;
   a.ctx = ctx;
   a.cache_blocks = (ctx + kAttnKeys - 1) / kAttnKeys;
+  a.tiles = a.cache_blocks + (T + kAttnKeys - 1) / kAttnKeys;
   const int R = T * a.group;
   const int RB = (R + kAttnRows - 1) / kAttnRows;
-  a.row_blocks = RB;
-  // one wave at two blocks per SM (OOS_ATTN_SPLITS overrides, for tuning)
+  // one wave at two blocks per SM, at most one cluster of kMaxAttnSplits
+  // blocks per row block, no block without a tile
   int splits = (2 * m.num_sms) / (a.nkv * RB);
-  if (const char* e = getenv("OOS_ATTN_SPLITS")) splits = atoi(e);
-  const int max_splits = a.cache_blocks > 0 ? (a.cache_blocks < kMaxAttnSplits ? a.cache_blocks : kMaxAttnSplits) : 1;
-  splits = splits < 1 ? 1 : (splits > max_splits ? max_splits : splits);
+  splits = splits < 1 ? 1 : (splits > kMaxAttnSplits ? kMaxAttnSplits : splits);
+  splits = splits > a.tiles ? a.tiles : splits;
   a.splits = splits;
   a.scale_log2 = 1.4426950408889634f / sqrtf((float)kAttnD);
-  a.o_part = m.ws.attn_o;
-  a.ml_part = m.ws.attn_ml;
-  a.cnt = m.ws.attn_cnt;
   a.out = (__nv_bfloat16*)m.ws.attn;
   a.out_lo_off = (size_t)kMaxT * c.n_q_heads * kAttnD;
-  return launch(m.pdl, k_attn_tc, dim3(RB, a.nkv, splits), dim3(128), (size_t)kAttnSmem, st, a);
+
+  cudaLaunchConfig_t lc = {};
+  lc.gridDim = dim3(RB, a.nkv, splits);
+  lc.blockDim = dim3(128);
+  lc.dynamicSmemBytes = (size_t)kAttnSmem;
+  lc.stream = st;
+  cudaLaunchAttribute attr[2];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 1;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = splits;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  lc.attrs = attr;
+  lc.numAttrs = m.pdl ? 2 : 1;
+  return cudaLaunchKernelEx(&lc, k_attn_tc, a);
 }
 
 }  // namespace oos

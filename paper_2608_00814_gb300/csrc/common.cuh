@@ -115,17 +115,40 @@ OOS_DEV bool mbar_test(uint32_t addr, uint32_t parity) {
       : "memory");
   return ok != 0;
 }
+// Same test, but a thread whose phase is not complete yet is suspended (issue
+// slots go to the warps with work) until it completes or `hint_ns` pass.
+OOS_DEV bool mbar_test_sleep(uint32_t addr, uint32_t parity, uint32_t hint_ns) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(addr), "r"(parity), "r"(hint_ns)
+      : "memory");
+  return ok != 0;
+}
+// First wait of the step to exceed its limit: status[1] = site code, [2] = phase,
+// [3] = unit or tile, [4] = CTA, [5] = block-local detail (first writer wins).
+OOS_DEV void record_timeout(uint32_t* status, uint32_t site, int phase, long long unit, int detail) {
+  if (atomicCAS(status + 1, 0u, site) == 0u) {
+    status[2] = (uint32_t)phase;
+    status[3] = (uint32_t)unit;
+    status[4] = blockIdx.x;
+    status[5] = (uint32_t)detail;
+  }
+}
+
 // Wait for the phase with `parity` to complete.  Gives up after kWaitLimitNs or
 // when *abort becomes nonzero (another role gave up); returns false then and
-// records ST_TIMEOUT in *status (only for a genuine timeout).
+// records ST_TIMEOUT in *status (only for a genuine timeout).  Between checks of
+// the abort flag the thread sleeps on the barrier (at most 20 us at a time).
 OOS_DEV bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort, uint32_t* status) {
   const uint32_t addr = smem_addr(bar);
   if (mbar_test(addr, parity)) return true;
   const unsigned long long t0 = globaltimer();
   while (true) {
-#pragma unroll 1
-    for (int i = 0; i < 32; ++i)
-      if (mbar_test(addr, parity)) return true;
+    if (mbar_test_sleep(addr, parity, 20000u)) return true;
     if (*abort) return false;
     if (globaltimer() - t0 > kWaitLimitNs) {
       *abort = 1;

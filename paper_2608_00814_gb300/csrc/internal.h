@@ -17,8 +17,7 @@ constexpr int kTile = 128;          // weight rows per MMA (tcgen05 M)
 constexpr int kWorkRowsWide = 256;  // weight rows per work tile of the gate/up GEMM and LM head
 constexpr int kBK = 64;             // reduction elements per pipeline stage (128 bytes of bf16)
 constexpr int kMaxLayers = 128;
-constexpr int kMaxAttnSplits = 16;  // cache splits of the attention kernel
-constexpr int kAttnCnt = 4096;      // attention arrival counters (kv heads x row blocks)
+constexpr int kMaxAttnSplits = 8;   // key ranges per row block (one cluster, portable size)
 constexpr int kMaxGridCTAs = 1024;  // upper bound on CTAs of a stream-K GEMM / LM head
 constexpr int kMaxSsChunks = 64;    // hidden <= 8192: RMSNorm partial sums per 128 features
 constexpr int kCntPer = 256;        // arrival counters per (layer, GEMM kind): one per work tile
@@ -81,8 +80,6 @@ struct Workspace {
   void* act;                 // SwiGLU activation [kMaxT][I]
   float* part;               // GEMM partial slices
   size_t part_floats;
-  float* attn_o;             // [kMaxAttnSplits][kMaxT*nq][d]
-  float* attn_ml;            // [kMaxAttnSplits][kMaxT*nq][2]
   float* lm_v1;              // LM-head partial states [kMaxGridCTAs][kMaxT]
   int32_t* lm_i;
   float* lm_v2;
@@ -93,7 +90,6 @@ struct Workspace {
   float* ss;                 // sum of x^2 per 128-feature chunk [kMaxSsChunks][kMaxT] (bf16 path)
   float2* rope;              // (cos, sin) per node and rotary pair [kMaxT][d/2] (bf16 path)
   int* cnt;                  // GEMM arrival counters [layer][4 kinds][kCntPer], zeroed at every step start
-  int* attn_cnt;             // attention split arrival counters [kAttnCnt]
 };
 
 // shape + addresses a captured verify graph was recorded with

@@ -76,10 +76,6 @@ size_t carve_workspace(const oos_model_config& c, int n_sms, uint8_t* base, Work
   }
   w.part_floats = pf;
   w.part = (float*)take(pf * 4);
-  const size_t att_rows = (size_t)kMaxT * c.n_q_heads;
-  const bool tc = c.dtype == OOS_DTYPE_BF16;
-  w.attn_o = (float*)take(tc ? kMaxAttnSplits * att_rows * c.head_dim * 4 : 0);
-  w.attn_ml = (float*)take(tc ? kMaxAttnSplits * att_rows * 2 * 4 : 0);
   const size_t lm = (size_t)kMaxGridCTAs * kMaxT;
   w.lm_v1 = (float*)take(lm * 4);
   w.lm_i = (int32_t*)take(lm * 4);
@@ -91,7 +87,6 @@ size_t carve_workspace(const oos_model_config& c, int n_sms, uint8_t* base, Work
   w.ss = (float*)take((size_t)kMaxSsChunks * kMaxT * 4);
   w.rope = (float2*)take((size_t)kMaxT * (c.head_dim / 2) * 8);
   w.cnt = (int*)take((size_t)c.n_layers * 4 * kCntPer * 4);
-  w.attn_cnt = (int*)take((size_t)kAttnCnt * 4);
   if (ws) *ws = w;
   return align_up(off, 256);
 }
@@ -115,8 +110,6 @@ static bool shape_supported(const oos_model_config* c) {
     if (2 * c->intermediate / kWorkRowsWide > kCntPer || (c->n_q_heads + 2 * c->n_kv_heads) > kCntPer ||
         c->hidden / kTile > kCntPer)
       return false;
-    const int rb = (kMaxT * (c->n_q_heads / c->n_kv_heads) + 63) / 64;
-    if (c->n_kv_heads * rb > kAttnCnt) return false;
   }
   return true;
 }
@@ -471,6 +464,16 @@ int oos_launch_stage(oos_model* m, int32_t layer, int32_t stage, int32_t T, void
     }
   }
   return e == cudaSuccess ? OOS_OK : OOS_ECUDA;
+}
+
+int oos_launch_attention(oos_model* m, const oos_kv_cache* kv, int32_t layer, int32_t ctx_len, int32_t T,
+                         void* stream) {
+  if (!m || !kv || kv->n_layers != m->cfg.n_layers || !kv->k || !kv->v) return OOS_EINVAL;
+  if (layer < 0 || layer >= m->cfg.n_layers || !kv->k[layer] || !kv->v[layer]) return OOS_EINVAL;
+  if (T < 1 || T > m->cfg.max_T || ctx_len < 0) return OOS_EINVAL;
+  if ((long long)ctx_len + T > kv->capacity) return OOS_ECAPACITY;
+  return launch_attention(*m, kv->k[layer], kv->v[layer], ctx_len, T, (cudaStream_t)stream) == cudaSuccess ? OOS_OK
+                                                                                                        : OOS_ECUDA;
 }
 
 int oos_last_status(oos_model* m, void* stream) {

@@ -32,6 +32,7 @@ __global__ void __launch_bounds__(kMaxT) k_tree_prep(const int32_t* __restrict__
   }
   __syncthreads();
   if (i == 0) *status = s_bad ? ST_TREE : 0u;
+  if (i >= 1 && i < 8) status[i] = 0u;   // where a pipeline wait gave up (see common.cuh)
   if (i < T) {
     int d = 0;
     unsigned long long lo = 0, hi = 0;
@@ -50,9 +51,13 @@ __global__ void __launch_bounds__(kMaxT) k_tree_prep(const int32_t* __restrict__
   }
 }
 
+// The first kernel of a step is launched without programmatic serialisation:
+// it starts only after all earlier work on the stream (the previous step's
+// compaction, the caller's cache writes) has completed, so later kernels of
+// the step may read cache positions < ctx before their own dependency wait.
 cudaError_t launch_tree_prep(Model& m, const int32_t* tokens, const int32_t* parent, int T, int ctx,
                              cudaStream_t st) {
-  return launch(m.pdl, k_tree_prep, dim3(1), dim3(kMaxT), 0, st, tokens, parent, T, ctx, m.cfg.vocab,
+  return launch(false, k_tree_prep, dim3(1), dim3(kMaxT), 0, st, tokens, parent, T, ctx, m.cfg.vocab,
                 m.ws.status, m.ws.depth, m.ws.pos, m.ws.anc);
 }
 
