@@ -4,7 +4,7 @@ Only the test suite, `__graft_entry__.smoke()` and the benchmark's CPU-baseline
 leg may import it.  The product path never does.
 """
 
-from .tree_verify import (TreeError, accept, attend, compact, decode_sequence,  # noqa: F401
+from .tree_verify import (TreeError, accept, attend, cache_format, compact, decode_sequence,  # noqa: F401
                           decode_step, greedy_continuation, lm_head_argmax, mlp, prefill,
                           qkv, rms_norm, rope, silu, tree_structure, verify_and_accept,
                           verify_tree)

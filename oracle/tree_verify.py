@@ -24,6 +24,8 @@ What the paper leaves open, and the reading taken here:
     (itself included): one forward pass over a tree is therefore the same as
     causal decoding along every root-to-leaf path.
   * RoPE position of node i is ctx_len + depth(i) (rotate-half convention).
+  * K and V are stored in the cache's format before anything attends to them
+    (bf16 for the bf16 models): the tree's own K/V go through the cache too.
   * "Longest prefix" is the deepest accepted node, lowest node id on ties;
     argmax ties go to the lowest vocabulary id.
   * The decoder is a pre-norm Llama/Qwen block: RMSNorm, q/k/v projections
@@ -97,6 +99,22 @@ def rope(x, pos, theta):
 
 def silu(z):
     return z / (1.0 + np.exp(-z))
+
+
+def cache_format(x, dtype):
+    """K or V as the KV cache stores it.
+
+    The target's KV cache is kept in the model's precision (the paper's targets
+    run BF16 or FP16 caches): a bf16 cache stores round-to-nearest-even bf16
+    values, so every K/V a node attends to -- cached or written by the tree
+    pass itself -- is bf16.  An fp32 cache is kept exact here (fp32 rounding of
+    K/V is far below the fp32 tolerance).
+    """
+    if dtype != "bf16":
+        return x
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    u = (u + 0x7FFF + ((u >> 16) & 1)) >> 16
+    return (u.astype(np.uint32) << 16).view(np.float32).astype(np.float64).reshape(np.shape(x))
 
 
 def attend(q, keys, values):
@@ -194,8 +212,8 @@ def verify_tree(m, cache_k, cache_v, ctx_len, tokens, parent, only=None):
         v = np.full((T, nkv, d), np.nan)
         for r, i in enumerate(nodes):
             q[i] = rope(q_s[r], ctx_len + depth[i], cfg.rope_theta)
-            k[i] = rope(k_s[r], ctx_len + depth[i], cfg.rope_theta)
-            v[i] = v_s[r]
+            k[i] = cache_format(rope(k_s[r], ctx_len + depth[i], cfg.rope_theta), cfg.dtype)
+            v[i] = cache_format(v_s[r], cfg.dtype)
         tree_k.append(k)
         tree_v.append(v)
         o = np.zeros((T, nq, d))
@@ -290,8 +308,8 @@ def decode_step(m, cache_k, cache_v, n_pos, token):
         h = rms_norm(x, W["attn_norm"], cfg.rms_eps)
         q, k, v = qkv(W, cfg, h)
         q = rope(q[0], n_pos, cfg.rope_theta)
-        k = rope(k[0], n_pos, cfg.rope_theta)
-        v = v[0]
+        k = cache_format(rope(k[0], n_pos, cfg.rope_theta), cfg.dtype)
+        v = cache_format(v[0], cfg.dtype)
         ks.append(k)
         vs.append(v)
         o = np.zeros((nq, d))

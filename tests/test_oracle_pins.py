@@ -316,3 +316,61 @@ def test_only_subset_matches_full_pass():
     for i in part["nodes"]:
         np.testing.assert_allclose(part["final_hidden"][i], full["final_hidden"][i], rtol=1e-12, atol=1e-12)
         assert part["argmax"][i] == full["argmax"][i]
+
+
+# ------------------------------------------------------------------ bf16 KV cache format
+
+def test_cache_format_is_bf16_round_to_nearest_even():
+    rng = np.random.default_rng(11)
+    x = np.concatenate([rng.standard_normal(4096) * 3.0, [0.0, -0.0, 1.0, -2.5, 1e-30, 65504.0]])
+    # exact bf16 halfway points (fp32 low half 0x8000), both parities of the kept bit
+    halves = (np.arange(64, dtype=np.uint32) << 16 | np.uint32(0x3F800000) | np.uint32(0x8000)).view(np.float32)
+    x = np.concatenate([x, halves.astype(np.float64), -halves.astype(np.float64)])
+    ref = torch.from_numpy(x).to(torch.float32).to(torch.bfloat16).to(torch.float64).numpy()
+    np.testing.assert_array_equal(oracle.cache_format(x, "bf16"), ref)
+    np.testing.assert_array_equal(oracle.cache_format(x, "f32"), x)
+
+
+def _mini_case(seed, T=7, ctx_len=12):
+    return build_case("mini-bf16", seed, T=T, recipe=dict(kind="uniform", max_depth=3), ctx_len=ctx_len, plant=0)
+
+
+def test_bf16_tree_kv_is_cache_format_and_tree_equals_causal_decoding():
+    """With a bf16 cache both the tree pass and plain decoding attend to bf16
+    K/V; the tree pass still equals causal decoding along every path."""
+    c = _mini_case(5)
+    r = oracle.verify_tree(c.view, c.cache_k64, c.cache_v64, c.ctx_len, c.tokens, c.parent)
+    for l in range(c.cfg.n_layers):
+        np.testing.assert_array_equal(oracle.cache_format(r["tree_k"][l], "bf16"), r["tree_k"][l])
+        np.testing.assert_array_equal(oracle.cache_format(r["tree_v"][l], "bf16"), r["tree_v"][l])
+    _, paths = oracle.tree_structure(c.parent)
+    leaves = [i for i in range(len(c.parent)) if i not in set(c.parent[1:].tolist())]
+    for leaf in leaves:
+        path = paths[leaf]
+        steps, _, _ = oracle.decode_sequence(c.view, c.cache_k64, c.cache_v64, c.ctx_len, c.tokens[path])
+        for j, node in enumerate(path):
+            np.testing.assert_allclose(r["final_hidden"][node], steps[j]["final_hidden"], rtol=1e-10, atol=1e-10)
+            for l in range(c.cfg.n_layers):
+                np.testing.assert_array_equal(r["tree_k"][l][node], steps[j]["k"][l])
+
+
+def test_bf16_layer0_tree_k_matches_library_restatement():
+    """Layer-0 K of every node: RMSNorm, W_k, per-head RMSNorm, rotary
+    embedding at ctx + depth, then bf16 -- restated with torch routines."""
+    c = _mini_case(6)
+    r = oracle.verify_tree(c.view, c.cache_k64, c.cache_v64, c.ctx_len, c.tokens, c.parent)
+    W = c.view.layer(0)
+    cfg = c.cfg
+    depth, _ = oracle.tree_structure(c.parent)
+    x = torch.from_numpy(c.view.embed_rows(c.tokens))
+    h = F.rms_norm(x, (cfg.hidden,), torch.from_numpy(W["attn_norm"]), eps=cfg.rms_eps)
+    k = (h @ torch.from_numpy(W["w_k"]).T).reshape(len(c.tokens), cfg.n_kv_heads, cfg.head_dim)
+    k = F.rms_norm(k, (cfg.head_dim,), torch.from_numpy(W["k_norm"]), eps=cfg.rms_eps)
+    half = cfg.head_dim // 2
+    freq = cfg.rope_theta ** (-2.0 * torch.arange(half, dtype=torch.float64) / cfg.head_dim)
+    pos = torch.tensor([c.ctx_len + d for d in depth], dtype=torch.float64)
+    rot = torch.polar(torch.ones(len(depth), half, dtype=torch.float64), pos[:, None] * freq[None, :])
+    kc = torch.complex(k[..., :half], k[..., half:]) * rot[:, None, :]
+    k_rot = torch.cat([kc.real, kc.imag], dim=-1)
+    ref = k_rot.to(torch.float32).to(torch.bfloat16).to(torch.float64).numpy()
+    np.testing.assert_allclose(r["tree_k"][0], ref, rtol=0, atol=0)
