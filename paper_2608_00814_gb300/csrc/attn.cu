@@ -11,7 +11,8 @@
 // masked with the 128-bit ancestor sets).  The blocks of the different ranges
 // of the same rows form one cluster.  K/V tiles are staged in shared memory by
 // a 3-deep cp.async ring; scores and P.V run on the tensor cores (mma.sync
-// m16n8k16, fp32 accumulate) with an online softmax in fp32.  Each block then
+// m16n8k16, fp32 accumulate; q as hi + lo bf16 halves) with an online softmax
+// in fp32.  Each block then
 // leaves its unnormalised O and (max, sum) in its own shared memory, and after
 // a cluster barrier every block merges a slice of the rows by log-sum-exp,
 // reading the other blocks' shared memory (fixed split order), and writes the
@@ -36,7 +37,8 @@ constexpr int kAttnStageElems = 2 * kAttnKeys * kAttnLd;   // K tile then V tile
 constexpr int kAttnSmem = kAttnStages * kAttnStageElems * 2;
 
 struct AttnArgs {
-  const __nv_bfloat16* q;   // [T][nq][d]
+  const __nv_bfloat16* q;   // [T][nq][d] hi halves, lo halves at q_lo_off
+  size_t q_lo_off;
   const __nv_bfloat16* kc;  // [cap][nkv][d]
   const __nv_bfloat16* vc;
   const unsigned long long* anc;
@@ -169,27 +171,32 @@ __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
   if (n_tiles > 0 && !pre0) load(0);
   if (n_tiles > 1 && !pre1) load(1);
 
-  // Q rows (row r -> node r / group, head g*group + r % group), staged through
-  // the last ring slot, then kept in registers as mma A fragments
+  // Q rows (row r -> node r / group, head g*group + r % group), hi halves in the
+  // K half and lo halves in the V half of the last ring slot, then kept in
+  // registers as mma A fragments: S = q_hi k + q_lo k sees ~16-bit q
   {
     __nv_bfloat16* Qs = stage_k(kAttnStages - 1);
+    __nv_bfloat16* Qls = stage_v(kAttnStages - 1);
     for (int c = threadIdx.x; c < kAttnRows * (kAttnD / 8); c += blockDim.x) {
       const int r = c >> 4, col = (c & 15) * 8;
       const int row = rb * kAttnRows + r;
       const bool valid = row < R;
       const int node = valid ? row / a.group : 0, hq = g * a.group + (valid ? row % a.group : 0);
-      cp_async16(Qs + r * kAttnLd + col, a.q + ((size_t)node * a.nq + hq) * kAttnD + col, valid);
+      const __nv_bfloat16* src = a.q + ((size_t)node * a.nq + hq) * kAttnD + col;
+      cp_async16(Qs + r * kAttnLd + col, src, valid);
+      cp_async16(Qls + r * kAttnLd + col, src + a.q_lo_off, valid);
     }
     cp_async_commit();
     cp_async_wait<0>();   // Q and tiles 0, 1
     __syncthreads();
   }
-  uint32_t qf[8][4];
+  uint32_t qf[8][4], qfl[8][4];
 #pragma unroll
   for (int ks = 0; ks < 8; ++ks) {
     const int row = warp * 16 + (lane & 7) + ((lane >> 3) & 1) * 8;
     const int col = ks * 16 + (lane >> 4) * 8;
     ldsm_x4(qf[ks], stage_k(kAttnStages - 1) + row * kAttnLd + col);
+    ldsm_x4(qfl[ks], stage_v(kAttnStages - 1) + row * kAttnLd + col);
   }
   __syncthreads();
   // tiles 0 and 1 have landed; iteration ti commits one group (tile ti + 2),
@@ -232,6 +239,10 @@ __global__ void __launch_bounds__(128) k_attn_tc(AttnArgs a) {
       for (int nt = 0; nt < 8; ++nt) mma_bf16(s[nt], qf[ks], b[nt][0], b[nt][1]);
 #pragma unroll
       for (int nt = 0; nt < 8; ++nt) mma_bf16(s[nt], qf[ks + 1], b[nt][2], b[nt][3]);
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt) mma_bf16(s[nt], qfl[ks], b[nt][0], b[nt][1]);
+#pragma unroll
+      for (int nt = 0; nt < 8; ++nt) mma_bf16(s[nt], qfl[ks + 1], b[nt][2], b[nt][3]);
     }
     // scale (+ mask on the tree tail and a partial last cache tile), tile row maxima
     float tmax_lo = -INFINITY, tmax_hi = -INFINITY;
@@ -455,6 +466,7 @@ cudaError_t launch_attention(Model& m, const void* kc, const void* vc, int ctx, 
   }
   AttnArgs a;
   a.q = (const __nv_bfloat16*)m.ws.q;
+  a.q_lo_off = (size_t)kMaxT * c.n_q_heads * kAttnD;
   a.kc = (const __nv_bfloat16*)kc;
   a.vc = (const __nv_bfloat16*)vc;
   a.anc = m.ws.anc;

@@ -26,7 +26,8 @@ namespace oos {
 // slices in slice order -- a fixed order, so results are deterministic -- and
 // applies the layer's elementwise step to the finished tile:
 //   EPI_QKV   : input RMSNorm scale, bias, per-head q/k RMSNorm, RoPE at
-//               ctx + depth; q to the query buffer, k/v to cache slot ctx + t.
+//               ctx + depth; q (hi/lo bf16) to the query buffer, k/v to cache
+//               slot ctx + t.
 //   EPI_RESID : x += W.a (O- and down-projections), then y = g (.) x for the
 //               next RMSNorm (hi/lo bf16) and per-tile sums of x^2.
 //   EPI_SILU  : gate and up tiles are interleaved (tile 2i = gate rows of
@@ -98,7 +99,14 @@ struct TcCfg {
   static constexpr int FIXED = 1024 /*align slack*/ + BAR_BYTES + EPI_BYTES + RED_BYTES;
   static constexpr int S_RAW = (227 * 1024 - FIXED) / STAGE;
   static constexpr int S = S_RAW > 8 ? 8 : S_RAW;
-  static constexpr int NCOLS = (2 * kSub * BN) < 32 ? 32 : 2 * kSub * BN;   // 2 buffers x kSub accumulators
+  // The hi and lo activation halves sit in one slot, hi rows then lo rows, so
+  // one MMA with N = 2 BN multiplies both ("paired": half the MMAs, the weight
+  // subtile read from shared memory once); the accumulator then holds the hi
+  // products in columns [0, BN) and the lo products in [BN, 2 BN).  Paired
+  // when two buffers of kSub such accumulators fit the 512 TMEM columns.
+  static constexpr bool PAIRED = 2 * kSub * 2 * BN <= 512;
+  static constexpr int SUB_COLS = PAIRED ? 2 * BN : BN;                      // accumulator columns per subtile
+  static constexpr int NCOLS = (2 * kSub * SUB_COLS) < 32 ? 32 : 2 * kSub * SUB_COLS;   // 2 buffers
   static constexpr int SMEM = FIXED + S * STAGE;
 };
 
@@ -290,12 +298,16 @@ OOS_DEV void finish_qkv(const GemmArgs& a, int n_part, int tile, int nc, const f
           v[c] = first_half ? v[c] * cs.x - other * cs.y : v[c] * cs.x + other * cs.y;
         }
       }
-      __nv_bfloat16* dst = kind == 0 ? a.q_out + ((size_t)t * a.nq + h) * kTile
-                                     : (kind == 1 ? a.kc : a.vc) + ((size_t)(a.ctx + t) * a.nkv + h) * kTile;
-      __nv_bfloat16 o[4];
+      if (kind == 0) {   // q as hi/lo bf16 halves: the attention product sees ~16-bit q
+        store_act4(a.q_out, ((size_t)t * a.nq + h) * kTile + 4 * l, (size_t)kMaxT * a.nq * kTile,
+                   make_float4(v[0], v[1], v[2], v[3]));
+      } else {           // K/V in the cache's bf16 format
+        __nv_bfloat16* dst = (kind == 1 ? a.kc : a.vc) + ((size_t)(a.ctx + t) * a.nkv + h) * kTile;
+        __nv_bfloat16 o[4];
 #pragma unroll
-      for (int c = 0; c < 4; ++c) o[c] = __float2bfloat16_rn(v[c]);
-      *reinterpret_cast<uint2*>(dst + 4 * l) = *reinterpret_cast<const uint2*>(o);
+        for (int c = 0; c < 4; ++c) o[c] = __float2bfloat16_rn(v[c]);
+        *reinterpret_cast<uint2*>(dst + 4 * l) = *reinterpret_cast<const uint2*>(o);
+      }
     }
   }
 }
@@ -478,7 +490,7 @@ __global__ void __launch_bounds__(192, 1)
   } else if (warp == 1) {
     // ------------------------------------------------------------ MMA issuer
     if (lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(kTile, BN);
+      constexpr uint32_t idesc = idesc_bf16_f32(kTile, C::PAIRED ? 2 * BN : BN);
       int stage = 0;
       uint32_t phase = 0;
       int acc = 0;
@@ -492,7 +504,7 @@ __global__ void __launch_bounds__(192, 1)
         if (seg_end > n_units) seg_end = n_units;
         if (!mbar_wait(&acce[acc], (acc_use[acc] & 1u) ^ 1u, abort_flag, a.status)) break;
         tc_fence_after();
-        const uint32_t d0 = tmem_base + (uint32_t)(acc * kSub * BN);
+        const uint32_t d0 = tmem_base + (uint32_t)(acc * kSub * C::SUB_COLS);
         for (int jj = j; jj < seg_end; ++jj) {
           if (!mbar_wait(&full[stage], phase, abort_flag, a.status)) {
             ok = false;
@@ -507,9 +519,9 @@ __global__ void __launch_bounds__(192, 1)
 #pragma unroll
             for (int sub = 0; sub < kSub; ++sub) {
               const uint64_t ad = smem_desc_sw128(sbase + sub * C::A_BYTES);
-              const uint32_t d = d0 + (uint32_t)(sub * BN);
+              const uint32_t d = d0 + (uint32_t)(sub * C::SUB_COLS);
               tc_mma_bf16(d, ad + 2 * k, bh + 2 * k, idesc, (jj > j || k > 0) ? 1u : 0u);
-              tc_mma_bf16(d, ad + 2 * k, bl + 2 * k, idesc, 1u);
+              if (!C::PAIRED) tc_mma_bf16(d, ad + 2 * k, bl + 2 * k, idesc, 1u);
             }
           }
           tc_commit(&empty[stage]);
@@ -555,23 +567,56 @@ __global__ void __launch_bounds__(192, 1)
       if (seg_end > n_units) seg_end = n_units;
       if (!mbar_wait(&accf[acc], acc_use[acc] & 1u, abort_flag, a.status)) break;
       tc_fence_after();
-      const uint32_t taddr0 = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kSub * BN);
+      const uint32_t taddr0 = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kSub * C::SUB_COLS);
+      // 16 accumulator columns (tokens) of subtile `sub`: paired hi + lo products
+      auto acc16 = [&](int sub, int cc, float (&v)[16]) {
+        tmem_ld16(taddr0 + sub * C::SUB_COLS + cc * 16, v);
+        if (C::PAIRED) {
+          float w[16];
+          tmem_ld16(taddr0 + sub * C::SUB_COLS + BN + cc * 16, w);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) v[i] += w[i];
+        }
+      };
       if (!ARGMAX) {
         int c0, c1;
         StreamK sk{a.n_work, a.kbt, a.total, G};
         sk.contributors(wt, c0, c1);
+        // lane l holds row q*32 + l; a 4 x 4 shuffle transpose per 4 tokens gives
+        // each lane 4 consecutive rows of one token: one float4 store, not four
+        const int li = lane & 3;
 #pragma unroll 1
         for (int sub = 0; sub < kSub; ++sub) {
-          float* dst = a.part + (size_t)(cta - c0) * kMaxT * n_part + (size_t)(wt * kSub + sub) * kTile + row;
+          float* dst = a.part + (size_t)(cta - c0) * kMaxT * n_part + (size_t)(wt * kSub + sub) * kTile + q * 32 +
+                       (lane & ~3);
 #pragma unroll 1
           for (int cc = 0; cc < BN / 16; ++cc) {
             if (cc * 16 >= a.T) break;
             float v[16];
-            tmem_ld16(taddr0 + sub * BN + cc * 16, v);
+            acc16(sub, cc, v);
 #pragma unroll
-            for (int i = 0; i < 16; ++i) {
-              const int t = cc * 16 + i;
-              if (t < a.T) dst[(size_t)t * n_part] = v[i];
+            for (int b = 0; b < 4; ++b) {
+              float x0 = v[4 * b], x1 = v[4 * b + 1], x2 = v[4 * b + 2], x3 = v[4 * b + 3];
+              const float y0 = __shfl_xor_sync(0xffffffffu, (li & 1) ? x0 : x1, 1);
+              const float y1 = __shfl_xor_sync(0xffffffffu, (li & 1) ? x2 : x3, 1);
+              if (li & 1) {
+                x0 = y0;
+                x2 = y1;
+              } else {
+                x1 = y0;
+                x3 = y1;
+              }
+              const float z0 = __shfl_xor_sync(0xffffffffu, (li & 2) ? x0 : x2, 2);
+              const float z1 = __shfl_xor_sync(0xffffffffu, (li & 2) ? x1 : x3, 2);
+              if (li & 2) {
+                x0 = z0;
+                x1 = z1;
+              } else {
+                x2 = z0;
+                x3 = z1;
+              }
+              const int t = cc * 16 + 4 * b + li;   // rows (lane & ~3) .. +3 of token t
+              if (t < a.T) *reinterpret_cast<float4*>(dst + (size_t)t * n_part) = make_float4(x0, x1, x2, x3);
             }
           }
         }
@@ -591,7 +636,7 @@ __global__ void __launch_bounds__(192, 1)
           for (int cc = 0; cc < BN / 16; ++cc) {
             if (cc * 16 >= a.T) break;
             float v[16];
-            tmem_ld16(taddr0 + sub * BN + cc * 16, v);
+            acc16(sub, cc, v);
 #pragma unroll
             for (int i = 0; i < 16; ++i) {
               Top2s s{f < a.N ? v[i] * rms[cc * 16 + i] : -INFINITY, f, -INFINITY};

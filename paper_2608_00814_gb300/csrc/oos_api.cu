@@ -60,7 +60,7 @@ size_t carve_workspace(const oos_model_config& c, int n_sms, uint8_t* base, Work
   const size_t halves = c.dtype == OOS_DTYPE_BF16 ? 2 : 1;   // bf16: hi rows then lo rows
   w.x = (float*)take(kMaxT * H * 4);
   w.xn = take(halves * kMaxT * H * es);
-  w.q = take(kMaxT * qd * es);
+  w.q = take(halves * kMaxT * qd * es);
   w.attn = take(halves * kMaxT * qd * es);
   w.act = take(halves * kMaxT * I * es);
   size_t pf = 0;
