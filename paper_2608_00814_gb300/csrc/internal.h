@@ -118,6 +118,16 @@ struct Model {
   std::vector<GemmW> g_qkv, g_o, g_gu, g_down;
   GemmW g_lm;
   CUtensorMap amap_xn[4], amap_attn[4], amap_act[4];  // per N-tile variant 16/32/64/128
+  CUtensorMap qmap_hi, qmap_lo;   // attention: q rows of one kv head, (d, head in group, kv head, node)
+  // attention: the last K/V cache maps encoded per layer (re-encoded only when
+  // the cache pointers or the valid extent change)
+  struct KvMaps {
+    const void* k = nullptr;
+    const void* v = nullptr;
+    int extent = -1;
+    CUtensorMap kmap, vmap;
+  };
+  std::vector<KvMaps> kv_maps;
   int lm_grid;
   // fp32 path plans (one slice)
   StreamK p_qkv, p_o, p_gu, p_down;
@@ -170,6 +180,10 @@ cudaError_t launch_accept_walk(const int32_t* tokens, const int32_t* parent, con
 
 // ---- GEMMs (gemm.cu)
 bool encode_weight_map(CUtensorMap* map, const void* ptr, int rows, int K);
+// bf16 tensor map with 128-byte swizzle: dims[0] contiguous, strides[i] = bytes
+// between consecutive indices of dim i + 1, box[] elements per dim
+bool encode_bf16_map(CUtensorMap* map, const void* ptr, int rank, const uint64_t* dims, const uint64_t* strides,
+                     const uint32_t* box);
 bool encode_act_map(CUtensorMap* map, const void* ptr, int K, int box_rows);
 int bn_index(int T);   // N-tile variant for T tree nodes: 0..3 -> 16/32/64/128
 cudaError_t gemm_setup();
@@ -187,6 +201,8 @@ cudaError_t launch_lm_head_f32(Model& m, int T, cudaStream_t st);
 
 // ---- attention (attn.cu)
 cudaError_t attn_setup();
-cudaError_t launch_attention(Model& m, const void* kc, const void* vc, int ctx, int T, cudaStream_t st);
+int attn_nodes_per_block(int group);   // tree nodes per attention block (x group q heads <= 128 rows)
+bool attn_encode_q_maps(Model& m);     // TMA maps of the q buffer (bf16 path), at model creation
+cudaError_t launch_attention(Model& m, int layer, const void* kc, const void* vc, int ctx, int T, cudaStream_t st);
 
 }  // namespace oos

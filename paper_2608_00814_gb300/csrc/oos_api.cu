@@ -156,14 +156,14 @@ static int enqueue_verify(Model& m, const oos_kv_cache* kv, int ctx, const int32
       // five kernels per layer; every elementwise step runs in a GEMM epilogue
       const GemmW* after_down = (l + 1 < L) ? &m.g_qkv[l + 1] : &m.g_lm;
       OOS_TRY(launch_gemm_qkv(m, l, kv->k[l], kv->v[l], ctx, T, &m.g_o[l], st));
-      OOS_TRY(launch_attention(m, kv->k[l], kv->v[l], ctx, T, st));
+      OOS_TRY(launch_attention(m, l, kv->k[l], kv->v[l], ctx, T, st));
       OOS_TRY(launch_gemm_o(m, l, T, &m.g_gu[l], st));
       OOS_TRY(launch_gemm_gu(m, l, T, &m.g_down[l], st));
       OOS_TRY(launch_gemm_down(m, l, T, after_down, st));
     } else {
       OOS_TRY(launch_gemm_f32(m, W.w_q, W.w_k, W.w_v, qd, kvd, kvd, c.hidden, m.ws.xn, T, st));
       OOS_TRY(launch_qkv_post(m, l, m.p_qkv, kv->k[l], kv->v[l], ctx, T, st));
-      OOS_TRY(launch_attention(m, kv->k[l], kv->v[l], ctx, T, st));
+      OOS_TRY(launch_attention(m, l, kv->k[l], kv->v[l], ctx, T, st));
       OOS_TRY(launch_gemm_f32(m, W.w_o, nullptr, nullptr, c.hidden, 0, 0, qd, m.ws.attn, T, st));
       OOS_TRY(launch_resid_norm(m, m.p_o, W.mlp_norm, nullptr, T, st));
       OOS_TRY(launch_gemm_f32(m, W.w_gate, W.w_up, nullptr, c.intermediate, c.intermediate, 0, c.hidden, m.ws.xn, T,
@@ -350,6 +350,7 @@ int oos_model_create(const oos_model_config* cfg, const oos_weights* w, void* wo
         ok = encode_act_map(&m->amap_xn[b], m->ws.xn, H, boxes[b]) &&
              encode_act_map(&m->amap_attn[b], m->ws.attn, qd, boxes[b]) &&
              encode_act_map(&m->amap_act[b], m->ws.act, I, boxes[b]);
+      ok = ok && attn_encode_q_maps(*m);
       if (!ok) {
         rc = OOS_ECUDA;
         break;
@@ -472,7 +473,7 @@ int oos_launch_attention(oos_model* m, const oos_kv_cache* kv, int32_t layer, in
   if (layer < 0 || layer >= m->cfg.n_layers || !kv->k[layer] || !kv->v[layer]) return OOS_EINVAL;
   if (T < 1 || T > m->cfg.max_T || ctx_len < 0) return OOS_EINVAL;
   if ((long long)ctx_len + T > kv->capacity) return OOS_ECAPACITY;
-  return launch_attention(*m, kv->k[layer], kv->v[layer], ctx_len, T, (cudaStream_t)stream) == cudaSuccess ? OOS_OK
+  return launch_attention(*m, layer, kv->k[layer], kv->v[layer], ctx_len, T, (cudaStream_t)stream) == cudaSuccess ? OOS_OK
                                                                                                         : OOS_ECUDA;
 }
 
