@@ -405,16 +405,13 @@ __global__ void __launch_bounds__(224, 1) k_attn_tc(const __grid_constant__ Attn
       // masked keys: past the cache end of a partial tile, tree slots that are
       // not ancestors of this node (a tile-uniform branch: full cache tiles skip it)
       if (tree || key_end < key0 + kAttnKeys) {
+        // key key0 + i is valid when i < n_valid and, for tree tile tt, bit i of
+        // the node's ancestor word tt (tree slot 64 tt + i) is set
+        const int n_valid = key_end - key0;
+        const unsigned long long word = !tree ? ~0ull : ((key0 - ctx) < 64 ? anc0 : anc1);
 #pragma unroll
-        for (int i = 0; i < kAttnKeys; ++i) {
-          const int key = key0 + i;
-          bool valid = key < key_end;
-          if (tree && valid) {
-            const int jn = key - ctx;
-            valid = ((jn < 64 ? (anc0 >> jn) : (anc1 >> (jn - 64))) & 1ull) != 0;
-          }
-          if (!valid) s[i] = -INFINITY;
-        }
+        for (int i = 0; i < kAttnKeys; ++i)
+          if (i >= n_valid || !((word >> i) & 1ull)) s[i] = -INFINITY;
       }
       // row maximum of the raw scores, four independent chains
       float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};

@@ -371,7 +371,8 @@ __global__ void __launch_bounds__(192, 1)
       mbar_init(&acce[b], 4);
     }
     mbar_init(drain, 1);
-    *abort_flag = 0;
+    abort_flag[0] = 0;
+    abort_flag[1] = 0;
     mbar_fence_init();
   }
   if (warp == 2) tmem_alloc(tmem_slot, C::NCOLS);
@@ -548,6 +549,16 @@ __global__ void __launch_bounds__(192, 1)
     const int q = warp & 3;               // TMEM lane quarter this warp may access
     const int row = q * 32 + lane;
     const int e = threadIdx.x - 64;       // 0..127
+    // Abort decisions of the epilogue warps are taken on one sample of the
+    // flag, so all 128 threads leave together and no named barrier is left
+    // waiting for threads that have gone.
+    volatile int* epi_abort = abort_flag + 1;
+    auto epi_aborted = [&]() -> bool {
+      epi_bar();
+      if (e == 0) *epi_abort = *abort_flag;
+      epi_bar();
+      return *epi_abort != 0;
+    };
     if (EPI != EPI_RESID) {
       if (e < a.T) {
         float s = 0.f;
@@ -565,7 +576,8 @@ __global__ void __launch_bounds__(192, 1)
       unit_tile(j, wt, kb);
       int seg_end = j + (a.kbt - kb);
       if (seg_end > n_units) seg_end = n_units;
-      if (!mbar_wait(&accf[acc], acc_use[acc] & 1u, abort_flag, a.status)) break;
+      mbar_wait(&accf[acc], acc_use[acc] & 1u, abort_flag, a.status);
+      if (epi_aborted()) break;
       tc_fence_after();
       const uint32_t taddr0 = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kSub * C::SUB_COLS);
       // 16 accumulator columns (tokens) of subtile `sub`: paired hi + lo products
@@ -671,7 +683,7 @@ __global__ void __launch_bounds__(192, 1)
       acc ^= 1;
       j = seg_end;
     }
-    if (!ARGMAX && !*abort_flag) {
+    if (!ARGMAX && !epi_aborted()) {
       // Finish every work tile this CTA touched: once all nc contributions of
       // the tile have arrived, contributor i (in CTA order) finishes token rows
       // [T*i/nc, T*(i+1)/nc) -- slices are still added in slice order, so the
@@ -692,6 +704,10 @@ __global__ void __launch_bounds__(192, 1)
         if (e == 0) {
           const unsigned long long t0 = globaltimer();
           while (*(volatile int*)&a.cnt[wt] < nc) {
+            if (*abort_flag || (*(volatile uint32_t*)a.status & ST_TIMEOUT)) {
+              *abort_flag = 1;
+              break;
+            }
             if (globaltimer() - t0 > kWaitLimitNs) {
               atomicOr(a.status, ST_TIMEOUT);
               *abort_flag = 1;
@@ -699,8 +715,7 @@ __global__ void __launch_bounds__(192, 1)
             }
           }
         }
-        epi_bar();
-        if (*abort_flag) break;
+        if (epi_aborted()) break;
         __threadfence();
         const int share = cta - c0;
         const int tb = (int)((long long)a.T * share / nc), te = (int)((long long)a.T * (share + 1) / nc);
