@@ -11,12 +11,16 @@
 // tiles (cache tiles first, the tree tail last, masked with the 128-bit
 // ancestor sets).  The blocks of the different ranges of the same rows form
 // one cluster.  Per tile: S = q K^T on the tensor cores into TMEM (q as hi + lo
-// bf16 halves, two MMA passes), a softmax pass with one thread per row reading
-// its S row from TMEM, P (bf16) to shared memory, O += P V on the tensor cores
-// into TMEM.  The running maximum is moved only when a tile's maximum exceeds
+// bf16 halves, two MMA passes, with q itself held in TMEM as the A operand), a
+// softmax pass with one thread per row reading its S row from TMEM and writing
+// P (bf16) back into TMEM, O += P V on the tensor cores into TMEM (P the A
+// operand from TMEM).  Two threads issue the MMAs, one the S products and one
+// the P.V products, so neither waits behind the other's barriers.  The
+// running maximum is moved only when a tile's maximum exceeds
 // it by more than 2^8 (O rescaled in TMEM then); otherwise exp2(s - m) stays
-// below 256.  V tiles are transposed in shared memory (ldmatrix +
-// stmatrix.trans) so that both MMA operands are K-major.  Each block then
+// below 256.  V tiles enter the P.V MMA as they arrive ([key][d], d
+// contiguous: the MN-major operand layout), through a ring of kKvStages K and V
+// tiles that keeps several tile loads in flight.  Each block then
 // leaves its unnormalised O and (max, sum) in its own shared memory, and after
 // a cluster barrier every block merges a slice of the rows by log-sum-exp,
 // reading the other blocks' shared memory (fixed split order), and writes the
@@ -39,22 +43,27 @@ constexpr int kAttnD = 128;       // head dim of the bf16 path
 // shared memory (bytes): operand tiles in the 128-byte-swizzled K-major layout
 constexpr int kQBytes = 2 * kAttnRows * 128;       // 64 of d per 128-byte block: 2 blocks x 128 rows
 constexpr int kKBytes = 2 * kAttnKeys * 128;       // K tile: 2 d-blocks x 64 keys
-constexpr int kVtBytes = kAttnD * 128;             // V^T tile: 128 d-rows x 64 keys
-constexpr int kPBytes = kAttnRows * 128;           // P tile: 128 rows x 64 keys
-constexpr int kVrawBytes = 2 * kAttnKeys * 128;   // raw V tile: 2 d-blocks x 64 keys, swizzled
+constexpr int kVBytes = 2 * kAttnKeys * 128;       // V tile: 2 d-blocks x 64 keys
+constexpr int kKvStages = 4;                       // K and V tiles in flight
 constexpr int kOffQhi = 0;
 constexpr int kOffQlo = kOffQhi + kQBytes;
-constexpr int kOffK = kOffQlo + kQBytes;           // [2]
-constexpr int kOffVt = kOffK + 2 * kKBytes;        // [2]
-constexpr int kOffP = kOffVt + 2 * kVtBytes;       // [2]
-constexpr int kOffVraw = kOffP + 2 * kPBytes;      // [2]
-constexpr int kOffBar = kOffVraw + 2 * kVrawBytes;
+constexpr int kOffK = kOffQlo + kQBytes;           // [kKvStages]
+constexpr int kOffV = kOffK + kKvStages * kKBytes; // [kKvStages]
+constexpr int kOffBar = kOffV + kKvStages * kVBytes;
 constexpr int kAttnSmem = kOffBar + 256 + 1024;    // + barriers + alignment slack
+constexpr int kAttnThreads = 224;                  // 7 warps, roles below
 constexpr int kOLd = kAttnD + 4;                   // merge staging row (floats)
-constexpr int kOffStage = kOffK;                   // merge staging reuses K, V^T, P
-static_assert(kOffStage + kAttnRows * kOLd * 4 + kAttnRows * 8 + kAttnRows * 8 * 4 <= kOffVraw + 2 * kVrawBytes,
-              "merge staging");
-constexpr int kAttnTmemCols = 256;                 // S[2] (64 columns each), O (128 columns)
+constexpr int kOffStage = kOffK;                   // merge staging reuses K and V
+static_assert(kOffStage + kAttnRows * kOLd * 4 + kAttnRows * 8 + kAttnRows * 8 * 4 <= kOffBar, "merge staging");
+static_assert(kAttnSmem <= 227 * 1024, "shared memory per block");
+// TMEM columns (lane = query row): S[2] fp32 scores of a tile, O fp32, q hi
+// and lo as packed bf16 pairs along d, P[2] as packed bf16 pairs along the keys
+constexpr int kTmS = 0;                            // [2] x 64
+constexpr int kTmO = 2 * kAttnKeys;                // 128
+constexpr int kTmQ = kTmO + kAttnD;                // [hi, lo] x 64
+constexpr int kTmP = kTmQ + 2 * (kAttnD / 2);      // [2] x 32
+constexpr int kAttnTmemCols = 512;                 // power of two >= kTmP + 64
+static_assert(kTmP + 2 * (kAttnKeys / 2) <= kAttnTmemCols, "TMEM columns");
 
 struct AttnArgs {
   CUtensorMap qhi, qlo;     // q [node][nq][d] as (d, head in group, kv head, node), hi and lo halves
@@ -106,16 +115,28 @@ OOS_DEV void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memo
 template <int N>
 OOS_DEV void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
 
-OOS_DEV void ldsm_x4(uint32_t (&r)[4], const void* p) {
-  asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
-               : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3])
-               : "r"(smem_addr(p)));
+// Shared-memory descriptor of an MN-major operand in the 128-byte-swizzled
+// layout: 64 consecutive MN elements (bf16) per 128-byte row, one row per K
+// index, 8-row / 1024-byte swizzle atoms.  `lbo` is the byte distance between
+// consecutive 64-element MN blocks, the stride between 8-row K groups is 1024.
+// D[tmem] (+)= A[tmem] * B[smem]: A (M = 128 rows, one per lane) as packed
+// bf16 pairs, K index 2c and 2c + 1 in column c (low half first)
+OOS_DEV void tc_mma_bf16_ts(uint32_t tmem_d, uint32_t tmem_a, uint64_t bdesc, uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "setp.ne.b32 p, %4, 0;\n\t"
+      "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(tmem_d),
+      "r"(tmem_a), "l"(bdesc), "r"(idesc), "r"(accumulate)
+      : "memory");
 }
-
-OOS_DEV void stsm_x4_t(void* p, const uint32_t (&r)[4]) {
-  asm volatile("stmatrix.sync.aligned.m8n8.x4.trans.shared.b16 [%0], {%1,%2,%3,%4};" ::"r"(smem_addr(p)), "r"(r[0]),
-               "r"(r[1]), "r"(r[2]), "r"(r[3])
-               : "memory");
+OOS_DEV uint64_t smem_desc_sw128_mn(uint32_t saddr, uint32_t lbo) {
+  uint64_t d = 0;
+  d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+  d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+  d |= (uint64_t)(1024u >> 4) << 32;
+  d |= (uint64_t)1 << 46;
+  d |= (uint64_t)2 << 61;
+  return d;
 }
 OOS_DEV void cp_async_arrive(uint64_t* bar) {   // arrive once this thread's earlier cp.async have landed
   asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(smem_addr(bar)) : "memory");
@@ -140,13 +161,23 @@ OOS_DEV void tmem_st16(uint32_t taddr, const float (&v)[16]) {
       : "memory");
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
+// 32 lanes x 32 bit, 16 consecutive columns per thread, TMEM <- raw words
+OOS_DEV void tmem_st16u(uint32_t taddr, const uint32_t* v) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
+          taddr),
+      "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]), "r"(v[9]),
+      "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
 // 16-byte chunk c of row r of a 128-byte-swizzled tile (rows 128 bytes apart,
 // 8-row / 1024-byte swizzle atoms, tile base 1024-aligned)
 OOS_DEV uint32_t sw128(int r, int c) { return (uint32_t)(r * 128 + ((c ^ (r & 7)) << 4)); }
 
 // sites of the bounded waits (recorded on the status word when one expires)
-enum { AW_KEMPTY = 21, AW_VRAW_EMPTY, AW_VFULL, AW_PV_FOR_VT, AW_QFULL, AW_KFULL, AW_SEMPTY, AW_PFULL, AW_VTFULL,
-       AW_SFULL, AW_PV_RESCALE, AW_PV_FOR_P, AW_ODONE };
+enum { AW_KEMPTY = 21, AW_VEMPTY, AW_QFULL, AW_KFULL, AW_SEMPTY, AW_PFULL, AW_VFULL, AW_SFULL, AW_PV_RESCALE,
+       AW_PV_FOR_P, AW_ODONE };
 OOS_DEV bool attn_wait(uint64_t* bar, uint32_t parity, volatile int* abort, uint32_t* status, uint32_t site, int ti) {
   if (mbar_wait(bar, parity, abort, status)) return true;
   if (*(volatile uint32_t*)(status + 1) == 0u && (*(volatile uint32_t*)status & ST_TIMEOUT))
@@ -154,25 +185,26 @@ OOS_DEV bool attn_wait(uint64_t* bar, uint32_t parity, volatile int* abort, uint
   return false;
 }
 
-// Block roles: warp 0 loads (q once, K and raw V per tile, cp.async into the
-// swizzled layouts); warp 1 lane 0 issues tcgen05.mma; warps 2..5 run the
-// softmax (thread = query row = TMEM lane); warp 6 transposes V tiles.
-__global__ void __launch_bounds__(224, 1) k_attn_tc(const __grid_constant__ AttnArgs a) {
+// Block roles: warp 0 lane 0 loads (q once, K and V per tile, by TMA into the
+// swizzled layouts); warp 1 lane 0 issues the S MMAs, warp 6 lane 0 the P.V
+// MMAs; warps 2..5 run the softmax (thread = query row = TMEM lane).
+__global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_constant__ AttnArgs a) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* sm = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bar = reinterpret_cast<uint64_t*>(sm + kOffBar);
-  uint64_t* qfull = bar;            // TMA transaction bytes
-  uint64_t* kfull = bar + 1;        // [2] TMA transaction bytes
-  uint64_t* kempty = bar + 3;       // [2] S MMAs done
-  uint64_t* vfull = bar + 5;        // [2] TMA transaction bytes
-  uint64_t* vraw_empty = bar + 7;   // [2] transposer
-  uint64_t* vtfull = bar + 9;       // [2] transposer
-  uint64_t* sfull = bar + 11;       // [2] S MMAs done
-  uint64_t* sempty = bar + 13;      // [2] 4 softmax warps
-  uint64_t* pfull = bar + 15;       // [2] 4 softmax warps
-  uint64_t* pvdone = bar + 17;      // [2] P.V MMAs done (P and V^T buffers free, O current)
-  uint64_t* odone = bar + 19;       // all MMAs done
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar + 20);
+  uint64_t* qfull = bar;                      // TMA transaction bytes
+  uint64_t* kfull = bar + 1;                  // [kKvStages] TMA transaction bytes
+  uint64_t* kempty = kfull + kKvStages;       // [kKvStages] S MMAs done
+  uint64_t* vfull = kempty + kKvStages;       // [kKvStages] TMA transaction bytes
+  uint64_t* vempty = vfull + kKvStages;       // [kKvStages] P.V MMAs done
+  uint64_t* sfull = vempty + kKvStages;       // [2] S MMAs done
+  uint64_t* sempty = sfull + 2;               // [2] 4 softmax warps
+  uint64_t* pfull = sempty + 2;               // [2] 4 softmax warps
+  uint64_t* pvdone = pfull + 2;               // [2] P.V MMAs done (P buffer free, O current)
+  uint64_t* odone = pvdone + 2;               // all MMAs of both issuers done
+  uint64_t* qtm = odone + 1;                  // 4 softmax warps: q rows are in TMEM
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(qtm + 1);
+  static_assert((1 + 4 * kKvStages + 10) * 8 + 8 <= 256, "barrier block");
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   // the argument block is addressable (its TMA maps are passed by address), so
   // its fields are read once into registers here rather than in the loops
@@ -207,18 +239,20 @@ __global__ void __launch_bounds__(224, 1) k_attn_tc(const __grid_constant__ Attn
 
   if (threadIdx.x == 0) {
     mbar_init(qfull, 1);
+    for (int s = 0; s < kKvStages; ++s) {
+      mbar_init(&kfull[s], 1);
+      mbar_init(&kempty[s], 1);
+      mbar_init(&vfull[s], 1);
+      mbar_init(&vempty[s], 1);
+    }
     for (int b = 0; b < 2; ++b) {
-      mbar_init(&kfull[b], 1);
-      mbar_init(&kempty[b], 1);
-      mbar_init(&vfull[b], 1);
-      mbar_init(&vraw_empty[b], 1);
-      mbar_init(&vtfull[b], 1);
       mbar_init(&sfull[b], 1);
       mbar_init(&sempty[b], 4);
       mbar_init(&pfull[b], 4);
       mbar_init(&pvdone[b], 1);
     }
-    mbar_init(odone, 1);
+    mbar_init(odone, 2);   // both MMA issuers
+    mbar_init(qtm, 4);
     *abort_flag = 0;
     mbar_fence_init();
   }
@@ -234,7 +268,7 @@ __global__ void __launch_bounds__(224, 1) k_attn_tc(const __grid_constant__ Attn
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const uint32_t tmem_o = tmem + 2 * kAttnKeys;
+  const uint32_t tmem_o = tmem + kTmO;
 
   if (warp == 0) {
     // ------------------------------------------------------------ loader (one thread, TMA)
@@ -255,21 +289,21 @@ __global__ void __launch_bounds__(224, 1) k_attn_tc(const __grid_constant__ Attn
       tma_prefetch_desc(&a.kmap);
       tma_prefetch_desc(&a.vmap);
       const uint64_t pol_kv = policy_evict_first();
-      auto load_kv = [&](int ti, bool v) {   // K or raw V tile: two 64-wide d blocks of 64 keys
+      auto load_kv = [&](int ti, bool v) {   // K or V tile: two 64-wide d blocks of 64 keys
         int k0, ke;
         bool tr;
         tile_keys(ti, k0, ke, tr);
-        const int b = ti & 1;
-        uint64_t* full = v ? &vfull[b] : &kfull[b];
-        unsigned char* dst = sm + (v ? kOffVraw + b * kVrawBytes : kOffK + b * kKBytes);
+        const int s = ti % kKvStages;
+        uint64_t* full = v ? &vfull[s] : &kfull[s];
+        unsigned char* dst = sm + (v ? kOffV + s * kVBytes : kOffK + s * kKBytes);
         mbar_arrive_expect_tx(full, 2 * kAttnKeys * 128);
         tma_load_3d(dst, v ? &a.vmap : &a.kmap, full, 0, g, k0, pol_kv);
         tma_load_3d(dst + kAttnKeys * 128, v ? &a.vmap : &a.kmap, full, 64, g, k0, pol_kv);
       };
-      // cache tiles do not depend on the producing kernel: the first two are
-      // fetched before waiting for it; tree tiles and q after
+      // cache tiles do not depend on the producing kernel: the first stages
+      // are fetched before waiting for it; tree tiles and q after
       int pre = 0;
-      for (int ti = 0; ti < n_tiles && ti < 2; ++ti) {
+      for (int ti = 0; ti < n_tiles && ti < kKvStages; ++ti) {
         int k0, ke;
         bool tr;
         tile_keys(ti, k0, ke, tr);
@@ -290,99 +324,76 @@ __global__ void __launch_bounds__(224, 1) k_attn_tc(const __grid_constant__ Attn
       tma_load_4d(sm + kOffQlo, &a.qlo, qfull, 0, 0, g, node0, pol_q);
       tma_load_4d(sm + kOffQlo + kAttnRows * 128, &a.qlo, qfull, 64, 0, g, node0, pol_q);
       for (int ti = pre; ti < n_tiles; ++ti) {
-        const int b = ti & 1;
-        const uint32_t use = (uint32_t)(ti >> 1);
-        if (!attn_wait(&kempty[b], (use & 1u) ^ 1u, abort_flag, status, AW_KEMPTY, ti)) break;
+        const int st = ti % kKvStages;
+        const uint32_t use = (uint32_t)(ti / kKvStages);
+        if (!attn_wait(&kempty[st], (use & 1u) ^ 1u, abort_flag, status, AW_KEMPTY, ti)) break;
         load_kv(ti, false);
-        if (!attn_wait(&vraw_empty[b], (use & 1u) ^ 1u, abort_flag, status, AW_VRAW_EMPTY, ti)) break;
+        if (!attn_wait(&vempty[st], (use & 1u) ^ 1u, abort_flag, status, AW_VEMPTY, ti)) break;
         load_kv(ti, true);
       }
     }
-  } else if (warp == 6) {
-    // ------------------------------------------------------------ V transposer
-    // raw V [key][d] -> V^T [d][key], 128-byte rows of 64 keys, swizzled:
-    // ldmatrix reads four 8 x 8 (key x d) blocks, stmatrix.trans writes them as
-    // (d x key) rows
-    for (int ti = 0; ti < n_tiles; ++ti) {
-      const int b = ti & 1;
-      const uint32_t use = (uint32_t)(ti >> 1);
-      bool ok = true;
-      if (lane == 0) {
-        ok = attn_wait(&vfull[b], use & 1u, abort_flag, status, AW_VFULL, ti) &&
-             attn_wait(&pvdone[b], (use & 1u) ^ 1u, abort_flag, status, AW_PV_FOR_VT, ti);
-      }
-      ok = __shfl_sync(0xffffffffu, ok, 0);
-      if (!ok) break;
-      const unsigned char* vr = sm + kOffVraw + b * kVrawBytes;   // [d block][64 keys][128 B], swizzled
-      unsigned char* vt = sm + kOffVt + b * kVtBytes;
-      const int i = lane >> 3, j = lane & 7;   // matrix i of the x4, row j of it
-#pragma unroll 4
-      for (int blk = 0; blk < 32; ++blk) {
-        const int kb = blk >> 2;                // 8-key block
-        const int db = (blk & 3) * 4 + i;       // 8-d block of matrix i
-        uint32_t r[4];
-        ldsm_x4(r, vr + (db >> 3) * (kAttnKeys * 128) + sw128(kb * 8 + j, db & 7));
-        // row j of the transposed matrix i: d = db*8 + j, keys kb*8 .. kb*8+7
-        stsm_x4_t(vt + sw128(db * 8 + j, kb), r);
-      }
-      fence_async_smem();
-      __syncwarp();
-      if (lane == 0) {
-        mbar_arrive(&vraw_empty[b]);
-        mbar_arrive(&vtfull[b]);
-      }
-    }
-  } else if (warp == 1) {
-    // ------------------------------------------------------------ MMA issuer
-    if (lane == 0) {
+  } else if (warp == 1 || warp == 6) {
+    // ------------------------------------------------------------ MMA issuers
+    // warp 1 lane 0 issues S = q K^T, warp 6 lane 0 issues O += P V: two
+    // threads, so that neither kind waits behind the other's barriers and the
+    // tensor cores always have queued work.  Operands reach the tensor cores
+    // through the async proxy only: q, K and V by TMA, P from threads that
+    // fence before they arrive on pfull (the zeroed q padding rows were fenced
+    // before the block barrier).  Descriptors: the start address is the low
+    // field (16-byte units), so a byte offset o inside an operand region is
+    // added as o >> 4.
+    if (lane == 0 && warp == 1) {
       constexpr uint32_t idesc_s = idesc_bf16_f32(kAttnRows, kAttnKeys);
-      constexpr uint32_t idesc_pv = idesc_bf16_f32(kAttnRows, kAttnD);
-      bool ok = attn_wait(qfull, 0, abort_flag, status, AW_QFULL, 0);
-      fence_async_smem();   // cp.async (generic proxy) writes -> tensor-core reads (async proxy)
+      bool ok = attn_wait(qtm, 0, abort_flag, status, AW_QFULL, 0);
       tc_fence_after();
-      auto issue_pv = [&](int ti) {
-        const int b = ti & 1;
-        const uint32_t use = (uint32_t)(ti >> 1);
-        if (!attn_wait(&pfull[b], use & 1u, abort_flag, status, AW_PFULL, ti)) return false;
-        if (!attn_wait(&vtfull[b], use & 1u, abort_flag, status, AW_VTFULL, ti)) return false;
-        fence_async_smem();
-        tc_fence_after();
-        const uint64_t pd = smem_desc_sw128(smem_addr(sm + kOffP + b * kPBytes));
-        const uint64_t vd = smem_desc_sw128(smem_addr(sm + kOffVt + b * kVtBytes));
-#pragma unroll
-        for (int kk = 0; kk < kAttnKeys / 16; ++kk)
-          tc_mma_bf16(tmem_o, pd + 2 * kk, vd + 2 * kk, idesc_pv, (ti > 0 || kk > 0) ? 1u : 0u);
-        tc_commit(&pvdone[b]);
-        return true;
-      };
+      const uint64_t kdesc0 = smem_desc_sw128(smem_addr(sm + kOffK));
+      // S buffer ti & 1 is free once the softmax has read tile ti - 2's scores,
+      // before P of tile ti - 2 is ready: the scores run ahead of the softmax
       for (int ti = 0; ti < n_tiles && ok; ++ti) {
         const int b = ti & 1;
         const uint32_t use = (uint32_t)(ti >> 1);
-        if (!attn_wait(&kfull[b], use & 1u, abort_flag, status, AW_KFULL, ti) ||
-            !attn_wait(&sempty[b], (use & 1u) ^ 1u, abort_flag, status, AW_SEMPTY, ti)) {
-          ok = false;
+        const int st = ti % kKvStages;
+        if (!attn_wait(&kfull[st], (uint32_t)(ti / kKvStages) & 1u, abort_flag, status, AW_KFULL, ti) ||
+            !attn_wait(&sempty[b], (use & 1u) ^ 1u, abort_flag, status, AW_SEMPTY, ti))
           break;
-        }
-        fence_async_smem();
         tc_fence_after();
-        const uint32_t ks = smem_addr(sm + kOffK + b * kKBytes);
-        const uint32_t d = tmem + b * kAttnKeys;
-        // S = q_hi K^T + q_lo K^T over the 128 head dims (two 64-wide blocks)
+        const uint64_t kd0 = kdesc0 + (uint64_t)((st * kKBytes) >> 4);
+        const uint32_t d = tmem + kTmS + b * kAttnKeys;
+        // S = q_hi K^T + q_lo K^T over the 128 head dims: q from TMEM (8
+        // columns = 16 of d per MMA), K from the two 64-wide d blocks (32 bytes
+        // of d per MMA)
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
-          const uint32_t qs = smem_addr(sm + (half ? kOffQlo : kOffQhi));
 #pragma unroll
           for (int k = 0; k < kAttnD / 16; ++k) {
-            const uint64_t qd = smem_desc_sw128(qs + (k >> 2) * (kAttnRows * 128)) + 2 * (k & 3);
-            const uint64_t kd = smem_desc_sw128(ks + (k >> 2) * (kAttnKeys * 128)) + 2 * (k & 3);
-            tc_mma_bf16(d, qd, kd, idesc_s, (half > 0 || k > 0) ? 1u : 0u);
+            const uint64_t kd = kd0 + (uint64_t)(((k >> 2) * (kAttnKeys * 128)) >> 4) + 2 * (k & 3);
+            tc_mma_bf16_ts(d, tmem + kTmQ + half * (kAttnD / 2) + 8 * k, kd, idesc_s, (half > 0 || k > 0) ? 1u : 0u);
           }
         }
-        tc_commit(&kempty[b]);
+        tc_commit(&kempty[st]);
         tc_commit(&sfull[b]);
-        if (ti >= 1 && !issue_pv(ti - 1)) ok = false;
       }
-      if (ok && n_tiles > 0) issue_pv(n_tiles - 1);
+      tc_commit(odone);
+    } else if (lane == 0 && warp == 6) {
+      constexpr uint32_t idesc_pv = idesc_bf16_f32(kAttnRows, kAttnD) | (1u << 16);   // B (V) MN-major
+      // V tile: d blocks of 64 (8 KB apart) along N, 16 keys (2 KB) per MMA along K
+      const uint64_t vdesc0 = smem_desc_sw128_mn(smem_addr(sm + kOffV), kAttnKeys * 128);
+      for (int ti = 0; ti < n_tiles; ++ti) {
+        const int b = ti & 1;
+        const uint32_t use = (uint32_t)(ti >> 1);
+        const int st = ti % kKvStages;
+        if (!attn_wait(&pfull[b], use & 1u, abort_flag, status, AW_PFULL, ti) ||
+            !attn_wait(&vfull[st], (uint32_t)(ti / kKvStages) & 1u, abort_flag, status, AW_VFULL, ti))
+          break;
+        tc_fence_after();
+        const uint32_t pt = tmem + kTmP + b * (kAttnKeys / 2);   // P: 8 columns = 16 keys per MMA
+        const uint64_t vd = vdesc0 + (uint64_t)((st * kVBytes) >> 4);
+#pragma unroll
+        for (int kk = 0; kk < kAttnKeys / 16; ++kk)
+          tc_mma_bf16_ts(tmem_o, pt + 8 * kk, vd + (uint64_t)((kk * 16 * 128) >> 4), idesc_pv, (ti > 0 || kk > 0) ? 1u : 0u);
+        tc_commit(&pvdone[b]);
+        tc_commit(&vempty[st]);
+      }
       tc_commit(odone);
     }
   }
@@ -396,7 +407,30 @@ __global__ void __launch_bounds__(224, 1) k_attn_tc(const __grid_constant__ Attn
     const int node = min(rb * npc + min(lrow, rows - 1) / group, T - 1);
     pdl_wait();
     const unsigned long long anc0 = anc[2 * node], anc1 = anc[2 * node + 1];
-    for (int ti = 0; ti < n_tiles; ++ti) {
+    // this thread's q row (hi, lo) from the TMA tile into TMEM, the S MMAs'
+    // A operand: 16 columns per store = 32 of d as bf16 pairs; padding rows
+    // past the block's rows are the zeroed shared-memory rows
+    const bool qok = __all_sync(0xffffffffu, attn_wait(qfull, 0, abort_flag, status, AW_QFULL, 0));
+    if (qok) {
+#pragma unroll
+      for (int part = 0; part < 8; ++part) {   // (hi/lo, 64-wide d block, half of its 8 chunks)
+        const unsigned char* qb = sm + ((part >> 2) ? kOffQlo : kOffQhi) + ((part >> 1) & 1) * (kAttnRows * 128);
+        uint32_t w[16];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+          const uint4 v = *reinterpret_cast<const uint4*>(qb + sw128(lrow, (part & 1) * 4 + c));
+          w[4 * c] = v.x;
+          w[4 * c + 1] = v.y;
+          w[4 * c + 2] = v.z;
+          w[4 * c + 3] = v.w;
+        }
+        tmem_st16u(tmem + lane_off + kTmQ + part * 16, w);
+      }
+    }
+    tc_fence_before();
+    __syncwarp();
+    if (lane == 0) mbar_arrive(qtm);
+    for (int ti = 0; ti < (qok ? n_tiles : 0); ++ti) {
       const int b = ti & 1;
       const uint32_t use = (uint32_t)(ti >> 1);
       // every wait's outcome is made warp-uniform: the .sync.aligned TMEM
@@ -407,7 +441,7 @@ __global__ void __launch_bounds__(224, 1) k_attn_tc(const __grid_constant__ Attn
 #pragma unroll
       for (int c = 0; c < kAttnKeys / 16; ++c) {
         float v[16];
-        tmem_ld16(tmem + lane_off + b * kAttnKeys + c * 16, v);
+        tmem_ld16(tmem + lane_off + kTmS + b * kAttnKeys + c * 16, v);
 #pragma unroll
         for (int i = 0; i < 16; ++i) s[c * 16 + i] = v[i];
       }
@@ -484,11 +518,10 @@ __global__ void __launch_bounds__(224, 1) k_attn_tc(const __grid_constant__ Attn
       l_sum += psum;
       // P buffer b is free once P.V of tile ti - 2 has completed
       if (!__all_sync(0xffffffffu, attn_wait(&pvdone[b], (use & 1u) ^ 1u, abort_flag, status, AW_PV_FOR_P, ti))) break;
-      unsigned char* prow = sm + kOffP + b * kPBytes;
-#pragma unroll
-      for (int c = 0; c < 8; ++c)
-        *reinterpret_cast<uint4*>(prow + sw128(lrow, c)) = make_uint4(pk[4 * c], pk[4 * c + 1], pk[4 * c + 2], pk[4 * c + 3]);
-      fence_async_smem();
+      // P into TMEM, the P.V MMAs' A operand (key pairs, 32 columns)
+      tmem_st16u(tmem + lane_off + kTmP + b * (kAttnKeys / 2), pk);
+      tmem_st16u(tmem + lane_off + kTmP + b * (kAttnKeys / 2) + 16, pk + 16);
+      tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&pfull[b]);
     }
@@ -654,7 +687,7 @@ static int attn_max_clusters(int sp) {
   if (cached[sp] == 0) {
     cudaLaunchConfig_t lc = {};
     lc.gridDim = dim3(1, 1, sp);
-    lc.blockDim = dim3(224);
+    lc.blockDim = dim3(kAttnThreads);
     lc.dynamicSmemBytes = (size_t)kAttnSmem;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeClusterDimension;
@@ -737,7 +770,7 @@ cudaError_t launch_attention(Model& m, int layer, const void* kc, const void* vc
 
   cudaLaunchConfig_t lc = {};
   lc.gridDim = dim3(RB, a.nkv, splits);
-  lc.blockDim = dim3(224);
+  lc.blockDim = dim3(kAttnThreads);
   lc.dynamicSmemBytes = (size_t)kAttnSmem;
   lc.stream = st;
   cudaLaunchAttribute attr[2];
