@@ -141,16 +141,17 @@ OOS_DEV float4 f4_add(float4 a, float4 b) { return make_float4(a.x + b.x, a.y + 
 OOS_DEV float4 f4_ldcg(const float* p) { return __ldcg(reinterpret_cast<const float4*>(p)); }
 
 // acc[k] = (init ? init row : 0) + sum over nc slices of the partial tile rows,
-// rows t = t0 + 4k + w below T (the end of the token range).  Slices are
+// rows t = t0 + nw k + w below T (the end of the token range; w is this warp's
+// index among the nw warps finishing the tile).  Slices are
 // fetched BATCH at a time -- every load of a group is issued before any is
 // added -- and added in slice order, so the sum is the same for every finisher.
 template <int R, int BATCH>
 OOS_DEV void load_tile_rows(float4 (&acc)[R], const float* __restrict__ part, int nc, size_t slice, int n_part,
-                            int col, int t0, int T, const float* __restrict__ init, int init_ld, int init_col) {
-  const int w = (threadIdx.x - 64) >> 5;
+                            int col, int t0, int T, const float* __restrict__ init, int init_ld, int init_col, int w,
+                            int nw) {
 #pragma unroll
   for (int k = 0; k < R; ++k) {
-    const int t = t0 + 4 * k + w;
+    const int t = t0 + nw * k + w;
     acc[k] = (init && t < T) ? *reinterpret_cast<const float4*>(init + (size_t)t * init_ld + init_col)
                              : make_float4(0.f, 0.f, 0.f, 0.f);
   }
@@ -161,7 +162,7 @@ OOS_DEV void load_tile_rows(float4 (&acc)[R], const float* __restrict__ part, in
       const float* base = part + (size_t)(s0 + q) * slice + col;
 #pragma unroll
       for (int k = 0; k < R; ++k) {
-        const int t = t0 + 4 * k + w;
+        const int t = t0 + nw * k + w;
         v[q][k] = (s0 + q < nc && t < T) ? f4_ldcg(base + (size_t)t * n_part) : make_float4(0.f, 0.f, 0.f, 0.f);
       }
     }
@@ -175,8 +176,7 @@ OOS_DEV void load_tile_rows(float4 (&acc)[R], const float* __restrict__ part, in
 // gate (col) and up (col + up_off) rows of a SwiGLU pair, two slices per batch
 template <int R>
 OOS_DEV void load_pair_rows(float4 (&g)[R], float4 (&u)[R], const float* __restrict__ part, int nc, size_t slice,
-                            int n_part, int col, int up_off, int t0, int T) {
-  const int w = (threadIdx.x - 64) >> 5;
+                            int n_part, int col, int up_off, int t0, int T, int w, int nw) {
 #pragma unroll
   for (int k = 0; k < R; ++k) g[k] = u[k] = make_float4(0.f, 0.f, 0.f, 0.f);
   for (int s0 = 0; s0 < nc; s0 += 2) {
@@ -186,7 +186,7 @@ OOS_DEV void load_pair_rows(float4 (&g)[R], float4 (&u)[R], const float* __restr
       const float* base = part + (size_t)(s0 + q) * slice + col;
 #pragma unroll
       for (int k = 0; k < R; ++k) {
-        const int t = t0 + 4 * k + w;
+        const int t = t0 + nw * k + w;
         const bool ok = s0 + q < nc && t < T;
         vg[q][k] = ok ? f4_ldcg(base + (size_t)t * n_part) : make_float4(0.f, 0.f, 0.f, 0.f);
         vu[q][k] = ok ? f4_ldcg(base + (size_t)t * n_part + up_off) : make_float4(0.f, 0.f, 0.f, 0.f);
@@ -208,19 +208,19 @@ OOS_DEV float4 bf16x4(const __nv_bfloat16* p) {
   return make_float4(__bfloat162float(h[0]), __bfloat162float(h[1]), __bfloat162float(h[2]), __bfloat162float(h[3]));
 }
 
-// EPI_RESID on 128-row tile `tile`, tokens [tb, te): x += W.a; y = g (.) x;
-// per-tile sums of x^2
-OOS_DEV void finish_resid(const GemmArgs& a, int n_part, int tile, int nc, int tb, int te) {
-  const int e = threadIdx.x - 64, w = e >> 5, l = e & 31;
+// EPI_RESID on 128-row tile `tile`, tokens [tb, te), by warp w of nw: x += W.a;
+// y = g (.) x; per-tile sums of x^2
+OOS_DEV void finish_resid(const GemmArgs& a, int n_part, int tile, int nc, int tb, int te, int w, int nw) {
+  const int l = threadIdx.x & 31;
   const size_t slice = (size_t)kMaxT * n_part;
   const int f = tile * kTile + 4 * l;
   const float4 g = bf16x4(a.gain + f);
-  for (int t0 = tb; t0 < te; t0 += 4 * kFinRows) {
+  for (int t0 = tb; t0 < te; t0 += nw * kFinRows) {
     float4 acc[kFinRows];
-    load_tile_rows<kFinRows, 8>(acc, a.part, nc, slice, n_part, f, t0, te, a.x, a.N, f);   // x + sum of slices
+    load_tile_rows<kFinRows, 8>(acc, a.part, nc, slice, n_part, f, t0, te, a.x, a.N, f, w, nw);   // x + sum of slices
 #pragma unroll
     for (int k = 0; k < kFinRows; ++k) {
-      const int t = t0 + 4 * k + w;
+      const int t = t0 + nw * k + w;
       if (t >= te) break;
       const float4 xv = acc[k];
       *reinterpret_cast<float4*>(a.x + (size_t)t * a.N + f) = xv;
@@ -233,19 +233,20 @@ OOS_DEV void finish_resid(const GemmArgs& a, int n_part, int tile, int nc, int t
 }
 
 // EPI_SILU on work tile wt (subtile 0 = gate rows of block wt, subtile 1 = up
-// rows), tokens [tb, te)
-OOS_DEV void finish_silu(const GemmArgs& a, int n_part, int wt, int nc, const float* rms, int tb, int te) {
-  const int e = threadIdx.x - 64, w = e >> 5, l = e & 31;
+// rows), tokens [tb, te), by warp w of nw
+OOS_DEV void finish_silu(const GemmArgs& a, int n_part, int wt, int nc, const float* rms, int tb, int te, int w,
+                         int nw) {
+  const int l = threadIdx.x & 31;
   const size_t slice = (size_t)kMaxT * n_part;
   const int i = wt * kTile + 4 * l;
-  constexpr int R = 8;   // 32 tokens per pass
-  for (int t0 = tb; t0 < te; t0 += 4 * R) {
+  constexpr int R = 8;   // 8 token rows per warp per pass
+  for (int t0 = tb; t0 < te; t0 += nw * R) {
     float4 gv[R], uv[R];
     // gate and up slices of a pass in one batch of loads
-    load_pair_rows<R>(gv, uv, a.part, nc, slice, n_part, 2 * wt * kTile + 4 * l, kTile, t0, te);
+    load_pair_rows<R>(gv, uv, a.part, nc, slice, n_part, 2 * wt * kTile + 4 * l, kTile, t0, te, w, nw);
 #pragma unroll
     for (int k = 0; k < R; ++k) {
-      const int t = t0 + 4 * k + w;
+      const int t = t0 + nw * k + w;
       if (t >= te) break;
       const float r = rms[t];
       const float g4[4] = {gv[k].x * r, gv[k].y * r, gv[k].z * r, gv[k].w * r};
@@ -259,9 +260,10 @@ OOS_DEV void finish_silu(const GemmArgs& a, int n_part, int wt, int nc, const fl
 }
 
 // EPI_QKV on 128-row tile `tile` = one head (q heads, then k heads, then v
-// heads), tokens [tb, te)
-OOS_DEV void finish_qkv(const GemmArgs& a, int n_part, int tile, int nc, const float* rms, int tb, int te) {
-  const int e = threadIdx.x - 64, w = e >> 5, l = e & 31;
+// heads), tokens [tb, te), by warp w of nw
+OOS_DEV void finish_qkv(const GemmArgs& a, int n_part, int tile, int nc, const float* rms, int tb, int te, int w,
+                        int nw) {
+  const int l = threadIdx.x & 31;
   const size_t slice = (size_t)kMaxT * n_part;
   int kind, h;
   if (tile < a.nq) { kind = 0; h = tile; }
@@ -273,12 +275,12 @@ OOS_DEV void finish_qkv(const GemmArgs& a, int n_part, int tile, int nc, const f
   const float4 g4 = gn ? bf16x4(gn + 4 * l) : make_float4(1.f, 1.f, 1.f, 1.f);
   const int m0 = 4 * (l & 15);      // rotary frequency index of this lane's first feature
   const bool first_half = l < 16;   // features 0..63 pair with 64..127 held by lane ^ 16
-  for (int t0 = tb; t0 < te; t0 += 4 * kFinRows) {
+  for (int t0 = tb; t0 < te; t0 += nw * kFinRows) {
     float4 acc[kFinRows];
-    load_tile_rows<kFinRows, 8>(acc, a.part, nc, slice, n_part, tile * kTile + 4 * l, t0, te, nullptr, 0, 0);
+    load_tile_rows<kFinRows, 8>(acc, a.part, nc, slice, n_part, tile * kTile + 4 * l, t0, te, nullptr, 0, 0, w, nw);
 #pragma unroll
     for (int k = 0; k < kFinRows; ++k) {
-      const int t = t0 + 4 * k + w;
+      const int t = t0 + nw * k + w;
       if (t >= te) break;
       const float r = rms[t];
       float v[4] = {acc[k].x * r + b4.x, acc[k].y * r + b4.y, acc[k].z * r + b4.z, acc[k].w * r + b4.w};
@@ -689,46 +691,64 @@ __global__ void __launch_bounds__(192, 1)
       // [T*i/nc, T*(i+1)/nc) -- slices are still added in slice order, so the
       // result does not depend on who finishes.  All contributors end their
       // ranges at about the same time (balanced stream-K), and the grid never
-      // exceeds one CTA per SM, so every awaited CTA is resident.
+      // exceeds one CTA per SM, so every awaited CTA is resident.  Tiles are
+      // taken two at a time: both arrival counts are awaited first, then
+      // epilogue warps 0-1 finish the first tile and warps 2-3 the second, so
+      // the two latency-bound passes overlap instead of running back to back.
       StreamK sk{a.n_work, a.kbt, a.total, G};
       int jj = 0;
       while (jj < n_units) {
-        int wt, kb;
-        unit_tile(jj, wt, kb);
-        int seg_end = jj + (a.kbt - kb);
-        if (seg_end > n_units) seg_end = n_units;
-        jj = seg_end;
-        int c0, c1;
-        sk.contributors(wt, c0, c1);
-        const int nc = c1 - c0 + 1;
+        // the next one or two work tiles of the range: (tile, contributors, token share)
+        auto next_tile = [&](int& wt, int& nc, int& tb, int& te) {
+          int kb;
+          unit_tile(jj, wt, kb);
+          int seg_end = jj + (a.kbt - kb);
+          if (seg_end > n_units) seg_end = n_units;
+          jj = seg_end;
+          int c0, c1;
+          sk.contributors(wt, c0, c1);
+          nc = c1 - c0 + 1;
+          const int share = cta - c0;
+          tb = (int)((long long)a.T * share / nc);
+          te = (int)((long long)a.T * (share + 1) / nc);
+        };
+        int wt0, nc0, tb0, te0, wt1 = -1, nc1 = 0, tb1 = 0, te1 = 0;
+        next_tile(wt0, nc0, tb0, te0);
+        if (jj < n_units) next_tile(wt1, nc1, tb1, te1);
+        const bool two = wt1 >= 0;
         if (e == 0) {
           const unsigned long long t0 = globaltimer();
-          while (*(volatile int*)&a.cnt[wt] < nc) {
-            if (*abort_flag || (*(volatile uint32_t*)a.status & ST_TIMEOUT)) {
-              *abort_flag = 1;
-              break;
-            }
-            if (globaltimer() - t0 > kWaitLimitNs) {
-              atomicOr(a.status, ST_TIMEOUT);
-              *abort_flag = 1;
-              break;
+          for (int i = 0; i < (two ? 2 : 1) && !*abort_flag; ++i) {
+            const int wt = i ? wt1 : wt0, nc = i ? nc1 : nc0;
+            while (*(volatile int*)&a.cnt[wt] < nc) {
+              if (*abort_flag || (*(volatile uint32_t*)a.status & ST_TIMEOUT)) {
+                *abort_flag = 1;
+                break;
+              }
+              if (globaltimer() - t0 > kWaitLimitNs) {
+                atomicOr(a.status, ST_TIMEOUT);
+                *abort_flag = 1;
+                break;
+              }
             }
           }
         }
         if (epi_aborted()) break;
         __threadfence();
-        const int share = cta - c0;
-        const int tb = (int)((long long)a.T * share / nc), te = (int)((long long)a.T * (share + 1) / nc);
+        const int ew = e >> 5;   // epilogue warp 0..3
+        const bool second = two && ew >= 2;
+        const int nw = two ? 2 : 4, w = two ? (ew & 1) : ew;
+        const int wt = second ? wt1 : wt0, nc = second ? nc1 : nc0, tb = second ? tb1 : tb0, te = second ? te1 : te0;
         if (tb < te) {
           if (EPI == EPI_SILU) {
-            finish_silu(a, n_part, wt, nc, rms, tb, te);
+            finish_silu(a, n_part, wt, nc, rms, tb, te, w, nw);
           } else {
 #pragma unroll 1
             for (int sub = 0; sub < kSub; ++sub) {
               const int tile = wt * kSub + sub;
               if (tile >= a.n_tiles) break;
-              if (EPI == EPI_RESID) finish_resid(a, n_part, tile, nc, tb, te);
-              else finish_qkv(a, n_part, tile, nc, rms, tb, te);
+              if (EPI == EPI_RESID) finish_resid(a, n_part, tile, nc, tb, te, w, nw);
+              else finish_qkv(a, n_part, tile, nc, rms, tb, te, w, nw);
             }
           }
         }
