@@ -868,8 +868,8 @@ template <int EPI>
 static cudaError_t dispatch_tc(Model& m, const GemmW& g, const CUtensorMap* amaps, int T, int grid, GemmArgs& a,
                                const GemmW* next, cudaStream_t st) {
   if (next) {
-    // about 128 KB of the next GEMM's weights per CTA index
-    a.pf_units = 8 / next->sub;
+    // about 64 KB of the next GEMM's weights per CTA index
+    a.pf_units = 4 / next->sub;
     a.pf_n_tiles = (next->N + kTile - 1) / kTile;
     a.pf_n_work = next->plan.n_tiles;
     a.pf_kbt = next->plan.kbt;

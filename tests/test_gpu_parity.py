@@ -252,6 +252,7 @@ def test_mini_bf16_parity_seeds(mini_models):
     (100, dict(kind="chain"), 200),
     (12, dict(kind="uniform", max_depth=5), 0),          # empty cache
     (12, dict(kind="uniform", max_depth=5), 65),         # cache one key past a tile
+    (33, dict(kind="uniform", max_depth=8), 4600),       # ~9 tiles per attention block: the K/V ring wraps
 ])
 def test_mini_bf16_shapes(mini_models, T, recipe, ctx):
     case, model = _mini(mini_models, 1, T=T, recipe=recipe, ctx_len=ctx, plant=min(3, T - 1))
