@@ -93,6 +93,20 @@ typedef struct {
     float rope_theta;      /* RoPE base; pair (m, m + d/2) turns by pos * theta^(-2m/d) */
     int32_t max_T;         /* largest tree this handle verifies, 1..128 */
     int32_t use_graph;     /* nonzero: replay a captured CUDA graph when the call's shape repeats */
+    /* Rotary frequency rescaling of Llama-3.1 targets (the paper's Llama-3.1-8B),
+     * as published with that model.  With factor F > 1, low-frequency factor lo,
+     * high-frequency factor hi (hi > lo > 0) and original context L > 0, the
+     * rate f = theta^(-2m/d) of pair m, of wavelength 2 pi / f, becomes
+     *   f            when the wavelength is below L / hi,
+     *   f / F        when it is above L / lo,
+     *   (1 - w) f / F + w f,  w = (L / wavelength - lo) / (hi - lo), otherwise.
+     * rope_factor <= 1 (0 when zero-initialised): no rescaling, the other three
+     * fields are ignored.  Invalid values make oos_model_create fail with
+     * OOS_EINVAL. */
+    float rope_factor;
+    float rope_low_freq_factor;
+    float rope_high_freq_factor;
+    int32_t rope_orig_max_pos;
 } oos_model_config;
 
 /* Per-layer weights, all DEVICE pointers. */

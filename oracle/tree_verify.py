@@ -24,6 +24,9 @@ What the paper leaves open, and the reading taken here:
     (itself included): one forward pass over a tree is therefore the same as
     causal decoding along every root-to-leaf path.
   * RoPE position of node i is ctx_len + depth(i) (rotate-half convention).
+    Llama-3.1 targets turn their low-frequency pairs slower, by the frequency
+    rescaling published with that model (rope_inv_freq); the paper runs
+    Llama-3.1-8B and does not restate it.
   * K and V are stored in the cache's format before anything attends to them
     (bf16 for the bf16 models): the tree's own K/V go through the cache too.
   * "Longest prefix" is the deepest accepted node, lowest node id on ties;
@@ -35,6 +38,9 @@ What the paper leaves open, and the reading taken here:
 Model protocol (duck-typed; the seeded input module provides one):
   m.cfg                  object with n_layers, hidden, n_q_heads, n_kv_heads,
                          head_dim, intermediate, vocab, rms_eps, rope_theta
+                         (and, for rescaled rotary frequencies, rope_factor,
+                         rope_low_freq_factor, rope_high_freq_factor,
+                         rope_orig_max_pos)
   m.layer(l)             dict of fp64 arrays: attn_norm[H], w_q[nq*d,H],
                          w_k[nkv*d,H], w_v[nkv*d,H], b_q/b_k/b_v (or None),
                          q_norm/k_norm [d] (or None), w_o[H,nq*d], mlp_norm[H],
@@ -83,14 +89,51 @@ def rms_norm(x, gain, eps):
     return x / np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + eps) * gain
 
 
-def rope(x, pos, theta):
+def rope_scaling(cfg):
+    """(factor, low_freq_factor, high_freq_factor, original_context) of a
+    model whose rotary frequencies are rescaled (Llama 3.1), else None."""
+    f = float(getattr(cfg, "rope_factor", 0.0) or 0.0)
+    if f <= 1.0:
+        return None
+    return (f, float(cfg.rope_low_freq_factor), float(cfg.rope_high_freq_factor), float(cfg.rope_orig_max_pos))
+
+
+def rope_inv_freq(d, theta, scaling=None):
+    """Turning rates of the d/2 dimension pairs: theta^(-2m/d), optionally
+    rescaled the Llama 3.1 way.
+
+    With scaling = (factor, low, high, L): a pair whose wavelength 2 pi / f is
+    shorter than L / high keeps its rate; one longer than L / low turns factor
+    times slower; in between the rate blends the two, weighted by
+    (L / wavelength - low) / (high - low) towards the unscaled rate.
+    """
+    half = d // 2
+    inv_freq = theta ** (-2.0 * np.arange(half, dtype=np.float64) / d)
+    if scaling is None:
+        return inv_freq
+    factor, low, high, L = scaling
+    out = np.empty_like(inv_freq)
+    for m, f in enumerate(inv_freq):
+        wavelen = 2.0 * np.pi / f
+        if wavelen < L / high:
+            out[m] = f
+        elif wavelen > L / low:
+            out[m] = f / factor
+        else:
+            w = (L / wavelen - low) / (high - low)
+            out[m] = (1.0 - w) * f / factor + w * f
+    return out
+
+
+def rope(x, pos, theta, scaling=None):
     """Rotate-half rotary embedding of vectors x[..., d] at one position.
 
-    Dimension pairs (m, m + d/2) turn by the angle pos * theta^(-2m/d).
+    Dimension pairs (m, m + d/2) turn by the angle pos * inv_freq[m], with
+    inv_freq from rope_inv_freq (theta^(-2m/d) unless the model rescales it).
     """
     d = x.shape[-1]
     half = d // 2
-    inv_freq = theta ** (-2.0 * np.arange(half, dtype=np.float64) / d)
+    inv_freq = rope_inv_freq(d, theta, scaling)
     ang = float(pos) * inv_freq
     c, s = np.cos(ang), np.sin(ang)
     x1, x2 = x[..., :half], x[..., half:]
@@ -211,8 +254,8 @@ def verify_tree(m, cache_k, cache_v, ctx_len, tokens, parent, only=None):
         k = np.full((T, nkv, d), np.nan)
         v = np.full((T, nkv, d), np.nan)
         for r, i in enumerate(nodes):
-            q[i] = rope(q_s[r], ctx_len + depth[i], cfg.rope_theta)
-            k[i] = cache_format(rope(k_s[r], ctx_len + depth[i], cfg.rope_theta), cfg.dtype)
+            q[i] = rope(q_s[r], ctx_len + depth[i], cfg.rope_theta, rope_scaling(cfg))
+            k[i] = cache_format(rope(k_s[r], ctx_len + depth[i], cfg.rope_theta, rope_scaling(cfg)), cfg.dtype)
             v[i] = cache_format(v_s[r], cfg.dtype)
         tree_k.append(k)
         tree_v.append(v)
@@ -307,8 +350,8 @@ def decode_step(m, cache_k, cache_v, n_pos, token):
         W = m.layer(l)
         h = rms_norm(x, W["attn_norm"], cfg.rms_eps)
         q, k, v = qkv(W, cfg, h)
-        q = rope(q[0], n_pos, cfg.rope_theta)
-        k = cache_format(rope(k[0], n_pos, cfg.rope_theta), cfg.dtype)
+        q = rope(q[0], n_pos, cfg.rope_theta, rope_scaling(cfg))
+        k = cache_format(rope(k[0], n_pos, cfg.rope_theta, rope_scaling(cfg)), cfg.dtype)
         v = cache_format(v[0], cfg.dtype)
         ks.append(k)
         vs.append(v)

@@ -35,7 +35,9 @@ class OosModelConfig(ctypes.Structure):
     _fields_ = [("n_layers", c_i32), ("hidden", c_i32), ("n_q_heads", c_i32), ("n_kv_heads", c_i32),
                 ("head_dim", c_i32), ("intermediate", c_i32), ("vocab", c_i32), ("dtype", c_i32),
                 ("qk_norm", c_i32), ("qkv_bias", c_i32), ("rms_eps", ctypes.c_float),
-                ("rope_theta", ctypes.c_float), ("max_T", c_i32), ("use_graph", c_i32)]
+                ("rope_theta", ctypes.c_float), ("max_T", c_i32), ("use_graph", c_i32),
+                ("rope_factor", ctypes.c_float), ("rope_low_freq_factor", ctypes.c_float),
+                ("rope_high_freq_factor", ctypes.c_float), ("rope_orig_max_pos", c_i32)]
 
 
 LAYER_FIELDS = ("attn_norm", "w_q", "w_k", "w_v", "b_q", "b_k", "b_v", "q_norm", "k_norm", "w_o",
@@ -119,7 +121,10 @@ def make_config(cfg, max_T, use_graph=True):
                           cfg.intermediate, cfg.vocab,
                           OOS_DTYPE_BF16 if cfg.dtype == "bf16" else OOS_DTYPE_F32,
                           int(cfg.qk_norm), int(cfg.qkv_bias), cfg.rms_eps, cfg.rope_theta, max_T,
-                          int(use_graph))
+                          int(use_graph), float(getattr(cfg, "rope_factor", 0.0) or 0.0),
+                          float(getattr(cfg, "rope_low_freq_factor", 1.0)),
+                          float(getattr(cfg, "rope_high_freq_factor", 4.0)),
+                          int(getattr(cfg, "rope_orig_max_pos", 8192)))
 
 
 def oos_workspace_bytes(c_cfg):

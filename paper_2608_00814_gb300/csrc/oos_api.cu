@@ -7,6 +7,7 @@
 
 #include <algorithm>
 #include <new>
+#include <vector>
 
 #include "common.cuh"
 #include "internal.h"
@@ -91,6 +92,24 @@ size_t carve_workspace(const oos_model_config& c, int n_sms, uint8_t* base, Work
   return align_up(off, 256);
 }
 
+// Llama-3.1 rotary frequency rescaling of the pair rates theta^(-2m/d) (see
+// oos_model_config): pairs of short wavelength keep their rate, long ones turn
+// rope_factor times slower, the band between blends the two.
+static void rope_rescale(std::vector<double>& inv, const oos_model_config& c) {
+  const double F = c.rope_factor, lo = c.rope_low_freq_factor, hi = c.rope_high_freq_factor;
+  const double L = (double)c.rope_orig_max_pos;
+  for (double& f : inv) {
+    const double wavelen = 2.0 * M_PI / f;
+    if (wavelen < L / hi) continue;
+    if (wavelen > L / lo) {
+      f = f / F;
+    } else {
+      const double w = (L / wavelen - lo) / (hi - lo);
+      f = (1.0 - w) * f / F + w * f;
+    }
+  }
+}
+
 static bool config_ok(const oos_model_config* c) {
   if (!c) return false;
   if (c->n_layers < 1 || c->n_layers > kMaxLayers) return false;
@@ -100,6 +119,13 @@ static bool config_ok(const oos_model_config* c) {
   if (c->max_T < 1 || c->max_T > kMaxT) return false;
   if (c->dtype != OOS_DTYPE_F32 && c->dtype != OOS_DTYPE_BF16) return false;
   if (!(c->rms_eps >= 0.f) || !(c->rope_theta > 0.f)) return false;
+  if (c->rope_factor > 1.f) {
+    if (!(c->rope_low_freq_factor > 0.f) || !(c->rope_high_freq_factor > c->rope_low_freq_factor) ||
+        c->rope_orig_max_pos < 1)
+      return false;
+  } else if (!(c->rope_factor == c->rope_factor)) {   // NaN
+    return false;
+  }
   return true;
 }
 
@@ -290,6 +316,7 @@ int oos_model_create(const oos_model_config* cfg, const oos_weights* w, void* wo
     if (cudaMemset(workspace, 0, need) != cudaSuccess) { rc = OOS_ECUDA; break; }
     std::vector<double> inv(c.head_dim / 2);
     for (int j = 0; j < c.head_dim / 2; ++j) inv[j] = pow((double)c.rope_theta, -2.0 * j / (double)c.head_dim);
+    if (c.rope_factor > 1.f) rope_rescale(inv, c);
     if (cudaMemcpy(m->ws.inv_freq, inv.data(), inv.size() * 8, cudaMemcpyHostToDevice) != cudaSuccess) {
       rc = OOS_ECUDA;
       break;

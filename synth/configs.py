@@ -31,6 +31,11 @@ class ModelConfig:
     qkv_bias: bool        # Qwen2.5: bias on the q, k, v projections
     tied: bool            # LM head shares the embedding matrix
     init_std: float = 0.02
+    # Llama 3.1 rotary frequency rescaling (factor <= 1: none)
+    rope_factor: float = 0.0
+    rope_low_freq_factor: float = 1.0
+    rope_high_freq_factor: float = 4.0
+    rope_orig_max_pos: int = 8192
 
     @property
     def q_dim(self):
@@ -73,10 +78,23 @@ QWEN3_8B = ModelConfig("qwen3-8b", n_layers=36, hidden=4096, n_q_heads=32,
                        vocab=151936, rms_eps=1e-6, rope_theta=1e6,
                        dtype="bf16", qk_norm=True, qkv_bias=False, tied=False)
 
+# Qwen3 targets of the paper's scaling study (4B .. 32B with one frozen sidecar)
+QWEN3_4B = ModelConfig("qwen3-4b", n_layers=36, hidden=2560, n_q_heads=32,
+                       n_kv_heads=8, head_dim=128, intermediate=9728,
+                       vocab=151936, rms_eps=1e-6, rope_theta=1e6,
+                       dtype="bf16", qk_norm=True, qkv_bias=False, tied=True)
+
+QWEN3_14B = ModelConfig("qwen3-14b", n_layers=40, hidden=5120, n_q_heads=40,
+                        n_kv_heads=8, head_dim=128, intermediate=17408,
+                        vocab=151936, rms_eps=1e-6, rope_theta=1e6,
+                        dtype="bf16", qk_norm=True, qkv_bias=False, tied=False)
+
 LLAMA31_8B = ModelConfig("llama3.1-8b", n_layers=32, hidden=4096, n_q_heads=32,
                          n_kv_heads=8, head_dim=128, intermediate=14336,
                          vocab=128256, rms_eps=1e-5, rope_theta=5e5,
-                         dtype="bf16", qk_norm=False, qkv_bias=False, tied=False)
+                         dtype="bf16", qk_norm=False, qkv_bias=False, tied=False,
+                         rope_factor=8.0, rope_low_freq_factor=1.0, rope_high_freq_factor=4.0,
+                         rope_orig_max_pos=8192)
 
 QWEN25_32B = ModelConfig("qwen2.5-32b", n_layers=64, hidden=5120, n_q_heads=40,
                          n_kv_heads=8, head_dim=128, intermediate=27648,
@@ -94,6 +112,10 @@ WORKLOADS = {
                             tree=dict(kind="wide", level_branch=8, max_depth=16)),
     "qwen2.5-32b": Workload(QWEN25_32B, ctx_len=4096, T=64, plant=10,
                             tree=dict(kind="branch", bmin=1, bmax=4, max_depth=12)),
+    "qwen3-4b": Workload(QWEN3_4B, ctx_len=2048, T=64, plant=10,
+                         tree=dict(kind="branch", bmin=1, bmax=4, max_depth=12)),
+    "qwen3-14b": Workload(QWEN3_14B, ctx_len=2048, T=64, plant=10,
+                          tree=dict(kind="branch", bmin=1, bmax=4, max_depth=12)),
 }
 
 # A small bf16 decoder with the head_dim of the real targets: runs every

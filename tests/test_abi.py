@@ -5,6 +5,8 @@ import ctypes
 import os
 import re
 
+import pytest
+
 from paper_2608_00814_gb300 import _build
 from paper_2608_00814_gb300 import binding as B
 
@@ -48,3 +50,21 @@ def test_status_strings_and_config_rejection():
 def test_library_is_sm103a_only():
     flags = _build._flags()
     assert "arch=compute_103a,code=sm_103a" in " ".join(flags)
+
+
+@pytest.mark.gpu
+def test_rope_rescaling_config_validation():
+    """Llama-3.1 rotary rescaling fields: accepted with hi > lo > 0 and L >= 1,
+    rejected otherwise (workspace size 0).  Needs a device: the workspace size
+    depends on its SM count."""
+    _build.build()
+    L = B.lib()
+    good = B.OosModelConfig(2, 256, 4, 2, 64, 512, 1024, 0, 0, 0, 1e-6, 5e5, 8, 0, 8.0, 1.0, 4.0, 8192)
+    assert L.oos_workspace_bytes(ctypes.byref(good)) > 0
+    plain = B.OosModelConfig(2, 256, 4, 2, 64, 512, 1024, 0, 0, 0, 1e-6, 5e5, 8, 0, 0.0, 0.0, 0.0, 0)
+    assert L.oos_workspace_bytes(ctypes.byref(plain)) > 0      # factor 0: the other fields are ignored
+    for lo, hi, orig in ((4.0, 4.0, 8192), (0.0, 4.0, 8192), (1.0, 4.0, 0)):
+        bad = B.OosModelConfig(2, 256, 4, 2, 64, 512, 1024, 0, 0, 0, 1e-6, 5e5, 8, 0, 8.0, lo, hi, orig)
+        assert L.oos_workspace_bytes(ctypes.byref(bad)) == 0
+    bad = B.OosModelConfig(2, 256, 4, 2, 64, 512, 1024, 0, 0, 0, 1e-6, 5e5, 8, 0, float("nan"), 1.0, 4.0, 8192)
+    assert L.oos_workspace_bytes(ctypes.byref(bad)) == 0

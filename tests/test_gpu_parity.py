@@ -54,7 +54,10 @@ def test_tiny_parity_many_seeds(tiny_models):
 
 
 @pytest.mark.parametrize("overrides,gain_std", [(dict(qk_norm=True), 0.0), (dict(qkv_bias=True), 0.2),
-                                                (dict(qk_norm=True, qkv_bias=True, tied=True), 0.2)])
+                                                (dict(qk_norm=True, qkv_bias=True, tied=True), 0.2),
+                                                # Llama-3.1 rotary rescaling, short original context so
+                                                # that all three frequency regions occur
+                                                (dict(rope_factor=8.0, rope_orig_max_pos=64), 0.0)])
 def test_tiny_variants(tiny_models, overrides, gain_std):
     case, model = _tiny(tiny_models, 3, cfg_overrides=overrides, gain_std=gain_std)
     kv = gpu_cache(case, case.ctx_len + 128)
@@ -263,7 +266,8 @@ def test_mini_bf16_shapes(mini_models, T, recipe, ctx):
 
 
 @pytest.mark.parametrize("overrides,gain_std", [(dict(qk_norm=False, qkv_bias=True), 0.2),
-                                                (dict(tied=True), 0.1)])
+                                                (dict(tied=True), 0.1),
+                                                (dict(qk_norm=False, rope_factor=8.0, rope_orig_max_pos=256), 0.0)])
 def test_mini_bf16_variants(mini_models, overrides, gain_std):
     case, model = _mini(mini_models, 2, cfg_overrides=overrides, gain_std=gain_std)
     kv = gpu_cache(case, case.ctx_len + 16)
@@ -323,8 +327,16 @@ def test_bf16_qwen3_8b_bench_shape_sampled():
 
 
 def test_bf16_llama31_8b_wide_tree_sampled():
-    """T=128 wide tree over an 8192-position cache (RoPE theta 5e5, no q/k norm)."""
+    """T=128 wide tree over an 8192-position cache (RoPE theta 5e5 with the
+    Llama-3.1 frequency rescaling, no q/k norm)."""
     _sampled_check("llama3.1-8b")
+
+
+@pytest.mark.parametrize("name", ["qwen3-4b", "qwen3-14b"])
+def test_bf16_qwen3_scaling_targets_sampled(name):
+    """Qwen3 targets of the paper's scaling study: 4B (tied head, q width 4096
+    over hidden 2560) and 14B (40/8 heads, hidden 5120)."""
+    _sampled_check(name)
 
 
 def test_bf16_qwen25_32b_sampled():

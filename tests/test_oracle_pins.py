@@ -80,6 +80,60 @@ def test_rope_relative_position_and_norm():
     assert abs(np.linalg.norm(oracle.rope(q, 77, 5e5)) - np.linalg.norm(q)) < 1e-12
 
 
+LLAMA31_ROPE = (8.0, 1.0, 4.0, 8192.0)   # factor, low- and high-frequency factors, original context
+
+
+def test_rope_rescaling_regions_for_llama31_shape():
+    """Llama-3.1 rescaling at theta 5e5, d 128, split by hand.
+
+    Pair m has wavelength 2 pi 5e5^(m/64).  It stays below 8192/4 = 2048 while
+    m/64 < ln(2048 / 2 pi) / ln 5e5 = 0.4410, so m <= 28 keep their rate.  It
+    exceeds 8192/1 while m/64 > ln(8192 / 2 pi) / ln 5e5 = 0.5467, so m >= 35 turn
+    8 times slower.  m = 29..34 are blended.
+    """
+    base = oracle.rope_inv_freq(128, 5e5)
+    np.testing.assert_array_equal(base, 5e5 ** (-np.arange(64) / 64.0))
+    r = oracle.rope_inv_freq(128, 5e5, LLAMA31_ROPE) / base
+    np.testing.assert_array_equal(r[:29], 1.0)
+    np.testing.assert_allclose(r[35:], 1.0 / 8.0, rtol=1e-15)
+    mid = r[29:35]
+    assert np.all(mid < 1.0) and np.all(mid > 1.0 / 8.0)
+    # the blend moves monotonically from the kept rate to the slowed one
+    assert np.all(np.diff(r) <= 0.0)
+
+
+def test_rope_rescaling_blend_is_continuous_at_both_edges():
+    """A pair exactly on an edge of the blended band gets the rate of the region
+    beyond that edge (the blend weight is 1 at L/hi and 0 at L/lo)."""
+    L, lo, hi, F = 8192.0, 1.0, 4.0, 8.0
+    for wavelen, want in ((L / hi, 1.0), (L / lo, 1.0 / F)):
+        f = 2.0 * np.pi / wavelen
+        # theta such that pair m = 1 of d = 4 has rate f: theta^(-1/2) = f
+        theta = f ** -2.0
+        got = oracle.rope_inv_freq(4, theta, (F, lo, hi, L))[1] / f
+        assert abs(got - want) < 1e-12, (wavelen, got, want)
+
+
+def test_rope_rescaling_none_and_still_a_rotation():
+    rng = np.random.default_rng(5)
+    q, k = rng.normal(size=128), rng.normal(size=128)
+    for sc in (None, (1.0, 1.0, 4.0, 8192.0)):
+        # factor <= 1 through the config path means no rescaling at all
+        cfg = type("C", (), dict(rope_factor=sc[0] if sc else 0.0, rope_low_freq_factor=1.0,
+                                 rope_high_freq_factor=4.0, rope_orig_max_pos=8192))()
+        assert oracle.rope_scaling(cfg) is None
+    a = oracle.rope(q, 40, 5e5, LLAMA31_ROPE) @ oracle.rope(k, 33, 5e5, LLAMA31_ROPE)
+    b = oracle.rope(q, 9040, 5e5, LLAMA31_ROPE) @ oracle.rope(k, 9033, 5e5, LLAMA31_ROPE)
+    assert abs(a - b) < 1e-9
+    assert abs(np.linalg.norm(oracle.rope(q, 8300, 5e5, LLAMA31_ROPE)) - np.linalg.norm(q)) < 1e-12
+    # the slowest pairs turn 8 times less far than without rescaling
+    x = np.zeros(128)
+    x[63] = 1.0
+    ang_scaled = np.arctan2(oracle.rope(x, 1000, 5e5, LLAMA31_ROPE)[127], oracle.rope(x, 1000, 5e5, LLAMA31_ROPE)[63])
+    ang_plain = np.arctan2(oracle.rope(x, 1000, 5e5)[127], oracle.rope(x, 1000, 5e5)[63])
+    assert abs(ang_scaled * 8.0 - ang_plain) < 1e-12
+
+
 def test_attend_matches_sdpa():
     rng = np.random.default_rng(4)
     q = rng.normal(size=64)
