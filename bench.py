@@ -339,6 +339,32 @@ def run_ours(args):
     k_gbs = k_bytes / (k_ms * 1e-3) / 1e9
     traffic = traffic_for("gemm_gate_up_%s_T%d" % (args.workload, T), GEMM_SRC)
 
+    # ---- target prefill: a ctx_len-token synthetic prompt (seeded) into slots [0, ctx) of the
+    # cache, run as 128-token chains through the verify kernels (after every verify
+    # measurement: it overwrites the synthetic cache they read)
+    prefill = None
+    if not args.no_prefill:
+        pf_model = B.OosModel(cfg, weights, max_T=128, use_graph=False)
+        prompt = np.random.default_rng(seed).integers(0, cfg.vocab, size=ctx).astype(np.int32)
+        p_tok = torch.as_tensor(prompt, device="cuda")
+        nxt = torch.zeros(1, dtype=torch.int32, device="cuda")
+        B.oos_prefill(pf_model, kv, 0, p_tok, ctx, nxt, stream)   # warm
+        torch.cuda.synchronize()
+        if B.oos_last_status(pf_model) != B.OOS_OK:
+            raise RuntimeError("prefill status %s" % B.oos_status_string(B.oos_last_status(pf_model)))
+        reps = 2
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            B.oos_prefill(pf_model, kv, 0, p_tok, ctx, nxt, stream)
+        b.record(stream)
+        torch.cuda.synchronize()
+        pf_ms = a.elapsed_time(b) / reps
+        prefill = {"tokens": ctx, "ms": pf_ms, "tokens_per_s": ctx / (pf_ms * 1e-3), "chain": 128,
+                   "note": "prompt as causal chains of 128 tokens through the verify kernels; "
+                           "every chain streams the weights once"}
+        pf_model.close()
+
     # ---- CPU checker on the host cores (rank 0, N = 1 only)
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
@@ -372,6 +398,7 @@ def run_ours(args):
             "e2e": {"value": world * T / e2e_s, "unit": UNIT, "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
             "gpu_launches": launches_per_step * args.steps,
             "clocks": clk,
+            "prefill": prefill,
         }), flush=True)
     model.close()
     if world > 1:
@@ -387,6 +414,7 @@ def main():
                                                                       if w.model.dtype == "bf16"))
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-prefill", action="store_true", help="skip the prefill measurement")
     ap.add_argument("--layers", type=int, default=0,
                     help="profiling captures only: keep the first N layers of the workload's model")
     args = ap.parse_args()

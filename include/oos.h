@@ -162,6 +162,23 @@ int oos_model_create(const oos_model_config* cfg, const oos_weights* w, void* wo
 
 int oos_model_destroy(oos_model* m);
 
+/* Target prefill: the step before tree verification, which fills the cache
+ * with a prompt (the paper's targets start decoding from a prefilled request).
+ *   kv            cache; slots [0, ctx_len) are read, slots [ctx_len,
+ *                 ctx_len + n) receive the prompt's K/V.
+ *   tokens        DEVICE int32[n], the prompt after the ctx_len cached positions.
+ *   n             >= 1; any length that fits the cache: it runs as chains of at
+ *                 most max_T tokens, each a tree pass of the verify kernels (a
+ *                 chain's tree attention is causal attention).
+ *   out_next_token  DEVICE int32[1] or NULL: the greedy next token after the
+ *                 prompt (argmax of the last position's logits, Eq. 1).
+ * Stream-ordered, no host synchronisation.  Returns OOS_EINVAL on NULL handle,
+ * cache or tokens, n < 1 or ctx_len < 0; OOS_ECAPACITY when ctx_len + n exceeds
+ * the cache; a token outside [0, vocab) is reported by oos_last_status
+ * (OOS_ETREE), as for a tree. */
+int oos_prefill(oos_model* m, const oos_kv_cache* kv, int32_t ctx_len, const int32_t* tokens, int32_t n,
+                int32_t* out_next_token, void* stream);
+
 /* One verification step (Eq. 1; "Verify and commit").
  *   kv            committed cache; slots [0, ctx_len) are read, slots
  *                 [ctx_len, ctx_len+T) are overwritten with the tree's K/V.

@@ -77,6 +77,7 @@ def lib():
         L.oos_tree_verify_debug.argtypes = [c_vp, P(OosKvCache), c_i32, c_vp, c_vp, c_i32, c_vp, c_vp, c_vp, c_vp,
                                             c_vp, c_vp, c_vp, c_vp, c_vp]
         L.oos_kv_compact.argtypes = [c_vp, P(OosKvCache), c_i32, c_vp, c_vp, c_i32, c_vp]
+        L.oos_prefill.argtypes = [c_vp, P(OosKvCache), c_i32, c_vp, c_i32, c_vp, c_vp]
         L.oos_accept_walk.argtypes = [c_vp, c_vp, c_vp, c_i32, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp]
         L.oos_last_status.argtypes = [c_vp, c_vp]
         L.oos_launch_stage.argtypes = [c_vp, c_i32, c_i32, c_i32, c_vp]
@@ -88,7 +89,7 @@ def lib():
         L.oos_status_string.argtypes = [ctypes.c_int]
         L.oos_status_string.restype = ctypes.c_char_p
         for fn in ("oos_model_create", "oos_model_destroy", "oos_tree_verify", "oos_tree_verify_debug",
-                   "oos_kv_compact", "oos_accept_walk", "oos_last_status"):
+                   "oos_kv_compact", "oos_accept_walk", "oos_last_status", "oos_prefill"):
             getattr(L, fn).restype = ctypes.c_int
         _lib = L
     return _lib
@@ -210,6 +211,11 @@ def oos_tree_verify_debug(model, kv, ctx_len, tree_tokens, tree_parent, T, out_a
                                        _ptr(out_accepted_tokens), _ptr(out_bonus_token), _ptr(out_final_hidden),
                                        _ptr(out_argmax), _ptr(out_top1), _ptr(out_top2), _stream(stream)),
            "oos_tree_verify_debug")
+
+
+def oos_prefill(model, kv, ctx_len, tokens, n, out_next_token=None, stream=None):
+    _check(lib().oos_prefill(model.handle, ctypes.byref(kv.c), ctx_len, _ptr(tokens), n, _ptr(out_next_token),
+                             _stream(stream)), "oos_prefill")
 
 
 def oos_kv_compact(model, kv, ctx_len, accepted_nodes, accepted_len, max_len, stream=None):

@@ -90,6 +90,8 @@ struct Workspace {
   float* ss;                 // sum of x^2 per 128-feature chunk [kMaxSsChunks][kMaxT] (bf16 path)
   float2* rope;              // (cos, sin) per node and rotary pair [kMaxT][d/2] (bf16 path)
   int* cnt;                  // GEMM arrival counters [layer][4 kinds][kCntPer], zeroed at every step start
+  int32_t* chain_parent;     // [kMaxT]: -1, 0, 1, ... (the chains a prefill runs as trees)
+  int32_t* pf_scratch;       // prefill's unused accept outputs: len, bonus, nodes[kMaxT], tokens[kMaxT]
 };
 
 // shape + addresses a captured verify graph was recorded with

@@ -88,6 +88,8 @@ size_t carve_workspace(const oos_model_config& c, int n_sms, uint8_t* base, Work
   w.ss = (float*)take((size_t)kMaxSsChunks * kMaxT * 4);
   w.rope = (float2*)take((size_t)kMaxT * (c.head_dim / 2) * 8);
   w.cnt = (int*)take((size_t)c.n_layers * 4 * kCntPer * 4);
+  w.chain_parent = (int32_t*)take(kMaxT * 4);
+  w.pf_scratch = (int32_t*)take((2 + 2 * kMaxT) * 4);
   if (ws) *ws = w;
   return align_up(off, 256);
 }
@@ -164,10 +166,10 @@ static unsigned long long kv_hash(const oos_kv_cache* kv) {
     if ((x) != cudaSuccess) return OOS_ECUDA; \
   } while (0)
 
-// the whole verify step on stream st
-static int enqueue_verify(Model& m, const oos_kv_cache* kv, int ctx, const int32_t* tokens, const int32_t* parent,
-                          int T, int32_t* len, int32_t* nodes, int32_t* toks, int32_t* bonus, float* hidden,
-                          int32_t* dbg_arg, float* dbg_t1, float* dbg_t2, cudaStream_t st) {
+// tree prep, embedding and every decoder layer of a tree on stream st: the
+// K/V of the T nodes land in slots ctx.., the final-norm input in ws.x
+static int enqueue_layers(Model& m, const oos_kv_cache* kv, int ctx, const int32_t* tokens, const int32_t* parent,
+                          int T, float* hidden, cudaStream_t st) {
   const auto& c = m.cfg;
   const int L = c.n_layers;
   const int qd = c.n_q_heads * c.head_dim, kvd = c.n_kv_heads * c.head_dim;
@@ -199,6 +201,16 @@ static int enqueue_verify(Model& m, const oos_kv_cache* kv, int ctx, const int32
       OOS_TRY(launch_resid_norm(m, m.p_down, next_gain, hid, T, st));
     }
   }
+  return OOS_OK;
+}
+
+// the whole verify step on stream st
+static int enqueue_verify(Model& m, const oos_kv_cache* kv, int ctx, const int32_t* tokens, const int32_t* parent,
+                          int T, int32_t* len, int32_t* nodes, int32_t* toks, int32_t* bonus, float* hidden,
+                          int32_t* dbg_arg, float* dbg_t1, float* dbg_t2, cudaStream_t st) {
+  const auto& c = m.cfg;
+  const int rc = enqueue_layers(m, kv, ctx, tokens, parent, T, hidden, st);
+  if (rc != OOS_OK) return rc;
   if (c.dtype == OOS_DTYPE_BF16) {
     if (hidden) OOS_TRY(launch_final_hidden(m, hidden, T, st));
     OOS_TRY(launch_lm_head_tc(m, T, st));
@@ -206,6 +218,29 @@ static int enqueue_verify(Model& m, const oos_kv_cache* kv, int ctx, const int32
     OOS_TRY(launch_lm_head_f32(m, T, st));
   }
   OOS_TRY(launch_argmax_accept(m, tokens, parent, T, m.lm_grid, len, nodes, toks, bonus, dbg_arg, dbg_t1, dbg_t2, st));
+  return OOS_OK;
+}
+
+// Prefill: the prompt as chains of at most max_T tokens.  In a chain node j's
+// ancestors are nodes 0..j and its depth is j, so each chunk's tree pass is
+// causal decoding of the chunk after everything before it, and node j's K/V
+// land in their final slot ctx + off + j (no compaction).  Only the last chunk
+// runs the LM head: the argmax of its last node is the greedy next token.
+static int prefill_impl(Model& m, const oos_kv_cache* kv, int ctx, const int32_t* tokens, int n, int32_t* next_token,
+                        cudaStream_t st) {
+  const auto& c = m.cfg;
+  int32_t* sc = m.ws.pf_scratch;
+  for (int off = 0; off < n; off += c.max_T) {
+    const int T = std::min(c.max_T, n - off);
+    const int rc = enqueue_layers(m, kv, ctx + off, tokens + off, m.ws.chain_parent, T, nullptr, st);
+    if (rc != OOS_OK) return rc;
+    if (off + T < n) continue;
+    if (c.dtype == OOS_DTYPE_BF16) OOS_TRY(launch_lm_head_tc(m, T, st));
+    else OOS_TRY(launch_lm_head_f32(m, T, st));
+    OOS_TRY(launch_argmax_accept(m, tokens + off, m.ws.chain_parent, T, m.lm_grid, sc, sc + 2, sc + 2 + kMaxT,
+                                 sc + 1, nullptr, nullptr, nullptr, st));
+    if (next_token) OOS_TRY(cudaMemcpyAsync(next_token, m.ws.argmax + (T - 1), 4, cudaMemcpyDeviceToDevice, st));
+  }
   return OOS_OK;
 }
 
@@ -321,6 +356,12 @@ int oos_model_create(const oos_model_config* cfg, const oos_weights* w, void* wo
       rc = OOS_ECUDA;
       break;
     }
+    std::vector<int32_t> chain(kMaxT);
+    for (int i = 0; i < kMaxT; ++i) chain[i] = i - 1;
+    if (cudaMemcpy(m->ws.chain_parent, chain.data(), kMaxT * 4, cudaMemcpyHostToDevice) != cudaSuccess) {
+      rc = OOS_ECUDA;
+      break;
+    }
     if (gemm_setup() != cudaSuccess || attn_setup() != cudaSuccess || compact_setup() != cudaSuccess) {
       rc = OOS_ECUDA;
       break;
@@ -415,6 +456,16 @@ int oos_tree_verify(oos_model* m, const oos_kv_cache* kv, int32_t ctx_len, const
                     int32_t* out_accepted_tokens, int32_t* out_bonus_token, void* stream) {
   return verify_impl(m, kv, ctx_len, tree_tokens, tree_parent, T, out_accepted_len, out_accepted_nodes,
                      out_accepted_tokens, out_bonus_token, nullptr, nullptr, nullptr, nullptr, stream);
+}
+
+int oos_prefill(oos_model* m, const oos_kv_cache* kv, int32_t ctx_len, const int32_t* tokens, int32_t n,
+                int32_t* out_next_token, void* stream) {
+  if (!m || !kv || !tokens || n < 1 || ctx_len < 0) return OOS_EINVAL;
+  if (kv->n_layers != m->cfg.n_layers || !kv->k || !kv->v || kv->capacity < 1) return OOS_EINVAL;
+  for (int l = 0; l < kv->n_layers; ++l)
+    if (!kv->k[l] || !kv->v[l]) return OOS_EINVAL;
+  if ((long long)ctx_len + n > kv->capacity) return OOS_ECAPACITY;
+  return prefill_impl(*m, kv, ctx_len, tokens, n, out_next_token, (cudaStream_t)stream);
 }
 
 int oos_tree_verify_debug(oos_model* m, const oos_kv_cache* kv, int32_t ctx_len, const int32_t* tree_tokens,

@@ -9,7 +9,8 @@ import torch
 
 import oracle
 from cases import GOLDEN, build_case, load_planted
-from gpu_util import GATE, check_case, check_compaction, gpu_cache, gpu_model, ok_nodes, run
+from gpu_util import (GATE, TOL, check_case, check_compaction, gpu_cache, gpu_model, max_rel_err, ok_nodes, run,
+                      to_f64)
 from synth import trees
 
 pytestmark = pytest.mark.gpu
@@ -342,3 +343,39 @@ def test_bf16_qwen3_scaling_targets_sampled(name):
 def test_bf16_qwen25_32b_sampled():
     """64 layers, 40/8 heads, q/k/v bias: about 64 GB of bf16 weights on one GPU."""
     _sampled_check("qwen2.5-32b")
+
+
+@pytest.mark.parametrize("name,ctx,n", [
+    ("tiny", 0, 300),          # empty cache, three chains of at most 128 tokens (the last one ragged)
+    ("tiny", 128, 129),        # after a cached prefix; one full chain and a one-token chain
+    ("mini-bf16", 200, 290),   # bf16 tensor-core path
+    ("mini-bf16", 0, 1),       # one-token prompt
+])
+def test_prefill_matches_causal_decoding(tiny_models, mini_models, name, ctx, n):
+    """oos_prefill == causal decoding of the prompt after ctx cached positions:
+    every layer's K/V of the prompt positions, and the greedy next token (when
+    its margin clears the gate)."""
+    if name == "tiny":
+        case, model = _tiny(tiny_models, 4, ctx_len=ctx)
+    else:
+        case, model = _mini(mini_models, 4, ctx_len=ctx)
+    cfg = case.cfg
+    prompt = np.random.default_rng(11 + n).integers(0, cfg.vocab, size=n)
+    kv = gpu_cache(case, ctx + n + 8)
+    tok = torch.as_tensor(prompt.astype(np.int32), device="cuda")
+    nxt = torch.full((1,), -1, dtype=torch.int32, device="cuda")
+    B.oos_prefill(model, kv, ctx, tok, n, nxt)
+    torch.cuda.synchronize()
+    assert B.oos_last_status(model) == B.OOS_OK
+    steps, ck, cv = oracle.decode_sequence(case.view, case.cache_k64, case.cache_v64, ctx, prompt.tolist())
+    tol = TOL[cfg.dtype]
+    for l in range(cfg.n_layers):
+        ek = max_rel_err(to_f64(cfg, kv.k[l][ctx:ctx + n]), ck[l][ctx:ctx + n])
+        ev = max_rel_err(to_f64(cfg, kv.v[l][ctx:ctx + n]), cv[l][ctx:ctx + n])
+        assert ek <= tol and ev <= tol, "layer %d prompt K/V error %.3g/%.3g" % (l, ek, ev)
+    last = steps[-1]
+    if last["top1"] - last["top2"] > GATE[cfg.dtype]:
+        assert int(nxt.item()) == int(last["argmax"])
+    # the cached prefix is left as it was
+    if ctx:
+        np.testing.assert_array_equal(to_f64(cfg, kv.k[0][:ctx]), to_f64(cfg, gpu_cache(case, ctx).k[0][:ctx]))
