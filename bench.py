@@ -365,6 +365,47 @@ def run_ours(args):
                            "every chain streams the weights once"}
         pf_model.close()
 
+    # ---- hint-bank candidate step (suffix match + tree packing): a 64M-token bank (256 MB,
+    # larger than L2) with a 7-token key planted at three places, and a 50k-token bank
+    hint = None
+    if not args.no_hint:
+        g = torch.Generator(device="cuda")
+        g.manual_seed(seed)
+        eos = 2
+        key = torch.randint(3, cfg.vocab, (7,), dtype=torch.int32, device="cuda", generator=g)
+        prefix = torch.cat([torch.randint(3, cfg.vocab, (30,), dtype=torch.int32, device="cuda", generator=g), key])
+        tok_o = torch.zeros(T, dtype=torch.int32, device="cuda")
+        par_o = torch.zeros(T, dtype=torch.int32, device="cuda")
+        T_o = torch.zeros(1, dtype=torch.int32, device="cuda")
+        info = torch.zeros(3, dtype=torch.int32, device="cuda")
+        res = {}
+        for label, nb in (("large", 64 << 20), ("request", 50_000)):
+            bank = torch.randint(3, cfg.vocab, (nb,), dtype=torch.int32, device="cuda", generator=g)
+            for f in (0.1, 0.5, 0.9):
+                at = int(f * (nb - 20))
+                bank[at:at + 7] = key
+                bank[at + 7:at + 9] = torch.tensor([11 + at % 7, 12], dtype=torch.int32, device="cuda")
+            ws = torch.empty(B.oos_hint_workspace_bytes(nb), dtype=torch.uint8, device="cuda")
+            run_h = lambda: B.oos_hint_tree(bank, eos, prefix, None, None, 8, 16, T, ws, tok_o, par_o, T_o, info,
+                                            stream)
+            run_h()
+            torch.cuda.synchronize()
+            reps = 5
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            for _ in range(reps):
+                run_h()
+            b.record(stream)
+            torch.cuda.synchronize()
+            us = a.elapsed_time(b) / reps * 1e3
+            res[label] = (nb, us, info.cpu().tolist(), int(T_o.item()))
+        nb, us, inf, tn = res["large"]
+        h_bytes = 5 * nb   # bank tokens read, one match byte written per position
+        hint = {"bank_tokens": nb, "us": us, "gbs": h_bytes / (us * 1e-6) / 1e9,
+                "frac_of_measured_hbm": h_bytes / (us * 1e-6) / 1e9 / peak, "match_n": inf[0], "hint_lanes": inf[1],
+                "tree_nodes": tn, "request_bank_tokens": res["request"][0], "request_us": res["request"][1]}
+        del bank, ws
+
     # ---- CPU checker on the host cores (rank 0, N = 1 only)
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
@@ -399,6 +440,7 @@ def run_ours(args):
             "gpu_launches": launches_per_step * args.steps,
             "clocks": clk,
             "prefill": prefill,
+            "hint": hint,
         }), flush=True)
     model.close()
     if world > 1:
@@ -415,6 +457,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-prefill", action="store_true", help="skip the prefill measurement")
+    ap.add_argument("--no-hint", action="store_true", help="skip the hint-bank step measurement")
     ap.add_argument("--layers", type=int, default=0,
                     help="profiling captures only: keep the first N layers of the workload's model")
     args = ap.parse_args()

@@ -162,6 +162,32 @@ int oos_model_create(const oos_model_config* cfg, const oos_weights* w, void* wo
 
 int oos_model_destroy(oos_model* m);
 
+/* Hint-bank candidate step: the next verification tree (Section 4, "Suffix
+ * matching" and "Candidate boundary"; the tree is Merge_B of the hint lanes and
+ * the verifier's native lanes).
+ *   bank          DEVICE int32[bank_len]: the tokenised views joined by eos.
+ *   prefix        DEVICE int32[prefix_len] (>= 1): the committed prefix y; its
+ *                 last token is the tree's root, its last 7 tokens are matched.
+ *   For n = min(7, prefix_len) down to 1, the length-n suffix of y is searched
+ *   in the bank; an occurrence counts only when a non-eos token follows it, and
+ *   the longest n with a counted occurrence is used.  Each of its occurrences,
+ *   in bank order, proposes a lane: up to `depth` tokens after it, cut before
+ *   an eos.  The native lanes follow: DEVICE int32[n_native][native_stride]
+ *   with lengths native_len[n_native] (cut to depth), NULL when n_native == 0.
+ *   Lanes are merged into a prefix tree rooted at y's last token, a node
+ *   numbered when created (parents first); a lane counts towards max_lanes only
+ *   when it creates a node; at most max_nodes nodes (1..128), depth 1..128.
+ *   workspace     DEVICE, >= oos_hint_workspace_bytes(bank_len), 256-byte aligned.
+ * Outputs (DEVICE): out_tokens / out_parent int32[max_nodes] (entries [0, T)
+ * written), out_T int32[1], out_info int32[3] = (matched n, 0 when none; hint
+ * lanes used; all lanes used).  Stream-ordered.  Returns OOS_EINVAL on a NULL
+ * or out-of-range argument, OOS_EWORKSPACE on a small or misaligned workspace. */
+size_t oos_hint_workspace_bytes(int32_t bank_len);
+int oos_hint_tree(const int32_t* bank, int32_t bank_len, int32_t eos, const int32_t* prefix, int32_t prefix_len,
+                  const int32_t* native, const int32_t* native_len, int32_t n_native, int32_t native_stride,
+                  int32_t max_lanes, int32_t depth, int32_t max_nodes, void* workspace, size_t ws_bytes,
+                  int32_t* out_tokens, int32_t* out_parent, int32_t* out_T, int32_t* out_info, void* stream);
+
 /* Target prefill: the step before tree verification, which fills the cache
  * with a prompt (the paper's targets start decoding from a prefilled request).
  *   kv            cache; slots [0, ctx_len) are read, slots [ctx_len,

@@ -78,6 +78,11 @@ def lib():
                                             c_vp, c_vp, c_vp, c_vp, c_vp]
         L.oos_kv_compact.argtypes = [c_vp, P(OosKvCache), c_i32, c_vp, c_vp, c_i32, c_vp]
         L.oos_prefill.argtypes = [c_vp, P(OosKvCache), c_i32, c_vp, c_i32, c_vp, c_vp]
+        L.oos_hint_workspace_bytes.argtypes = [c_i32]
+        L.oos_hint_workspace_bytes.restype = ctypes.c_size_t
+        L.oos_hint_tree.argtypes = [c_vp, c_i32, c_i32, c_vp, c_i32, c_vp, c_vp, c_i32, c_i32, c_i32, c_i32, c_i32,
+                                    c_vp, ctypes.c_size_t, c_vp, c_vp, c_vp, c_vp, c_vp]
+        L.oos_hint_tree.restype = ctypes.c_int
         L.oos_accept_walk.argtypes = [c_vp, c_vp, c_vp, c_i32, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp]
         L.oos_last_status.argtypes = [c_vp, c_vp]
         L.oos_launch_stage.argtypes = [c_vp, c_i32, c_i32, c_i32, c_vp]
@@ -211,6 +216,21 @@ def oos_tree_verify_debug(model, kv, ctx_len, tree_tokens, tree_parent, T, out_a
                                        _ptr(out_accepted_tokens), _ptr(out_bonus_token), _ptr(out_final_hidden),
                                        _ptr(out_argmax), _ptr(out_top1), _ptr(out_top2), _stream(stream)),
            "oos_tree_verify_debug")
+
+
+def oos_hint_workspace_bytes(bank_len):
+    return int(lib().oos_hint_workspace_bytes(bank_len))
+
+
+def oos_hint_tree(bank, eos, prefix, native, native_len, max_lanes, depth, max_nodes, workspace, out_tokens,
+                  out_parent, out_T, out_info, stream=None):
+    """native: int32 [n_native, stride] device tensor (or None), native_len: int32 [n_native]."""
+    n_native = 0 if native is None else int(native.shape[0])
+    stride = 1 if native is None else int(native.shape[1])
+    _check(lib().oos_hint_tree(_ptr(bank), int(bank.numel()), eos, _ptr(prefix), int(prefix.numel()), _ptr(native),
+                               _ptr(native_len), n_native, stride, max_lanes, depth, max_nodes, _ptr(workspace),
+                               workspace.numel() * workspace.element_size(), _ptr(out_tokens), _ptr(out_parent),
+                               _ptr(out_T), _ptr(out_info), _stream(stream)), "oos_hint_tree")
 
 
 def oos_prefill(model, kv, ctx_len, tokens, n, out_next_token=None, stream=None):

@@ -1,0 +1,273 @@
+// Hint-bank candidate step: the next verification tree from the request's
+// hint bank (Section 4, "Suffix matching" and "Candidate boundary").
+//
+// The committed prefix y is matched against the bank (tokenised views joined
+// by EOS): for n = 7 down to 1 the length-n suffix of y is searched, and the
+// tokens after each occurrence become candidate lanes, ahead of the native
+// lanes, under a lane budget; the lanes are packed into a prefix tree rooted
+// at y's last token.  An occurrence counts only when a non-EOS token follows
+// it; the longest n with any counted occurrence is used; lanes are taken in
+// bank order, cut at the lane depth or before an EOS; a lane counts towards
+// the budget only when it creates a node.
+//
+// k_hint_match: one thread per bank position (a block per 256-position chunk,
+// grid-stride over chunks) computes the longest n whose suffix ends there, 0
+// when nothing follows, as one byte; each chunk's maximum is kept too, and the
+// block maxima give the n of the call.  k_hint_pack: one block walks the chunk
+// maxima in bank order, 256 chunks per round, and visits only chunks that hold
+// an occurrence; in a visited chunk the positions' bytes, gathered in order by
+// warp ballots, give the occurrences, and warp 0 inserts each lane into the
+// tree held in shared memory: a lane token looks for an existing child with
+// one ballot over the nodes.
+#include <stdint.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace oos {
+
+constexpr int kHintMaxN = 7;        // longest suffix tried
+constexpr int kHintThreads = 256;   // threads of both kernels
+
+__global__ void __launch_bounds__(kHintThreads) k_hint_match(const int32_t* __restrict__ bank, int N, int eos,
+                                                             const int32_t* __restrict__ prefix, int prefix_len,
+                                                             uint8_t* __restrict__ mlen, uint8_t* __restrict__ cmax,
+                                                             int* __restrict__ best) {
+  __shared__ int suf[kHintMaxN];
+  __shared__ int wmax[kHintThreads / 32];
+  const int nmax = prefix_len < kHintMaxN ? prefix_len : kHintMaxN;
+  // suf[nmax - 1] is y's last token, suf[nmax - 1 - j] the one j before it
+  if (threadIdx.x < nmax) suf[threadIdx.x] = prefix[prefix_len - nmax + threadIdx.x];
+  __syncthreads();
+  const long long n_chunks = ((long long)N + kHintThreads - 1) / kHintThreads;
+  int bmax = 0;   // thread 0: this block's maximum
+  for (long long c = blockIdx.x; c < n_chunks; c += gridDim.x) {
+    const long long p = c * kHintThreads + threadIdx.x;
+    int m = 0;
+    // the next bank token must exist and not be EOS
+    if (p + 1 < N && bank[p + 1] != eos) {
+      while (m < nmax && p - m >= 0 && bank[p - m] == suf[nmax - 1 - m]) ++m;
+    }
+    if (p < N) mlen[p] = (uint8_t)m;
+    int cm = m;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) cm = max(cm, __shfl_xor_sync(0xffffffffu, cm, o));
+    if ((threadIdx.x & 31) == 0) wmax[threadIdx.x >> 5] = cm;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+      int b = 0;
+      for (int w = 0; w < kHintThreads / 32; ++w) b = max(b, wmax[w]);
+      cmax[c] = (uint8_t)b;
+      bmax = max(bmax, b);
+    }
+    __syncthreads();
+  }
+  if (threadIdx.x == 0 && bmax > 0) atomicMax(best, bmax);
+}
+
+// Insert one lane into the tree (warp 0, all lanes of the warp together).
+// Returns whether a node was created.  The caller stops when the lane or
+// node budget is spent.
+OOS_DEV bool hint_insert(int32_t* s_tok, int32_t* s_par, int& T, int max_nodes, const int32_t* lane, int len) {
+  const int lane_id = threadIdx.x & 31;
+  int cur = 0;
+  bool created = false;
+  for (int j = 0; j < len; ++j) {
+    const int t = lane[j];
+    // the child of cur with token t, if any (nodes are distinct per (parent, token))
+    int found = -1;
+    for (int base = 1; base < T && found < 0; base += 32) {
+      const int i = base + lane_id;
+      const unsigned hit = __ballot_sync(0xffffffffu, i < T && s_par[i] == cur && s_tok[i] == t);
+      if (hit) found = base + __ffs(hit) - 1;
+    }
+    if (found >= 0) {
+      cur = found;
+      continue;
+    }
+    if (T >= max_nodes) break;
+    if (lane_id == 0) {
+      s_tok[T] = t;
+      s_par[T] = cur;
+    }
+    __syncwarp();
+    cur = T;
+    ++T;
+    created = true;
+  }
+  return created;
+}
+
+__global__ void __launch_bounds__(kHintThreads) k_hint_pack(const int32_t* __restrict__ bank, int N, int eos,
+                                                            const int32_t* __restrict__ prefix, int prefix_len,
+                                                            const uint8_t* __restrict__ mlen,
+                                                            const uint8_t* __restrict__ cmax,
+                                                            const int* __restrict__ best,
+                                                            const int32_t* __restrict__ native,
+                                                            const int32_t* __restrict__ native_len, int n_native,
+                                                            int native_stride, int max_lanes, int depth,
+                                                            int max_nodes, int32_t* out_tok, int32_t* out_par,
+                                                            int32_t* out_T, int32_t* out_info) {
+  __shared__ int32_t s_tok[kMaxT], s_par[kMaxT];
+  __shared__ int32_t s_pos[kHintThreads];     // occurrences in the chunk being visited, in bank order
+  __shared__ int32_t s_chunk[kHintThreads];   // this round's chunks holding an occurrence, in order
+  __shared__ int32_t s_lane[kMaxT];           // the lane being inserted
+  __shared__ int s_wcnt[kHintThreads / 32];
+  __shared__ int s_n, s_nc, s_done;
+  const int warp = threadIdx.x >> 5, lane_id = threadIdx.x & 31;
+  const int n = *best;
+  int T = 1, lanes = 0, hint_lanes = 0;       // warp 0's copies are the authoritative ones
+  if (threadIdx.x == 0) {
+    s_tok[0] = prefix[prefix_len - 1];
+    s_par[0] = -1;
+    s_done = (max_lanes <= 0 || max_nodes <= 1) ? 1 : 0;
+  }
+  __syncthreads();
+  // hint lanes: occurrences of the length-n suffix (match length >= n), bank order
+  const long long n_chunks = ((long long)N + kHintThreads - 1) / kHintThreads;
+  for (long long cb = 0; n > 0 && cb < n_chunks; cb += kHintThreads) {
+    if (s_done) break;
+    // the chunks of this round that hold an occurrence, in order
+    {
+      const long long c = cb + threadIdx.x;
+      const bool has = c < n_chunks && cmax[c] >= n;
+      const unsigned bal = __ballot_sync(0xffffffffu, has);
+      if (lane_id == 0) s_wcnt[warp] = __popc(bal);
+      __syncthreads();
+      if (has) {
+        int off = __popc(bal & ((1u << lane_id) - 1u));
+        for (int w = 0; w < warp; ++w) off += s_wcnt[w];
+        s_chunk[off] = (int32_t)c;
+      }
+      if (threadIdx.x == 0) {
+        int k = 0;
+        for (int w = 0; w < kHintThreads / 32; ++w) k += s_wcnt[w];
+        s_nc = k;
+      }
+      __syncthreads();
+    }
+    // visit them: the chunk's occurrences in order, then warp 0 inserts their lanes
+    for (int ci = 0; ci < s_nc; ++ci) {
+      if (s_done) break;
+      const long long p = (long long)s_chunk[ci] * kHintThreads + threadIdx.x;
+      const bool m = p < N && mlen[p] >= n;
+      const unsigned bal = __ballot_sync(0xffffffffu, m);
+      if (lane_id == 0) s_wcnt[warp] = __popc(bal);
+      __syncthreads();
+      if (m) {
+        int off = __popc(bal & ((1u << lane_id) - 1u));
+        for (int w = 0; w < warp; ++w) off += s_wcnt[w];
+        s_pos[off] = (int32_t)p;
+      }
+      if (threadIdx.x == 0) {
+        int c = 0;
+        for (int w = 0; w < kHintThreads / 32; ++w) c += s_wcnt[w];
+        s_n = c;
+      }
+      __syncthreads();
+      if (warp == 0) {
+        for (int k = 0; k < s_n; ++k) {
+          if (lanes >= max_lanes || T >= max_nodes) break;
+          // lane: up to depth tokens after the occurrence, stopping before an EOS
+          const long long q0 = (long long)s_pos[k] + 1;
+          int len = 0;
+          for (int j = 0; j < depth; ++j) {
+            const long long q = q0 + j;
+            if (q >= N) break;
+            const int t = bank[q];
+            if (t == eos) break;
+            if (lane_id == 0) s_lane[j] = t;
+            ++len;
+          }
+          __syncwarp();
+          if (hint_insert(s_tok, s_par, T, max_nodes, s_lane, len)) {
+            ++lanes;
+            ++hint_lanes;
+          }
+          __syncwarp();
+        }
+        if (lane_id == 0 && (lanes >= max_lanes || T >= max_nodes)) s_done = 1;
+      }
+      __syncthreads();
+    }
+  }
+  // native lanes fill what the budgets leave
+  if (warp == 0) {
+    for (int i = 0; i < n_native; ++i) {
+      if (lanes >= max_lanes || T >= max_nodes) break;
+      int len = native_len[i];
+      len = len < depth ? len : depth;
+      len = len < native_stride ? len : native_stride;
+      len = len < 0 ? 0 : len;
+      for (int j = lane_id; j < len; j += 32) s_lane[j] = native[(size_t)i * native_stride + j];
+      __syncwarp();
+      if (hint_insert(s_tok, s_par, T, max_nodes, s_lane, len)) ++lanes;
+      __syncwarp();
+    }
+    for (int i = lane_id; i < T; i += 32) {
+      out_tok[i] = s_tok[i];
+      out_par[i] = s_par[i];
+    }
+    if (lane_id == 0) {
+      *out_T = T;
+      out_info[0] = n;
+      out_info[1] = hint_lanes;
+      out_info[2] = lanes;
+    }
+  }
+}
+
+// workspace: [best | pad to 256][mlen: one byte per position, padded to 256][cmax: one byte per chunk]
+size_t hint_workspace_bytes(long long bank_len) {
+  const size_t chunks = (size_t)((bank_len + kHintThreads - 1) / kHintThreads);
+  return 256 + chunks * kHintThreads + (chunks + 255) / 256 * 256;
+}
+
+cudaError_t launch_hint_tree(const int32_t* bank, int N, int eos, const int32_t* prefix, int prefix_len,
+                             const int32_t* native, const int32_t* native_len, int n_native, int native_stride,
+                             int max_lanes, int depth, int max_nodes, void* ws, int32_t* out_tok, int32_t* out_par,
+                             int32_t* out_T, int32_t* out_info, cudaStream_t st) {
+  int* best = (int*)ws;
+  uint8_t* mlen = (uint8_t*)ws + 256;
+  const long long n_chunks = ((long long)N + kHintThreads - 1) / kHintThreads;
+  uint8_t* cmax = mlen + n_chunks * kHintThreads;
+  cudaError_t e = cudaMemsetAsync(best, 0, sizeof(int), st);
+  if (e != cudaSuccess) return e;
+  int dev = 0, sms = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const int grid = (int)(n_chunks < (long long)sms * 8 ? n_chunks : (long long)sms * 8);
+  k_hint_match<<<grid, kHintThreads, 0, st>>>(bank, N, eos, prefix, prefix_len, mlen, cmax, best);
+  e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  k_hint_pack<<<1, kHintThreads, 0, st>>>(bank, N, eos, prefix, prefix_len, mlen, cmax, best, native, native_len,
+                                          n_native, native_stride, max_lanes, depth, max_nodes, out_tok, out_par,
+                                          out_T, out_info);
+  return cudaGetLastError();
+}
+
+}  // namespace oos
+
+using namespace oos;
+
+extern "C" {
+
+size_t oos_hint_workspace_bytes(int32_t bank_len) { return bank_len < 1 ? 0 : hint_workspace_bytes(bank_len); }
+
+int oos_hint_tree(const int32_t* bank, int32_t bank_len, int32_t eos, const int32_t* prefix, int32_t prefix_len,
+                  const int32_t* native, const int32_t* native_len, int32_t n_native, int32_t native_stride,
+                  int32_t max_lanes, int32_t depth, int32_t max_nodes, void* workspace, size_t ws_bytes,
+                  int32_t* out_tokens, int32_t* out_parent, int32_t* out_T, int32_t* out_info, void* stream) {
+  if (!bank || bank_len < 1 || !prefix || prefix_len < 1 || n_native < 0 || max_lanes < 0) return OOS_EINVAL;
+  if (n_native > 0 && (!native || !native_len || native_stride < 1)) return OOS_EINVAL;
+  if (depth < 1 || depth > kMaxT || max_nodes < 1 || max_nodes > kMaxT) return OOS_EINVAL;
+  if (!out_tokens || !out_parent || !out_T || !out_info) return OOS_EINVAL;
+  if (!workspace || ((uintptr_t)workspace & 255) || ws_bytes < hint_workspace_bytes(bank_len)) return OOS_EWORKSPACE;
+  return launch_hint_tree(bank, bank_len, eos, prefix, prefix_len, native, native_len, n_native, native_stride,
+                          max_lanes, depth, max_nodes, workspace, out_tokens, out_parent, out_T, out_info,
+                          (cudaStream_t)stream) == cudaSuccess
+             ? OOS_OK
+             : OOS_ECUDA;
+}
+
+}  // extern "C"
