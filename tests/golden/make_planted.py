@@ -30,7 +30,7 @@ from synth import gen  # noqa: E402
 from synth.configs import WORKLOADS  # noqa: E402
 from synth.model import ROOT as ROOT_KIND, SynthModel  # noqa: E402
 
-OUT = os.path.join(HERE, "planted.json")
+OUT = os.environ.get("PLANTED_OUT") or os.path.join(HERE, "planted.json")   # override: write elsewhere
 MIN_MARGIN = 0.06       # the tests gate at 0.05
 MAX_ROOTS = 64
 
