@@ -12,13 +12,14 @@
 //
 // k_hint_match: one thread per bank position (a block per 256-position chunk,
 // grid-stride over chunks) computes the longest n whose suffix ends there, 0
-// when nothing follows, as one byte; each chunk's maximum is kept too, and the
-// block maxima give the n of the call.  k_hint_pack: one block walks the chunk
-// maxima in bank order, 256 chunks per round, and visits only chunks that hold
-// an occurrence; in a visited chunk the positions' bytes, gathered in order by
-// warp ballots, give the occurrences, and warp 0 inserts each lane into the
-// tree held in shared memory: a lane token looks for an existing child with
-// one ballot over the nodes.
+// when nothing follows, as one byte; the maximum of each chunk and of each run
+// of 256 chunks (a "span") is kept too, and the block maxima give the n of the
+// call.  k_hint_pack: one block descends the two summaries in bank order --
+// spans, then their chunks, then positions, 256 at a time, each level's hits
+// gathered in order by warp ballots -- so only spans and chunks that hold an
+// occurrence are read, and warp 0 inserts each lane into the tree held in
+// shared memory: a lane token looks for an existing child with one ballot over
+// the nodes.
 #include <stdint.h>
 
 #include "common.cuh"
@@ -32,7 +33,7 @@ constexpr int kHintThreads = 256;   // threads of both kernels
 __global__ void __launch_bounds__(kHintThreads) k_hint_match(const int32_t* __restrict__ bank, int N, int eos,
                                                              const int32_t* __restrict__ prefix, int prefix_len,
                                                              uint8_t* __restrict__ mlen, uint8_t* __restrict__ cmax,
-                                                             int* __restrict__ best) {
+                                                             int* __restrict__ smax, int* __restrict__ best) {
   __shared__ int suf[kHintMaxN];
   __shared__ int wmax[kHintThreads / 32];
   const int nmax = prefix_len < kHintMaxN ? prefix_len : kHintMaxN;
@@ -58,11 +59,34 @@ __global__ void __launch_bounds__(kHintThreads) k_hint_match(const int32_t* __re
       int b = 0;
       for (int w = 0; w < kHintThreads / 32; ++w) b = max(b, wmax[w]);
       cmax[c] = (uint8_t)b;
+      if (b > 0) atomicMax(&smax[c / kHintThreads], b);
       bmax = max(bmax, b);
     }
     __syncthreads();
   }
   if (threadIdx.x == 0 && bmax > 0) atomicMax(best, bmax);
+}
+
+// Whole block: the values of the threads whose `has` is set, in thread order,
+// into out[0..count); returns count (the same in every thread).  Two block
+// barriers; every thread of the block must call it.
+OOS_DEV int ordered_select(bool has, int32_t value, int32_t* out, int* s_wcnt, int* s_cnt) {
+  const int warp = threadIdx.x >> 5, lane_id = threadIdx.x & 31;
+  const unsigned bal = __ballot_sync(0xffffffffu, has);
+  if (lane_id == 0) s_wcnt[warp] = __popc(bal);
+  __syncthreads();
+  if (has) {
+    int off = __popc(bal & ((1u << lane_id) - 1u));
+    for (int w = 0; w < warp; ++w) off += s_wcnt[w];
+    out[off] = value;
+  }
+  if (threadIdx.x == 0) {
+    int k = 0;
+    for (int w = 0; w < kHintThreads / 32; ++w) k += s_wcnt[w];
+    *s_cnt = k;
+  }
+  __syncthreads();
+  return *s_cnt;
 }
 
 // Insert one lane into the tree (warp 0, all lanes of the warp together).
@@ -102,6 +126,7 @@ __global__ void __launch_bounds__(kHintThreads) k_hint_pack(const int32_t* __res
                                                             const int32_t* __restrict__ prefix, int prefix_len,
                                                             const uint8_t* __restrict__ mlen,
                                                             const uint8_t* __restrict__ cmax,
+                                                            const int* __restrict__ smax,
                                                             const int* __restrict__ best,
                                                             const int32_t* __restrict__ native,
                                                             const int32_t* __restrict__ native_len, int n_native,
@@ -110,10 +135,11 @@ __global__ void __launch_bounds__(kHintThreads) k_hint_pack(const int32_t* __res
                                                             int32_t* out_T, int32_t* out_info) {
   __shared__ int32_t s_tok[kMaxT], s_par[kMaxT];
   __shared__ int32_t s_pos[kHintThreads];     // occurrences in the chunk being visited, in bank order
-  __shared__ int32_t s_chunk[kHintThreads];   // this round's chunks holding an occurrence, in order
+  __shared__ int32_t s_chunk[kHintThreads];   // the span's chunks holding an occurrence, in order
+  __shared__ int32_t s_span[kHintThreads];    // this round's spans holding an occurrence, in order
   __shared__ int32_t s_lane[kMaxT];           // the lane being inserted
   __shared__ int s_wcnt[kHintThreads / 32];
-  __shared__ int s_n, s_nc, s_done;
+  __shared__ int s_n, s_nc, s_ns, s_done;
   const int warp = threadIdx.x >> 5, lane_id = threadIdx.x & 31;
   const int n = *best;
   int T = 1, lanes = 0, hint_lanes = 0;       // warp 0's copies are the authoritative ones
@@ -125,70 +151,45 @@ __global__ void __launch_bounds__(kHintThreads) k_hint_pack(const int32_t* __res
   __syncthreads();
   // hint lanes: occurrences of the length-n suffix (match length >= n), bank order
   const long long n_chunks = ((long long)N + kHintThreads - 1) / kHintThreads;
-  for (long long cb = 0; n > 0 && cb < n_chunks; cb += kHintThreads) {
+  const long long n_spans = (n_chunks + kHintThreads - 1) / kHintThreads;
+  for (long long sb = 0; n > 0 && sb < n_spans; sb += kHintThreads) {
     if (s_done) break;
-    // the chunks of this round that hold an occurrence, in order
-    {
-      const long long c = cb + threadIdx.x;
-      const bool has = c < n_chunks && cmax[c] >= n;
-      const unsigned bal = __ballot_sync(0xffffffffu, has);
-      if (lane_id == 0) s_wcnt[warp] = __popc(bal);
-      __syncthreads();
-      if (has) {
-        int off = __popc(bal & ((1u << lane_id) - 1u));
-        for (int w = 0; w < warp; ++w) off += s_wcnt[w];
-        s_chunk[off] = (int32_t)c;
-      }
-      if (threadIdx.x == 0) {
-        int k = 0;
-        for (int w = 0; w < kHintThreads / 32; ++w) k += s_wcnt[w];
-        s_nc = k;
-      }
-      __syncthreads();
-    }
-    // visit them: the chunk's occurrences in order, then warp 0 inserts their lanes
-    for (int ci = 0; ci < s_nc; ++ci) {
+    const long long sp = sb + threadIdx.x;
+    const int ns = ordered_select(sp < n_spans && smax[sp] >= n, (int32_t)sp, s_span, s_wcnt, &s_ns);
+    for (int si = 0; si < ns; ++si) {
       if (s_done) break;
-      const long long p = (long long)s_chunk[ci] * kHintThreads + threadIdx.x;
-      const bool m = p < N && mlen[p] >= n;
-      const unsigned bal = __ballot_sync(0xffffffffu, m);
-      if (lane_id == 0) s_wcnt[warp] = __popc(bal);
-      __syncthreads();
-      if (m) {
-        int off = __popc(bal & ((1u << lane_id) - 1u));
-        for (int w = 0; w < warp; ++w) off += s_wcnt[w];
-        s_pos[off] = (int32_t)p;
-      }
-      if (threadIdx.x == 0) {
-        int c = 0;
-        for (int w = 0; w < kHintThreads / 32; ++w) c += s_wcnt[w];
-        s_n = c;
-      }
-      __syncthreads();
-      if (warp == 0) {
-        for (int k = 0; k < s_n; ++k) {
-          if (lanes >= max_lanes || T >= max_nodes) break;
-          // lane: up to depth tokens after the occurrence, stopping before an EOS
-          const long long q0 = (long long)s_pos[k] + 1;
-          int len = 0;
-          for (int j = 0; j < depth; ++j) {
-            const long long q = q0 + j;
-            if (q >= N) break;
-            const int t = bank[q];
-            if (t == eos) break;
-            if (lane_id == 0) s_lane[j] = t;
-            ++len;
+      const long long c = (long long)s_span[si] * kHintThreads + threadIdx.x;
+      const int nc = ordered_select(c < n_chunks && cmax[c] >= n, (int32_t)c, s_chunk, s_wcnt, &s_nc);
+      // visit the chunks: their occurrences in order, then warp 0 inserts their lanes
+      for (int ci = 0; ci < nc; ++ci) {
+        if (s_done) break;
+        const long long p = (long long)s_chunk[ci] * kHintThreads + threadIdx.x;
+        const int np = ordered_select(p < N && mlen[p] >= n, (int32_t)p, s_pos, s_wcnt, &s_n);
+        if (warp == 0) {
+          for (int k = 0; k < np; ++k) {
+            if (lanes >= max_lanes || T >= max_nodes) break;
+            // lane: up to depth tokens after the occurrence, stopping before an EOS
+            const long long q0 = (long long)s_pos[k] + 1;
+            int len = 0;
+            for (int j = 0; j < depth; ++j) {
+              const long long q = q0 + j;
+              if (q >= N) break;
+              const int t = bank[q];
+              if (t == eos) break;
+              if (lane_id == 0) s_lane[j] = t;
+              ++len;
+            }
+            __syncwarp();
+            if (hint_insert(s_tok, s_par, T, max_nodes, s_lane, len)) {
+              ++lanes;
+              ++hint_lanes;
+            }
+            __syncwarp();
           }
-          __syncwarp();
-          if (hint_insert(s_tok, s_par, T, max_nodes, s_lane, len)) {
-            ++lanes;
-            ++hint_lanes;
-          }
-          __syncwarp();
+          if (lane_id == 0 && (lanes >= max_lanes || T >= max_nodes)) s_done = 1;
         }
-        if (lane_id == 0 && (lanes >= max_lanes || T >= max_nodes)) s_done = 1;
+        __syncthreads();
       }
-      __syncthreads();
     }
   }
   // native lanes fill what the budgets leave
@@ -217,10 +218,12 @@ __global__ void __launch_bounds__(kHintThreads) k_hint_pack(const int32_t* __res
   }
 }
 
-// workspace: [best | pad to 256][mlen: one byte per position, padded to 256][cmax: one byte per chunk]
+// workspace: [best | pad to 256][mlen: one byte per position, padded to 256]
+//            [cmax: one byte per chunk, padded to 256][smax: one int per span]
 size_t hint_workspace_bytes(long long bank_len) {
   const size_t chunks = (size_t)((bank_len + kHintThreads - 1) / kHintThreads);
-  return 256 + chunks * kHintThreads + (chunks + 255) / 256 * 256;
+  const size_t spans = (chunks + kHintThreads - 1) / kHintThreads;
+  return 256 + chunks * kHintThreads + spans * kHintThreads + spans * 4;
 }
 
 cudaError_t launch_hint_tree(const int32_t* bank, int N, int eos, const int32_t* prefix, int prefix_len,
@@ -230,19 +233,22 @@ cudaError_t launch_hint_tree(const int32_t* bank, int N, int eos, const int32_t*
   int* best = (int*)ws;
   uint8_t* mlen = (uint8_t*)ws + 256;
   const long long n_chunks = ((long long)N + kHintThreads - 1) / kHintThreads;
+  const long long n_spans = (n_chunks + kHintThreads - 1) / kHintThreads;
   uint8_t* cmax = mlen + n_chunks * kHintThreads;
+  int* smax = (int*)(cmax + n_spans * kHintThreads);
   cudaError_t e = cudaMemsetAsync(best, 0, sizeof(int), st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(smax, 0, (size_t)n_spans * sizeof(int), st);
   if (e != cudaSuccess) return e;
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int grid = (int)(n_chunks < (long long)sms * 8 ? n_chunks : (long long)sms * 8);
-  k_hint_match<<<grid, kHintThreads, 0, st>>>(bank, N, eos, prefix, prefix_len, mlen, cmax, best);
+  k_hint_match<<<grid, kHintThreads, 0, st>>>(bank, N, eos, prefix, prefix_len, mlen, cmax, smax, best);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
-  k_hint_pack<<<1, kHintThreads, 0, st>>>(bank, N, eos, prefix, prefix_len, mlen, cmax, best, native, native_len,
-                                          n_native, native_stride, max_lanes, depth, max_nodes, out_tok, out_par,
-                                          out_T, out_info);
+  k_hint_pack<<<1, kHintThreads, 0, st>>>(bank, N, eos, prefix, prefix_len, mlen, cmax, smax, best, native,
+                                          native_len, n_native, native_stride, max_lanes, depth, max_nodes, out_tok,
+                                          out_par, out_T, out_info);
   return cudaGetLastError();
 }
 

@@ -92,3 +92,20 @@ def test_edges():
     _check([4, 5, 6], 0, [4, 5], [[1]], 4, 4, 1)            # root only
     _check([4, 5, 6], 0, [4, 5], [[1]], 0, 4, 8)            # no lanes allowed
     _check([3, 3, 3, 3, 3], 0, [3] * 9, [], 4, 4, 16)       # overlapping occurrences, suffix capped at 7
+
+
+@pytest.mark.parametrize("spots", [(3_000, 140_000, 290_000), (299_000,)])
+def test_bank_over_several_spans(spots):
+    """A 300k-token bank covers five 65536-position spans of the kernel's
+    summaries; occurrences in the first, middle and last (partial) spans, or
+    in the last one only."""
+    rng = np.random.default_rng(len(spots))
+    vocab, eos = 50000, 1
+    bank = rng.integers(2, vocab, size=300_000)
+    key = rng.integers(2, vocab, size=7)
+    for i, at in enumerate(spots):
+        bank[at:at + 7] = key
+        bank[at + 7:at + 10] = [40 + i, 41, 42]
+    y = np.concatenate([rng.integers(2, vocab, size=12), key]).tolist()
+    r = _check(bank.tolist(), eos, y, [[5, 6]], 6, 8, 96)
+    assert r["match_n"] == 7 and r["hint_lanes"] == len(spots)
