@@ -1,5 +1,6 @@
 """The C-ABI library builds for sm_103a, loads, and exports every entry point
-declared in include/oos.h (host-only checks: no GPU needed)."""
+declared in include/oos.h (host-only checks, except the one gpu-marked test of
+config validation, which needs the device's SM count)."""
 
 import ctypes
 import os
