@@ -107,18 +107,6 @@ OOS_DEV float2 dsmem_ld2(uint32_t a) {
   return v;
 }
 
-OOS_DEV void cp_async16(void* smem, const void* gmem, bool valid) {
-  const int n = valid ? 16 : 0;
-  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(smem_addr(smem)), "l"(gmem), "r"(n) : "memory");
-}
-OOS_DEV void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
-template <int N>
-OOS_DEV void cp_async_wait() { asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory"); }
-
-// Shared-memory descriptor of an MN-major operand in the 128-byte-swizzled
-// layout: 64 consecutive MN elements (bf16) per 128-byte row, one row per K
-// index, 8-row / 1024-byte swizzle atoms.  `lbo` is the byte distance between
-// consecutive 64-element MN blocks, the stride between 8-row K groups is 1024.
 // D[tmem] (+)= A[tmem] * B[smem]: A (M = 128 rows, one per lane) as packed
 // bf16 pairs, K index 2c and 2c + 1 in column c (low half first)
 OOS_DEV void tc_mma_bf16_ts(uint32_t tmem_d, uint32_t tmem_a, uint64_t bdesc, uint32_t idesc, uint32_t accumulate) {
@@ -129,6 +117,10 @@ OOS_DEV void tc_mma_bf16_ts(uint32_t tmem_d, uint32_t tmem_a, uint64_t bdesc, ui
       "r"(tmem_a), "l"(bdesc), "r"(idesc), "r"(accumulate)
       : "memory");
 }
+// Shared-memory descriptor of an MN-major operand in the 128-byte-swizzled
+// layout: 64 consecutive MN elements (bf16) per 128-byte row, one row per K
+// index, 8-row / 1024-byte swizzle atoms.  `lbo` is the byte distance between
+// consecutive 64-element MN blocks, the stride between 8-row K groups is 1024.
 OOS_DEV uint64_t smem_desc_sw128_mn(uint32_t saddr, uint32_t lbo) {
   uint64_t d = 0;
   d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
@@ -137,9 +129,6 @@ OOS_DEV uint64_t smem_desc_sw128_mn(uint32_t saddr, uint32_t lbo) {
   d |= (uint64_t)1 << 46;
   d |= (uint64_t)2 << 61;
   return d;
-}
-OOS_DEV void cp_async_arrive(uint64_t* bar) {   // arrive once this thread's earlier cp.async have landed
-  asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(smem_addr(bar)) : "memory");
 }
 OOS_DEV void fence_async_smem() { asm volatile("fence.proxy.async.shared::cta;" ::: "memory"); }
 // 2^x by the hardware approximation (relative error ~2^-22; -inf gives +0)
