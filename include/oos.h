@@ -177,7 +177,8 @@ int oos_model_destroy(oos_model* m);
  *   Lanes are merged into a prefix tree rooted at y's last token, a node
  *   numbered when created (parents first); a lane counts towards max_lanes only
  *   when it creates a node; at most max_nodes nodes (1..128), depth 1..128.
- *   workspace     DEVICE, >= oos_hint_workspace_bytes(bank_len), 256-byte aligned.
+ *   workspace     DEVICE, >= oos_hint_workspace_bytes(bank_len) (0 for bank_len < 1),
+ *                 256-byte aligned; owned by the caller, scratch for the one call.
  * Outputs (DEVICE): out_tokens / out_parent int32[max_nodes] (entries [0, T)
  * written), out_T int32[1], out_info int32[3] = (matched n, 0 when none; hint
  * lanes used; all lanes used).  Stream-ordered.  Returns OOS_EINVAL on a NULL
