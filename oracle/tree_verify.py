@@ -150,9 +150,14 @@ def cache_format(x, dtype):
     The target's KV cache is kept in the model's precision (the paper's targets
     run BF16 or FP16 caches): a bf16 cache stores round-to-nearest-even bf16
     values, so every K/V a node attends to -- cached or written by the tree
-    pass itself -- is bf16.  An fp32 cache is kept exact here (fp32 rounding of
-    K/V is far below the fp32 tolerance).
+    pass itself -- is bf16.  An fp16 cache (the paper's Qwen2.5 and Llama
+    backend) stores the fp32 value rounded to IEEE binary16, nearest-even,
+    overflowing to infinity.  An fp32 cache is kept exact here (fp32 rounding
+    of K/V is far below the fp32 tolerance).
     """
+    if dtype == "f16":
+        with np.errstate(over="ignore"):          # overflow to infinity is the format's rule
+            return np.asarray(x, dtype=np.float32).astype(np.float16).astype(np.float64)
     if dtype != "bf16":
         return x
     u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)

@@ -385,6 +385,25 @@ def test_cache_format_is_bf16_round_to_nearest_even():
     np.testing.assert_array_equal(oracle.cache_format(x, "f32"), x)
 
 
+def test_cache_format_f16_round_to_nearest_even():
+    """fp16 cache format: hand-worked binary16 cases, then torch's conversion."""
+    u = 2.0 ** -11                      # half a unit in the last place at 1.0
+    sub = 2.0 ** -24                    # smallest binary16 subnormal
+    cases = [(1.0 + u, 1.0),            # tie, kept bit even: down
+             (1.0 + 3 * u, 1.0 + 4 * u),  # tie, kept bit odd: up
+             (65504.0, 65504.0),        # largest finite
+             (65520.0, np.inf),         # tie between 65504 and 2^16: to even, which overflows
+             (sub / 2, 0.0),            # tie between 0 and the smallest subnormal: to 0
+             (1.5 * sub, 2 * sub),      # tie between 1 and 2 subnormal units: to 2
+             (-1.0 - u, -1.0)]
+    x = np.array([c[0] for c in cases])
+    np.testing.assert_array_equal(oracle.cache_format(x, "f16"), np.array([c[1] for c in cases]))
+    rng = np.random.default_rng(12)
+    y = rng.standard_normal(4096) * 50.0
+    ref = torch.from_numpy(y).to(torch.float32).to(torch.float16).to(torch.float64).numpy()
+    np.testing.assert_array_equal(oracle.cache_format(y, "f16"), ref)
+
+
 def _mini_case(seed, T=7, ctx_len=12):
     return build_case("mini-bf16", seed, T=T, recipe=dict(kind="uniform", max_depth=3), ctx_len=ctx_len, plant=0)
 
