@@ -206,6 +206,43 @@ int oos_hint_tree(const int32_t* bank, int32_t bank_len, int32_t eos, const int3
 int oos_prefill(oos_model* m, const oos_kv_cache* kv, int32_t ctx_len, const int32_t* tokens, int32_t n,
                 int32_t* out_next_token, void* stream);
 
+/* Multi-step decoding on the device: the decoding loop of Section 2 ("The
+ * ToolSpec decoding loop") with this library's verifier, n_rounds rounds with
+ * no host round trip between them.  One round:
+ *   1. the next tree from the hint bank, exactly as oos_hint_tree builds it,
+ *      with the committed tokens as the prefix (their last token is the root),
+ *      no native lanes, and max_nodes as the node budget;
+ *   2. one verification of that tree (oos_tree_verify) at the committed cache
+ *      length; the tree is padded to max_nodes nodes on the device, and the
+ *      padding is never accepted;
+ *   3. compaction of the accepted path (oos_kv_compact);
+ *   4. the commit ("Verify and commit"): the accepted draft tokens and the
+ *      bonus are appended to `committed` -- accepted_len tokens, the round's
+ *      #MAT of Section 5 -- and the committed cache length grows by
+ *      accepted_len (the root's K/V entered the cache; the bonus is the next
+ *      root, its K/V written by the round that verifies it).
+ * Arguments:
+ *   kv             cache; slots [0, ctx_len) are committed.  Needs
+ *                  ctx_len + n_rounds * max_nodes <= capacity.
+ *   committed      DEVICE int32[committed_cap]: the committed tokens
+ *                  [0, committed_len) (at least the root); the call appends.
+ *                  Needs committed_len + n_rounds * max_nodes <= committed_cap.
+ *   bank, bank_len, eos, max_lanes, depth   as oos_hint_tree (DEVICE bank).
+ *   max_nodes      node budget of every tree, 1..max_T of the handle.
+ *   out_mat        DEVICE int32[n_rounds]: accepted_len of every round.
+ *   out_state      DEVICE int32[3]: after the call, the committed cache length,
+ *                  the committed token count and the rounds run.
+ *   workspace      DEVICE, >= oos_decode_workspace_bytes(bank_len), 256-byte
+ *                  aligned; caller-owned scratch for the call.
+ * Stream-ordered.  Host errors: OOS_EINVAL, OOS_ECAPACITY, OOS_EWORKSPACE,
+ * OOS_ECUDA.  Device errors (a wait limit) go to oos_last_status; a round
+ * whose verification failed commits nothing. */
+size_t oos_decode_workspace_bytes(int32_t bank_len);
+int oos_decode(oos_model* m, const oos_kv_cache* kv, int32_t ctx_len, int32_t* committed, int32_t committed_len,
+               int32_t committed_cap, const int32_t* bank, int32_t bank_len, int32_t eos, int32_t max_lanes,
+               int32_t depth, int32_t max_nodes, int32_t n_rounds, int32_t* out_mat, int32_t* out_state,
+               void* workspace, size_t ws_bytes, void* stream);
+
 /* One verification step (Eq. 1; "Verify and commit").
  *   kv            committed cache; slots [0, ctx_len) are read, slots
  *                 [ctx_len, ctx_len+T) are overwritten with the tree's K/V.
@@ -291,21 +328,34 @@ int oos_launch_attention(oos_model* m, const oos_kv_cache* kv, int32_t layer, in
  *   hidden      DEVICE float [T, hidden_dim]: final-RMSNorm rows (for example
  *               out_final_hidden of oos_tree_verify_debug).
  *   lm_head     DEVICE [vocab, hidden_dim], element type `dtype`.
- *   out_argmax  DEVICE int32 [T]: argmax_v hidden[t] . lm_head[v] (Eq. 1; ties
- *               to the lowest id); out_top1 / out_top2 DEVICE float [T]: the
- *               largest and second-largest logit.
+ *   out_argmax  DEVICE int32 [T]: the v maximising hidden[t] . lm_head[v], the
+ *               lowest such v on ties; out_top1 / out_top2 DEVICE float [T]:
+ *               the largest and second-largest of those logits.
  * Scratch: a fixed 0.8 MB array in the library's device memory (allocated when
  * the library is loaded, held on every GPU that loads it until exit) holds the
  * per-block partial results; T must be <= 128, larger T returns OOS_EINVAL.
- * The first call on a device looks up that array's address (a one-time set-up
- * per device): make it before any stream capture.  Every call shares the
- * array, so calls that may overlap on the GPU (different streams, different
- * host threads) race and must be serialised by the caller.  CUDA cores only; a
- * correctness and portability path, not the fused tensor-core LM head of
- * oos_tree_verify. */
+ * The kernel needs that array's device address, which a call made outside
+ * stream capture looks up (cudaGetSymbolAddress) and caches for the device; a
+ * call made while its stream is being captured uses the cached address.  So
+ * make one uncaptured call on each device before any capture, and again after
+ * a cudaDeviceReset.  Every call shares the array, so calls that may overlap
+ * on the GPU (different streams, different host threads) race and must be
+ * serialised by the caller.  CUDA cores only; a correctness and portability
+ * path, not the fused tensor-core LM head of oos_tree_verify.  A row whose
+ * logits contain NaN gets an unspecified argmax. */
 int oos_lm_head_argmax_static(int32_t dtype, int32_t vocab, int32_t hidden_dim, const void* lm_head,
                               const float* hidden, int32_t T, int32_t* out_argmax, float* out_top1,
                               float* out_top2, void* stream);
+
+/* Limit, in nanoseconds, of every pipeline wait inside this handle's kernels
+ * (a TMA or tensor-core stage, a split-K partner, an attention split): a wait
+ * that runs out sets OOS_ETIMEOUT in the status word, the kernel drains its
+ * own copies and MMAs, frees its tensor memory and returns, and the rest of
+ * the step returns early.  0 or a value above the default restores the
+ * default of 2 s.  Meant for tests and diagnostics of the failure path (the
+ * paper has no counterpart).  Applies to work enqueued on `stream` after the
+ * call; synchronises `stream`. */
+int oos_set_wait_limit(oos_model* m, uint64_t limit_ns, void* stream);
 
 /* Synchronise `stream` and return the device status of the last verify on
  * this handle: OOS_OK, OOS_ETREE or OOS_ETIMEOUT (or OOS_ECUDA). */

@@ -14,7 +14,7 @@ ROOT = os.path.dirname(PKG)
 SRC = os.path.join(PKG, "csrc")
 OUT_DIR = os.path.join(PKG, "_lib")
 LIB = os.path.join(OUT_DIR, "liboos.so")
-UNITS = ["oos_api.cu", "small.cu", "gemm.cu", "attn.cu", "noalloc.cu", "hint.cu"]
+UNITS = ["oos_api.cu", "small.cu", "gemm.cu", "attn.cu", "noalloc.cu", "hint.cu", "decode.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

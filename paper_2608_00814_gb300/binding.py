@@ -84,7 +84,14 @@ def lib():
                                     c_vp, ctypes.c_size_t, c_vp, c_vp, c_vp, c_vp, c_vp]
         L.oos_hint_tree.restype = ctypes.c_int
         L.oos_accept_walk.argtypes = [c_vp, c_vp, c_vp, c_i32, c_vp, c_vp, c_vp, c_vp, c_vp, c_vp]
+        L.oos_decode_workspace_bytes.argtypes = [c_i32]
+        L.oos_decode_workspace_bytes.restype = ctypes.c_size_t
+        L.oos_decode.argtypes = [c_vp, P(OosKvCache), c_i32, c_vp, c_i32, c_i32, c_vp, c_i32, c_i32, c_i32, c_i32,
+                                 c_i32, c_i32, c_vp, c_vp, c_vp, ctypes.c_size_t, c_vp]
+        L.oos_decode.restype = ctypes.c_int
         L.oos_last_status.argtypes = [c_vp, c_vp]
+        L.oos_set_wait_limit.argtypes = [c_vp, ctypes.c_uint64, c_vp]
+        L.oos_set_wait_limit.restype = ctypes.c_int
         L.oos_launch_stage.argtypes = [c_vp, c_i32, c_i32, c_i32, c_vp]
         L.oos_launch_stage.restype = ctypes.c_int
         L.oos_launch_attention.argtypes = [c_vp, P(OosKvCache), c_i32, c_i32, c_i32, c_vp]
@@ -233,6 +240,19 @@ def oos_hint_tree(bank, eos, prefix, native, native_len, max_lanes, depth, max_n
                                _ptr(out_T), _ptr(out_info), _stream(stream)), "oos_hint_tree")
 
 
+def oos_decode_workspace_bytes(bank_len):
+    return int(lib().oos_decode_workspace_bytes(bank_len))
+
+
+def oos_decode(model, kv, ctx_len, committed, committed_len, bank, eos, max_lanes, depth, max_nodes, n_rounds,
+               out_mat, out_state, workspace, stream=None):
+    """committed: int32 device tensor (its size is the capacity); bank: int32 device tensor."""
+    _check(lib().oos_decode(model.handle, ctypes.byref(kv.c), ctx_len, _ptr(committed), committed_len,
+                            int(committed.numel()), _ptr(bank), int(bank.numel()), eos, max_lanes, depth, max_nodes,
+                            n_rounds, _ptr(out_mat), _ptr(out_state), _ptr(workspace),
+                            workspace.numel() * workspace.element_size(), _stream(stream)), "oos_decode")
+
+
 def oos_prefill(model, kv, ctx_len, tokens, n, out_next_token=None, stream=None):
     _check(lib().oos_prefill(model.handle, ctypes.byref(kv.c), ctx_len, _ptr(tokens), n, _ptr(out_next_token),
                              _stream(stream)), "oos_prefill")
@@ -268,6 +288,10 @@ def oos_lm_head_argmax_static(dtype, vocab, hidden_dim, lm_head, hidden, T, out_
     _check(lib().oos_lm_head_argmax_static(dtype, vocab, hidden_dim, _ptr(lm_head), _ptr(hidden), T, _ptr(out_argmax),
                                            _ptr(out_top1), _ptr(out_top2), _stream(stream)),
            "oos_lm_head_argmax_static")
+
+
+def oos_set_wait_limit(model, limit_ns, stream=None):
+    _check(lib().oos_set_wait_limit(model.handle, int(limit_ns), _stream(stream)), "oos_set_wait_limit")
 
 
 def oos_last_status(model, stream=None):

@@ -2,30 +2,39 @@
 //
 // Node i, query head h (kv head g = h / (nq/nkv)) attends to the committed
 // cache positions [0, ctx) and to the tree slots ctx + a for every ancestor a
-// of i (itself included): softmax(q k / sqrt(d)) v.
+// of i (itself included): softmax(q k / sqrt(d)) v.  The tree's own K/V sit in
+// slots ctx .. ctx+T-1 right after the committed ones, so the keys of one
+// (node, head) are a masked prefix of the contiguous slot range [0, ctx+T).
 //
-// bf16 path (tcgen05): split-K over the keys (flash-decoding) inside one
-// thread-block cluster.  A block owns 128 query rows of one kv head -- the
-// (node, q-head) pairs of the group, so GQA reuses every K/V tile for nq/nkv
-// heads, and 128 rows are the MMA's M -- and one contiguous range of 64-key
-// tiles (cache tiles first, the tree tail last, masked with the 128-bit
-// ancestor sets).  The blocks of the different ranges of the same rows form
-// one cluster.  Per tile: S = q K^T on the tensor cores into TMEM (q as hi + lo
-// bf16 halves, two MMA passes, with q itself held in TMEM as the A operand), a
-// softmax pass with one thread per row reading its S row from TMEM and writing
-// P (bf16) back into TMEM, O += P V on the tensor cores into TMEM (P the A
-// operand from TMEM).  Two threads issue the MMAs, one the S products and one
-// the P.V products, so neither waits behind the other's barriers.  The
-// running maximum is moved only when a tile's maximum exceeds
-// it by more than 2^8 (O rescaled in TMEM then); otherwise exp2(s - m) stays
-// below 256.  V tiles enter the P.V MMA as they arrive ([key][d], d
-// contiguous: the MN-major operand layout), through a ring of kKvStages K and V
-// tiles that keeps several tile loads in flight.  Each block then
-// leaves its unnormalised O and (max, sum) in its own shared memory, and after
-// a cluster barrier every block merges a slice of the rows by log-sum-exp,
-// reading the other blocks' shared memory (fixed split order), and writes the
-// hi/lo bf16 GEMM input.  The first cache tiles are fetched before the wait on
-// the producing kernel: no kernel of the step writes cache positions < ctx.
+// bf16 path (tcgen05), split-K over the keys inside one thread-block cluster.
+// A block owns up to 128 query rows of one kv head -- the (node, q-head) pairs
+// of the group, so GQA reuses every K/V tile for nq/nkv heads, and 128 rows
+// are the MMA's M -- and one contiguous range of 128-key tiles of [0, ctx+T).
+// The blocks of the different ranges of the same rows form one cluster (up to
+// 16 blocks, non-portable size, chosen so that every cluster is resident at
+// once).  Per tile:
+//   - S = q K^T on the tensor cores into TMEM, N = 128 keys, q as hi + lo
+//     bf16 halves (two MMA chains) held in TMEM as the A operand;
+//   - softmax, one thread per query row: the row's S from TMEM, the valid-key
+//     mask (cache keys, then the node's ancestors), exp2, and P (bf16 pairs)
+//     written back over the first 64 columns of the same S buffer;
+//   - O += P V on the tensor cores (P the A operand from TMEM, V in the
+//     MN-major layout TMA writes, [key][d]).
+// Two threads issue the MMAs (S, and P.V) so neither waits behind the other's
+// barriers; K/V tiles come by TMA through a two-stage ring.  The running
+// maximum moves only when a tile exceeds it by more than 2^8 (O is rescaled
+// in TMEM then).
+// Merge: each block stages its unnormalised O rows and (max, sum) in its own
+// shared memory, and one thread copies each owner's rows into that owner's
+// shared memory (bulk copies that complete on the owner's barrier, no round
+// trips); the owner adds the splits by log-sum-exp in split order
+// (deterministic) and writes the hi/lo bf16 GEMM input.
+//
+// The slot range is read through tensor maps over the cache's whole capacity,
+// and ctx comes from device memory (written by the step's tree preparation), so
+// one launch serves any ctx.  Keys past ctx + T in the last tile are masked,
+// and their V rows are zeroed in shared memory before the P.V product, so
+// whatever the cache holds there cannot reach the output.
 //
 // fp32 path: one block per (node, head), CUDA cores (small models only).
 #include <math.h>
@@ -37,43 +46,48 @@
 
 namespace oos {
 
-constexpr int kAttnRows = 128;    // query rows per block (tcgen05 M)
-constexpr int kAttnKeys = 64;     // keys per tile (S MMA N, P.V MMA K)
-constexpr int kAttnD = 128;       // head dim of the bf16 path
-// shared memory (bytes): operand tiles in the 128-byte-swizzled K-major layout
-constexpr int kQBytes = 2 * kAttnRows * 128;       // 64 of d per 128-byte block: 2 blocks x 128 rows
-constexpr int kKBytes = 2 * kAttnKeys * 128;       // K tile: 2 d-blocks x 64 keys
-constexpr int kVBytes = 2 * kAttnKeys * 128;       // V tile: 2 d-blocks x 64 keys
-constexpr int kKvStages = 4;                       // K and V tiles in flight
-constexpr int kOffQhi = 0;
-constexpr int kOffQlo = kOffQhi + kQBytes;
-constexpr int kOffK = kOffQlo + kQBytes;           // [kKvStages]
-constexpr int kOffV = kOffK + kKvStages * kKBytes; // [kKvStages]
-constexpr int kOffBar = kOffV + kKvStages * kVBytes;
-constexpr int kAttnSmem = kOffBar + 256 + 1024;    // + barriers + alignment slack
-constexpr int kAttnThreads = 224;                  // 7 warps, roles below
-constexpr int kOLd = kAttnD + 4;                   // merge staging row (floats)
-constexpr int kOffStage = kOffK;                   // merge staging reuses K and V
-static_assert(kOffStage + kAttnRows * kOLd * 4 + kAttnRows * 8 + kAttnRows * 8 * 4 <= kOffBar, "merge staging");
+constexpr int kAttnRows = 128;     // query rows per block (tcgen05 M)
+constexpr int kAttnKeys = 128;     // keys per tile (N of the S MMAs)
+constexpr int kAttnD = 128;        // head dim of the bf16 path
+constexpr int kKvStages = 2;       // K and V tiles in flight
+// shared memory (bytes): operand tiles in the 128-byte-swizzled layout TMA
+// writes: per tile two 64-wide d blocks of 128 keys x 128 bytes
+constexpr int kDBlock = kAttnKeys * 128;                  // 16 KB
+constexpr int kTileBytes = 2 * kDBlock;                   // 32 KB
+constexpr int kOffK = 0;                                  // [kKvStages]
+constexpr int kOffV = kOffK + kKvStages * kTileBytes;     // [kKvStages]
+constexpr int kMaxSplits = 16;
+constexpr int kRecvRows = kAttnRows + kMaxSplits;         // >= splits * ceil(rows / splits)
+// a merge row: the unnormalised O row (128 fp32), then (max, sum), padded to 16 bytes
+constexpr int kMergeLd = kAttnD + 4;                      // floats
+constexpr int kMergeRowBytes = kMergeLd * 4;              // 528
+constexpr int kOffStage = kOffK;                          // merge: this block's rows, staged over the K/V ring
+constexpr int kOffRecv = kOffV + kKvStages * kTileBytes;  // merge: rows copied in by the splits [slot][kMergeLd]
+constexpr int kOffWgt = kOffRecv + kRecvRows * kMergeRowBytes;   // merge weights [owned row][split]
+constexpr int kOffBar = kOffWgt + kAttnRows * kMaxSplits * 4;
+static_assert(kAttnRows * kMergeRowBytes <= kKvStages * 2 * kTileBytes, "merge staging");
+constexpr int kAttnSmem = kOffBar + 256 + 1024;           // + barriers + alignment slack
+constexpr int kAttnThreads = 224;                         // 7 warps, roles below
 static_assert(kAttnSmem <= 227 * 1024, "shared memory per block");
-// TMEM columns (lane = query row): S[2] fp32 scores of a tile, O fp32, q hi
-// and lo as packed bf16 pairs along d, P[2] as packed bf16 pairs along the keys
-constexpr int kTmS = 0;                            // [2] x 64
+static_assert(kMaxSplits <= 16, "cluster size");
+// TMEM columns (lane = query row): S[2] fp32 scores of a tile (P, bf16 pairs,
+// overwrites the first 64 columns of its S buffer), O fp32, q hi and lo as
+// packed bf16 pairs along d
+constexpr int kTmS = 0;                            // [2] x 128
 constexpr int kTmO = 2 * kAttnKeys;                // 128
 constexpr int kTmQ = kTmO + kAttnD;                // [hi, lo] x 64
-constexpr int kTmP = kTmQ + 2 * (kAttnD / 2);      // [2] x 32
-constexpr int kAttnTmemCols = 512;                 // power of two >= kTmP + 64
-static_assert(kTmP + 2 * (kAttnKeys / 2) <= kAttnTmemCols, "TMEM columns");
+constexpr int kAttnTmemCols = 512;
+static_assert(kTmQ + kAttnD == kAttnTmemCols, "TMEM columns");
 
 struct AttnArgs {
-  CUtensorMap qhi, qlo;     // q [node][nq][d] as (d, head in group, kv head, node), hi and lo halves
-  CUtensorMap kmap, vmap;   // cache [cap][nkv][d] as (d, kv head, position)
+  CUtensorMap kmap, vmap;   // cache [capacity][nkv][d] as (d, kv head, slot)
+  const __nv_bfloat16* q;   // [kMaxT][nq][d] hi halves; lo halves at q_lo_off
+  size_t q_lo_off;
   const unsigned long long* anc;
-  int T, nq, nkv, group, ctx;
+  const int* ctx_dev;       // committed positions of the step (written by tree preparation)
+  int T, nq, group;
   int npc;                  // nodes per block: its rows are (node, head in group), npc * group <= 128
   int splits;               // blocks per cluster (key ranges of the same rows)
-  int cache_blocks;         // 64-key tiles of the committed cache
-  int tiles;                // cache_blocks + tree tiles
   float scale_log2;         // log2(e) / sqrt(d)
   __nv_bfloat16* out;       // [T][nq*d] hi rows, lo rows at out_lo_off
   size_t out_lo_off;
@@ -87,26 +101,14 @@ OOS_DEV uint32_t cluster_rank() {
   asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
   return r;
 }
-OOS_DEV void cluster_sync() {
-  asm volatile("barrier.cluster.arrive.release.aligned;\n\tbarrier.cluster.wait.acquire.aligned;" ::: "memory");
-}
-// address of the same shared-memory variable in block `rank` of the cluster
+OOS_DEV void cluster_arrive_release() { asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory"); }
+OOS_DEV void cluster_wait_acquire() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
+// address of the same shared-memory location in block `rank` of the cluster
 OOS_DEV uint32_t dsmem_addr(const void* p, uint32_t rank) {
   uint32_t r;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_addr(p)), "r"(rank));
   return r;
 }
-OOS_DEV float4 dsmem_ld4(uint32_t a) {
-  float4 v;
-  asm volatile("ld.shared::cluster.v4.f32 {%0,%1,%2,%3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(a) : "memory");
-  return v;
-}
-OOS_DEV float2 dsmem_ld2(uint32_t a) {
-  float2 v;
-  asm volatile("ld.shared::cluster.v2.f32 {%0,%1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(a) : "memory");
-  return v;
-}
-
 // D[tmem] (+)= A[tmem] * B[smem]: A (M = 128 rows, one per lane) as packed
 // bf16 pairs, K index 2c and 2c + 1 in column c (low half first)
 OOS_DEV void tc_mma_bf16_ts(uint32_t tmem_d, uint32_t tmem_a, uint64_t bdesc, uint32_t idesc, uint32_t accumulate) {
@@ -137,19 +139,6 @@ OOS_DEV float ex2_approx(float x) {
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
-// 32 lanes x 32 bit, 16 consecutive columns per thread, TMEM <- registers
-OOS_DEV void tmem_st16(uint32_t taddr, const float (&v)[16]) {
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
-          taddr),
-      "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])), "r"(__float_as_uint(v[3])),
-      "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])), "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])),
-      "r"(__float_as_uint(v[8])), "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])),
-      "r"(__float_as_uint(v[11])), "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])),
-      "r"(__float_as_uint(v[14])), "r"(__float_as_uint(v[15]))
-      : "memory");
-  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-}
 // 32 lanes x 32 bit, 16 consecutive columns per thread, TMEM <- raw words
 OOS_DEV void tmem_st16u(uint32_t taddr, const uint32_t* v) {
   asm volatile(
@@ -158,113 +147,192 @@ OOS_DEV void tmem_st16u(uint32_t taddr, const uint32_t* v) {
       "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]), "r"(v[8]), "r"(v[9]),
       "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15])
       : "memory");
-  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
-// 16-byte chunk c of row r of a 128-byte-swizzled tile (rows 128 bytes apart,
-// 8-row / 1024-byte swizzle atoms, tile base 1024-aligned)
-OOS_DEV uint32_t sw128(int r, int c) { return (uint32_t)(r * 128 + ((c ^ (r & 7)) << 4)); }
+OOS_DEV void tmem_wait_st() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+// 32 lanes x 32 bit, 32 consecutive columns per thread, without waiting: the
+// caller issues several, then tmem_wait_ld_regs over every register loaded
+OOS_DEV void tmem_ld32_nowait(uint32_t taddr, float* v) {
+  uint32_t* r = reinterpret_cast<uint32_t*>(v);
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+      "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+        "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15]),
+        "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]), "=r"(r[22]), "=r"(r[23]),
+        "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+}
+// wait for the thread's outstanding TMEM loads; the empty statements after it
+// make every later use of v[0..n) depend on the wait
+template <int N>
+OOS_DEV void tmem_wait_ld_regs(float (&v)[N]) {
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < N; ++i) asm volatile("" : "+f"(v[i]));
+}
+// all 128 columns of one lane row starting at taddr
+OOS_DEV void tmem_ld128(uint32_t taddr, float (&v)[128]) {
+#pragma unroll
+  for (int c = 0; c < 4; ++c) tmem_ld32_nowait(taddr + c * 32, v + c * 32);
+  tmem_wait_ld_regs(v);
+}
+// bulk copy shared::cta -> shared::cluster of another block, completing bytes on
+// that block's mbarrier (both remote addresses from mapa)
+OOS_DEV void bulk_copy_to_peer(uint32_t dst, const void* src, uint32_t bytes, uint32_t remote_bar) {
+  asm volatile("cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                   dst),
+               "r"(smem_addr(src)), "r"(bytes), "r"(remote_bar)
+               : "memory");
+}
+OOS_DEV void bulk_commit_and_wait_read() {
+  asm volatile("cp.async.bulk.commit_group;\n\tcp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+
+// 128-bit masks as (lo: bits 0..63, hi: bits 64..127)
+OOS_DEV void shr128(unsigned long long lo, unsigned long long hi, int s, unsigned long long& rlo,
+                    unsigned long long& rhi) {
+  if (s >= 128) { rlo = 0; rhi = 0; }
+  else if (s >= 64) { rlo = s == 64 ? hi : hi >> (s - 64); rhi = 0; }
+  else if (s == 0) { rlo = lo; rhi = hi; }
+  else { rlo = (lo >> s) | (hi << (64 - s)); rhi = hi >> s; }
+}
+OOS_DEV void shl128(unsigned long long lo, unsigned long long hi, int s, unsigned long long& rlo,
+                    unsigned long long& rhi) {
+  if (s >= 128) { rlo = 0; rhi = 0; }
+  else if (s >= 64) { rhi = s == 64 ? lo : lo << (s - 64); rlo = 0; }
+  else if (s == 0) { rlo = lo; rhi = hi; }
+  else { rhi = (hi << s) | (lo >> (64 - s)); rlo = lo << s; }
+}
 
 // sites of the bounded waits (recorded on the status word when one expires)
-enum { AW_KEMPTY = 21, AW_VEMPTY, AW_QFULL, AW_KFULL, AW_SEMPTY, AW_PFULL, AW_VFULL, AW_SFULL, AW_PV_RESCALE,
-       AW_PV_FOR_P, AW_ODONE };
+enum { AW_KEMPTY = 21, AW_VEMPTY, AW_QTM, AW_KFULL, AW_SFREE, AW_PFULL, AW_VFULL, AW_SFULL, AW_PV_RESCALE,
+       AW_VZERO, AW_ODONE, AW_RECV };
 OOS_DEV bool attn_wait(uint64_t* bar, uint32_t parity, volatile int* abort, uint32_t* status, uint32_t site, int ti) {
   if (mbar_wait(bar, parity, abort, status)) return true;
   if (*(volatile uint32_t*)(status + 1) == 0u && (*(volatile uint32_t*)status & ST_TIMEOUT))
     record_timeout(status, site, ti, blockIdx.y, (int)blockIdx.z);
   return false;
 }
+// a CTA's own copies or MMAs draining after an abort: bounded by the default limit
+OOS_DEV void drain_wait(uint64_t* bar, uint32_t parity) {
+  const unsigned long long t0 = globaltimer();
+  while (!mbar_test(smem_addr(bar), parity) && globaltimer() - t0 < kWaitLimitNs) {
+  }
+}
 
-// Block roles: warp 0 lane 0 loads (q once, K and V per tile, by TMA into the
-// swizzled layouts); warp 1 lane 0 issues the S MMAs, warp 6 lane 0 the P.V
-// MMAs; warps 2..5 run the softmax (thread = query row = TMEM lane).
+// Block roles: warp 0 lane 0 loads K and V tiles (TMA into the swizzled
+// layouts); warp 1 lane 0 issues the S MMAs, warp 6 lane 0 the P.V MMAs;
+// warps 2..5 load q into TMEM and run the softmax (thread = query row = TMEM
+// lane); all warps take part in the merge.
 __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_constant__ AttnArgs a) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* sm = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   uint64_t* bar = reinterpret_cast<uint64_t*>(sm + kOffBar);
-  uint64_t* qfull = bar;                      // TMA transaction bytes
-  uint64_t* kfull = bar + 1;                  // [kKvStages] TMA transaction bytes
-  uint64_t* kempty = kfull + kKvStages;       // [kKvStages] S MMAs done
-  uint64_t* vfull = kempty + kKvStages;       // [kKvStages] TMA transaction bytes
-  uint64_t* vempty = vfull + kKvStages;       // [kKvStages] P.V MMAs done
-  uint64_t* sfull = vempty + kKvStages;       // [2] S MMAs done
-  uint64_t* sempty = sfull + 2;               // [2] 4 softmax warps
-  uint64_t* pfull = sempty + 2;               // [2] 4 softmax warps
-  uint64_t* pvdone = pfull + 2;               // [2] P.V MMAs done (P buffer free, O current)
-  uint64_t* odone = pvdone + 2;               // all MMAs of both issuers done
-  uint64_t* qtm = odone + 1;                  // 4 softmax warps: q rows are in TMEM
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(qtm + 1);
-  static_assert((1 + 4 * kKvStages + 10) * 8 + 8 <= 256, "barrier block");
+  uint64_t* kfull = bar;          // [2] TMA transaction bytes
+  uint64_t* kempty = bar + 2;     // [2] S MMAs of the stage's tile done
+  uint64_t* vfull = bar + 4;      // [2] TMA transaction bytes
+  uint64_t* vempty = bar + 6;     // [2] P.V MMAs of the stage's tile done
+  uint64_t* sfull = bar + 8;      // [2] S MMAs done
+  uint64_t* pfull = bar + 10;     // [2] 4 softmax warps: P written
+  uint64_t* pvdone = bar + 12;    // [2] P.V MMAs done (S/P buffer free, O current)
+  uint64_t* qtm = bar + 14;       // 4 softmax warps: q rows are in TMEM
+  uint64_t* odone = bar + 15;     // both MMA issuers done
+  uint64_t* recv_full = bar + 16; // merge: every split's rows for this block copied in (transaction bytes)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar + 17);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  // the argument block is addressable (its TMA maps are passed by address), so
-  // its fields are read once into registers here rather than in the loops
-  const int T = a.T, nq = a.nq, group = a.group, ctx = a.ctx, npc = a.npc, n_splits = a.splits;
-  const int cache_blocks = a.cache_blocks, n_all = a.tiles;
+  static_assert(17 * 8 + 8 <= 256, "barrier block");
+
+  const int T = a.T, nq = a.nq, G = a.group, npc = a.npc, S = a.splits;
   const float scale_log2 = a.scale_log2;
-  const unsigned long long* anc = a.anc;
-  __nv_bfloat16* const out = a.out;
-  const size_t out_lo_off = a.out_lo_off;
   uint32_t* status = a.status;
-  pdl_trigger();
   const int rb = blockIdx.x, g = blockIdx.y, split = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int rows = npc * group;   // query rows of this block: (node, head in group)
+  const int node0 = rb * npc;
+  const int rows = npc * G;                                   // query rows of the block
+  const int vrows = max(0, min(rows, (T - node0) * G));       // rows of real nodes
 
-  // tiles [t0, t1) of this block: cache tiles, then the tree tail
-  const int t0 = (int)((long long)split * n_all / n_splits);
-  const int t1 = (int)((long long)(split + 1) * n_all / n_splits);
-  const int n_tiles = t1 - t0;
-  auto tile_keys = [&](int ti, int& key0, int& key_end, bool& tree) {
-    const int t = t0 + ti;
-    if (t < cache_blocks) {
-      key0 = t * kAttnKeys;
-      key_end = min(ctx, key0 + kAttnKeys);
-      tree = false;
-    } else {
-      key0 = ctx + (t - cache_blocks) * kAttnKeys;
-      key_end = ctx + T;
-      tree = true;
-    }
-  };
+  // Committed positions of the step.  The step's tree preparation wrote them
+  // and has completed: every kernel of the step lets its dependents launch
+  // only after its own dependency wait, so when this kernel starts the kernel
+  // two launches back and everything before it are complete.
+  const int ctx = *a.ctx_dev;
+  const int n_all = (ctx + T + kAttnKeys - 1) / kAttnKeys;   // tiles over slots [0, ctx + T)
+  const int t0 = (int)((long long)split * n_all / S);
+  const int n_tiles = (int)((long long)(split + 1) * n_all / S) - t0;
+  // merge: rows [0, vrows) are dealt to the S blocks of the cluster, block j
+  // owning rows [vrows j / S, vrows (j+1) / S)
+  const int n_max = (vrows + S - 1) / S;
+  const int lr0_mine = (int)((long long)vrows * split / S);
+  const int n_mine = (int)((long long)vrows * (split + 1) / S) - lr0_mine;
 
   if (threadIdx.x == 0) {
-    mbar_init(qfull, 1);
-    for (int s = 0; s < kKvStages; ++s) {
+    for (int s = 0; s < 2; ++s) {
       mbar_init(&kfull[s], 1);
       mbar_init(&kempty[s], 1);
       mbar_init(&vfull[s], 1);
       mbar_init(&vempty[s], 1);
+      mbar_init(&sfull[s], 1);
+      mbar_init(&pfull[s], 4);
+      mbar_init(&pvdone[s], 1);
     }
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(&sfull[b], 1);
-      mbar_init(&sempty[b], 4);
-      mbar_init(&pfull[b], 4);
-      mbar_init(&pvdone[b], 1);
-    }
-    mbar_init(odone, 2);   // both MMA issuers
     mbar_init(qtm, 4);
+    mbar_init(odone, 2);
+    mbar_init(recv_full, 1);
+    // every split copies its rows of this block in: S * n_mine merge rows
+    mbar_arrive_expect_tx(recv_full, (uint32_t)(S * n_mine * kMergeRowBytes));
     *abort_flag = 0;
     mbar_fence_init();
   }
   if (warp == 2) tmem_alloc(tmem_slot, kAttnTmemCols);
-  // q rows past the block's (node, head) rows are MMA padding: zero them (the
-  // q loads fill rows [0, rows) only)
-  for (int i = threadIdx.x; i < 4 * (kAttnRows - rows) * 8; i += blockDim.x) {
-    const int blk = i / ((kAttnRows - rows) * 8), rr = rows + (i / 8) % (kAttnRows - rows), ch = i % 8;
-    *reinterpret_cast<uint4*>(sm + kOffQhi + blk * (kAttnRows * 128) + sw128(rr, ch)) = make_uint4(0, 0, 0, 0);
-  }
-  fence_async_smem();
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  // Another block may copy into this block's shared memory only once the
+  // block runs and its receive barrier is armed: arrive now, and every block
+  // waits for the whole cluster before its merge copies.
+  cluster_arrive_release();
   const uint32_t tmem = *tmem_slot;
   const uint32_t tmem_o = tmem + kTmO;
 
   if (warp == 0) {
     // ------------------------------------------------------------ loader (one thread, TMA)
     if (lane == 0) {
-      // HBM is nearly idle during attention: pull this block's share of the
-      // next GEMM's weights into L2
-      if (a.pf) {
+      tma_prefetch_desc(&a.kmap);
+      tma_prefetch_desc(&a.vmap);
+      const uint64_t pol_kv = policy_evict_first();
+      auto load = [&](int ti, bool v) {   // K or V tile: two 64-wide d blocks of 128 slots
+        const int st = ti & 1;
+        const int key0 = (t0 + ti) * kAttnKeys;
+        uint64_t* full = v ? &vfull[st] : &kfull[st];
+        unsigned char* dst = sm + (v ? kOffV : kOffK) + st * kTileBytes;
+        mbar_arrive_expect_tx(full, kTileBytes);
+        tma_load_3d(dst, v ? &a.vmap : &a.kmap, full, 0, g, key0, pol_kv);
+        tma_load_3d(dst + kDBlock, v ? &a.vmap : &a.kmap, full, 64, g, key0, pol_kv);
+      };
+      // tiles of committed slots only do not depend on the producing kernel:
+      // the first stages are fetched before waiting for it
+      int nk = 0, nv = 0;   // K and V tiles issued
+      while (nk < n_tiles && nk < kKvStages && (t0 + nk + 1) * kAttnKeys <= ctx) {
+        load(nk, false);
+        load(nk, true);
+        ++nk;
+        ++nv;
+      }
+      pdl_wait();
+      pdl_trigger();
+      for (int ti = nk; ti < n_tiles; ++ti) {
+        const int st = ti & 1;
+        const uint32_t use = (uint32_t)(ti >> 1);
+        if (!attn_wait(&kempty[st], (use & 1u) ^ 1u, abort_flag, status, AW_KEMPTY, ti)) break;
+        load(ti, false);
+        ++nk;
+        if (!attn_wait(&vempty[st], (use & 1u) ^ 1u, abort_flag, status, AW_VEMPTY, ti)) break;
+        load(ti, true);
+        ++nv;
+      }
+      // HBM is nearly idle for the rest of the attention: pull this block's
+      // share of the next GEMM's weights into L2 (after this block's own loads)
+      if (a.pf && !*abort_flag) {
         const size_t nb = (size_t)gridDim.x * gridDim.y * gridDim.z;
         const size_t bid = blockIdx.x + (size_t)gridDim.x * (blockIdx.y + (size_t)gridDim.y * blockIdx.z);
         const size_t per = ((a.pf_bytes + nb - 1) / nb + 4095) & ~(size_t)4095;
@@ -275,78 +343,33 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
           asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(a.pf + o), "r"(len & ~15u) : "memory");
         }
       }
-      tma_prefetch_desc(&a.kmap);
-      tma_prefetch_desc(&a.vmap);
-      const uint64_t pol_kv = policy_evict_first();
-      auto load_kv = [&](int ti, bool v) {   // K or V tile: two 64-wide d blocks of 64 keys
-        int k0, ke;
-        bool tr;
-        tile_keys(ti, k0, ke, tr);
-        const int s = ti % kKvStages;
-        uint64_t* full = v ? &vfull[s] : &kfull[s];
-        unsigned char* dst = sm + (v ? kOffV + s * kVBytes : kOffK + s * kKBytes);
-        mbar_arrive_expect_tx(full, 2 * kAttnKeys * 128);
-        tma_load_3d(dst, v ? &a.vmap : &a.kmap, full, 0, g, k0, pol_kv);
-        tma_load_3d(dst + kAttnKeys * 128, v ? &a.vmap : &a.kmap, full, 64, g, k0, pol_kv);
-      };
-      // cache tiles do not depend on the producing kernel: the first stages
-      // are fetched before waiting for it; tree tiles and q after
-      int pre = 0;
-      for (int ti = 0; ti < n_tiles && ti < kKvStages; ++ti) {
-        int k0, ke;
-        bool tr;
-        tile_keys(ti, k0, ke, tr);
-        if (tr) break;
-        load_kv(ti, false);
-        load_kv(ti, true);
-        pre = ti + 1;
-      }
-      pdl_wait();
-      // q rows of the block's nodes, hi and lo halves, two 64-wide d blocks each
-      tma_prefetch_desc(&a.qhi);
-      tma_prefetch_desc(&a.qlo);
-      const uint64_t pol_q = policy_evict_last();
-      mbar_arrive_expect_tx(qfull, 4 * rows * 128);
-      const int node0 = rb * npc;
-      tma_load_4d(sm + kOffQhi, &a.qhi, qfull, 0, 0, g, node0, pol_q);
-      tma_load_4d(sm + kOffQhi + kAttnRows * 128, &a.qhi, qfull, 64, 0, g, node0, pol_q);
-      tma_load_4d(sm + kOffQlo, &a.qlo, qfull, 0, 0, g, node0, pol_q);
-      tma_load_4d(sm + kOffQlo + kAttnRows * 128, &a.qlo, qfull, 64, 0, g, node0, pol_q);
-      for (int ti = pre; ti < n_tiles; ++ti) {
-        const int st = ti % kKvStages;
-        const uint32_t use = (uint32_t)(ti / kKvStages);
-        if (!attn_wait(&kempty[st], (use & 1u) ^ 1u, abort_flag, status, AW_KEMPTY, ti)) break;
-        load_kv(ti, false);
-        if (!attn_wait(&vempty[st], (use & 1u) ^ 1u, abort_flag, status, AW_VEMPTY, ti)) break;
-        load_kv(ti, true);
+      if (*abort_flag) {
+        // let this block's copies in flight land before it moves on
+        for (int ti = nk > 2 ? nk - 2 : 0; ti < nk; ++ti) drain_wait(&kfull[ti & 1], (uint32_t)(ti >> 1) & 1u);
+        for (int ti = nv > 2 ? nv - 2 : 0; ti < nv; ++ti) drain_wait(&vfull[ti & 1], (uint32_t)(ti >> 1) & 1u);
       }
     }
   } else if (warp == 1 || warp == 6) {
     // ------------------------------------------------------------ MMA issuers
-    // warp 1 lane 0 issues S = q K^T, warp 6 lane 0 issues O += P V: two
-    // threads, so that neither kind waits behind the other's barriers and the
-    // tensor cores always have queued work.  Operands reach the tensor cores
-    // through the async proxy only: q, K and V by TMA, P from threads that
-    // fence before they arrive on pfull (the zeroed q padding rows were fenced
-    // before the block barrier).  Descriptors: the start address is the low
-    // field (16-byte units), so a byte offset o inside an operand region is
-    // added as o >> 4.
+    // Operands reach the tensor cores through the async proxy only: K and V
+    // by TMA, q and P from threads that wait for their TMEM stores before they
+    // arrive, the zeroed V rows fenced by the threads that wrote them.
+    // Descriptors: the start address is the low field (16-byte units), so a
+    // byte offset o inside an operand region is added as o >> 4.
     if (lane == 0 && warp == 1) {
       constexpr uint32_t idesc_s = idesc_bf16_f32(kAttnRows, kAttnKeys);
-      bool ok = attn_wait(qtm, 0, abort_flag, status, AW_QFULL, 0);
+      bool ok = attn_wait(qtm, 0, abort_flag, status, AW_QTM, 0);
       tc_fence_after();
       const uint64_t kdesc0 = smem_desc_sw128(smem_addr(sm + kOffK));
-      // S buffer ti & 1 is free once the softmax has read tile ti - 2's scores,
-      // before P of tile ti - 2 is ready: the scores run ahead of the softmax
       for (int ti = 0; ti < n_tiles && ok; ++ti) {
         const int b = ti & 1;
         const uint32_t use = (uint32_t)(ti >> 1);
-        const int st = ti % kKvStages;
-        if (!attn_wait(&kfull[st], (uint32_t)(ti / kKvStages) & 1u, abort_flag, status, AW_KFULL, ti) ||
-            !attn_wait(&sempty[b], (use & 1u) ^ 1u, abort_flag, status, AW_SEMPTY, ti))
+        // S buffer b holds P of tile ti - 2 until that tile's P.V is done
+        if (!attn_wait(&kfull[b], use & 1u, abort_flag, status, AW_KFULL, ti) ||
+            !attn_wait(&pvdone[b], (use & 1u) ^ 1u, abort_flag, status, AW_SFREE, ti))
           break;
         tc_fence_after();
-        const uint64_t kd0 = kdesc0 + (uint64_t)((st * kKBytes) >> 4);
+        const uint64_t kd0 = kdesc0 + (uint64_t)((b * kTileBytes) >> 4);
         const uint32_t d = tmem + kTmS + b * kAttnKeys;
         // S = q_hi K^T + q_lo K^T over the 128 head dims: q from TMEM (8
         // columns = 16 of d per MMA), K from the two 64-wide d blocks (32 bytes
@@ -355,247 +378,254 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
         for (int half = 0; half < 2; ++half) {
 #pragma unroll
           for (int k = 0; k < kAttnD / 16; ++k) {
-            const uint64_t kd = kd0 + (uint64_t)(((k >> 2) * (kAttnKeys * 128)) >> 4) + 2 * (k & 3);
+            const uint64_t kd = kd0 + (uint64_t)(((k >> 2) * kDBlock) >> 4) + 2 * (k & 3);
             tc_mma_bf16_ts(d, tmem + kTmQ + half * (kAttnD / 2) + 8 * k, kd, idesc_s, (half > 0 || k > 0) ? 1u : 0u);
           }
         }
-        tc_commit(&kempty[st]);
+        tc_commit(&kempty[b]);
         tc_commit(&sfull[b]);
       }
       tc_commit(odone);
     } else if (lane == 0 && warp == 6) {
       constexpr uint32_t idesc_pv = idesc_bf16_f32(kAttnRows, kAttnD) | (1u << 16);   // B (V) MN-major
-      // V tile: d blocks of 64 (8 KB apart) along N, 16 keys (2 KB) per MMA along K
-      const uint64_t vdesc0 = smem_desc_sw128_mn(smem_addr(sm + kOffV), kAttnKeys * 128);
+      // V tile: d blocks of 64 (kDBlock apart) along N, 16 keys (2 KB) per MMA along K
+      const uint64_t vdesc0 = smem_desc_sw128_mn(smem_addr(sm + kOffV), kDBlock);
       for (int ti = 0; ti < n_tiles; ++ti) {
         const int b = ti & 1;
         const uint32_t use = (uint32_t)(ti >> 1);
-        const int st = ti % kKvStages;
         if (!attn_wait(&pfull[b], use & 1u, abort_flag, status, AW_PFULL, ti) ||
-            !attn_wait(&vfull[st], (uint32_t)(ti / kKvStages) & 1u, abort_flag, status, AW_VFULL, ti))
+            !attn_wait(&vfull[b], use & 1u, abort_flag, status, AW_VFULL, ti))
           break;
         tc_fence_after();
-        const uint32_t pt = tmem + kTmP + b * (kAttnKeys / 2);   // P: 8 columns = 16 keys per MMA
-        const uint64_t vd = vdesc0 + (uint64_t)((st * kVBytes) >> 4);
+        const uint32_t pt = tmem + kTmS + b * kAttnKeys;   // P: 8 columns = 16 keys per MMA
+        const uint64_t vd = vdesc0 + (uint64_t)((b * kTileBytes) >> 4);
 #pragma unroll
         for (int kk = 0; kk < kAttnKeys / 16; ++kk)
-          tc_mma_bf16_ts(tmem_o, pt + 8 * kk, vd + (uint64_t)((kk * 16 * 128) >> 4), idesc_pv, (ti > 0 || kk > 0) ? 1u : 0u);
+          tc_mma_bf16_ts(tmem_o, pt + 8 * kk, vd + (uint64_t)((kk * 16 * 128) >> 4), idesc_pv,
+                         (ti > 0 || kk > 0) ? 1u : 0u);
         tc_commit(&pvdone[b]);
-        tc_commit(&vempty[st]);
+        tc_commit(&vempty[b]);
       }
       tc_commit(odone);
     }
   }
 
-  // ------------------------------------------------------------ softmax (warps 2..5)
+  // ------------------------------------------------------------ q and softmax (warps 2..5)
   float m_used = -INFINITY, l_sum = 0.f;
   const int q4 = warp & 3;
   const int lrow = q4 * 32 + lane;                  // local row = TMEM lane
   const uint32_t lane_off = (uint32_t)(q4 * 32) << 16;
   if (warp >= 2 && warp <= 5) {
-    const int node = min(rb * npc + min(lrow, rows - 1) / group, T - 1);
+    const bool real = lrow < vrows;
+    const int node = real ? node0 + lrow / G : node0;
     pdl_wait();
-    const unsigned long long anc0 = anc[2 * node], anc1 = anc[2 * node + 1];
-    // this thread's q row (hi, lo) from the TMA tile into TMEM, the S MMAs'
-    // A operand: 16 columns per store = 32 of d as bf16 pairs; padding rows
-    // past the block's rows are the zeroed shared-memory rows
-    const bool qok = __all_sync(0xffffffffu, attn_wait(qfull, 0, abort_flag, status, AW_QFULL, 0));
-    if (qok) {
+    pdl_trigger();
+    const unsigned long long anc0 = a.anc[2 * node], anc1 = a.anc[2 * node + 1];
+    {
+      // this thread's q row (hi then lo, 64 columns each as bf16 pairs) into
+      // TMEM, the S MMAs' A operand; rows of padding nodes are zero
+      const __nv_bfloat16* qh = a.q + ((size_t)node * nq + g * G + (real ? lrow % G : 0)) * kAttnD;
+      uint4 w[2][16];
 #pragma unroll
-      for (int part = 0; part < 8; ++part) {   // (hi/lo, 64-wide d block, half of its 8 chunks)
-        const unsigned char* qb = sm + ((part >> 2) ? kOffQlo : kOffQhi) + ((part >> 1) & 1) * (kAttnRows * 128);
-        uint32_t w[16];
+      for (int h = 0; h < 2; ++h) {
+        const uint4* src = reinterpret_cast<const uint4*>(h ? qh + a.q_lo_off : qh);
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          const uint4 v = *reinterpret_cast<const uint4*>(qb + sw128(lrow, (part & 1) * 4 + c));
-          w[4 * c] = v.x;
-          w[4 * c + 1] = v.y;
-          w[4 * c + 2] = v.z;
-          w[4 * c + 3] = v.w;
-        }
-        tmem_st16u(tmem + lane_off + kTmQ + part * 16, w);
+        for (int c = 0; c < 16; ++c) w[h][c] = real ? __ldcg(src + c) : make_uint4(0, 0, 0, 0);
       }
+#pragma unroll
+      for (int h = 0; h < 2; ++h)
+#pragma unroll
+        for (int part = 0; part < 4; ++part)
+          tmem_st16u(tmem + lane_off + kTmQ + h * (kAttnD / 2) + part * 16,
+                     reinterpret_cast<const uint32_t*>(&w[h][part * 4]));
+      tmem_wait_st();
     }
     tc_fence_before();
     __syncwarp();
     if (lane == 0) mbar_arrive(qtm);
-    for (int ti = 0; ti < (qok ? n_tiles : 0); ++ti) {
+    for (int ti = 0; ti < n_tiles; ++ti) {
       const int b = ti & 1;
       const uint32_t use = (uint32_t)(ti >> 1);
       // every wait's outcome is made warp-uniform: the .sync.aligned TMEM
       // accesses and __syncwarp below need the whole warp on one path
       if (!__all_sync(0xffffffffu, attn_wait(&sfull[b], use & 1u, abort_flag, status, AW_SFULL, ti))) break;
       tc_fence_after();
-      float s[kAttnKeys];
-#pragma unroll
-      for (int c = 0; c < kAttnKeys / 16; ++c) {
-        float v[16];
-        tmem_ld16(tmem + lane_off + kTmS + b * kAttnKeys + c * 16, v);
-#pragma unroll
-        for (int i = 0; i < 16; ++i) s[c * 16 + i] = v[i];
+      const int key0 = (t0 + ti) * kAttnKeys;
+      // valid keys of this row in the tile: committed slots, then the tree
+      // slots of the node's ancestors (slot ctx + j for ancestor j); slots at
+      // or past ctx + T are never ancestors
+      const bool full_tile = key0 + kAttnKeys <= ctx;   // tile-uniform
+      unsigned long long mlo = ~0ull, mhi = ~0ull;
+      if (!full_tile) {
+        const int c = max(0, ctx - key0);                 // leading committed slots (< 128)
+        unsigned long long tlo, thi;
+        if (key0 >= ctx) shr128(anc0, anc1, key0 - ctx, tlo, thi);
+        else shl128(anc0, anc1, c, tlo, thi);
+        const unsigned long long clo = c >= 64 ? ~0ull : (c == 0 ? 0ull : (~0ull >> (64 - c)));
+        const unsigned long long chi = c <= 64 ? 0ull : (~0ull >> (128 - c));
+        mlo = clo | tlo;
+        mhi = chi | thi;
       }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&sempty[b]);
-      int key0, key_end;
-      bool tree;
-      tile_keys(ti, key0, key_end, tree);
-      // masked keys: past the cache end of a partial tile, tree slots that are
-      // not ancestors of this node (a tile-uniform branch: full cache tiles skip it)
-      if (tree || key_end < key0 + kAttnKeys) {
-        // key key0 + i is valid when i < n_valid and, for tree tile tt, bit i of
-        // the node's ancestor word tt (tree slot 64 tt + i) is set
-        const int n_valid = key_end - key0;
-        const unsigned long long word = !tree ? ~0ull : ((key0 - ctx) < 64 ? anc0 : anc1);
+      // the row's 128 scores, masked keys at -inf
+      float sv[kAttnKeys];
+      tmem_ld128(tmem + lane_off + kTmS + b * kAttnKeys, sv);
+      if (!full_tile) {
 #pragma unroll
         for (int i = 0; i < kAttnKeys; ++i)
-          if (i >= n_valid || !((word >> i) & 1ull)) s[i] = -INFINITY;
+          if (!((((i < 64) ? mlo : mhi) >> (i & 63)) & 1ull)) sv[i] = -INFINITY;
       }
-      // row maximum of the raw scores, four independent chains
       float mx[4] = {-INFINITY, -INFINITY, -INFINITY, -INFINITY};
 #pragma unroll
-      for (int i = 0; i < kAttnKeys; i += 4) {
-        mx[0] = fmaxf(mx[0], s[i]);
-        mx[1] = fmaxf(mx[1], s[i + 1]);
-        mx[2] = fmaxf(mx[2], s[i + 2]);
-        mx[3] = fmaxf(mx[3], s[i + 3]);
-      }
+      for (int i = 0; i < kAttnKeys; ++i) mx[i & 3] = fmaxf(mx[i & 3], sv[i]);
       const float tmax = fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])) * scale_log2;   // scale > 0
-      // move the running maximum only when this tile exceeds it by 2^8
-      // (a lane that moves its maximum rescales its O row; the whole warp takes
+      // move the running maximum only when this tile exceeds it by 2^8 (a
+      // lane that moves its maximum rescales its O row; the whole warp takes
       // part in the TMEM accesses, lanes that keep theirs scale by 1)
       const bool move = tmax > m_used + 8.f;
       const bool rescale = move && m_used != -INFINITY;
       if (__any_sync(0xffffffffu, rescale)) {
         // O holds P.V of tiles < ti: wait for the last of them, then rescale
-        {
-          const int pb = (ti - 1) & 1;
-          if (!__all_sync(0xffffffffu, attn_wait(&pvdone[pb], (uint32_t)((ti - 1) >> 1) & 1u, abort_flag, status,
-                                                 AW_PV_RESCALE, ti)))
-            break;
-          tc_fence_after();
-          const float f = rescale ? exp2f(m_used - tmax) : 1.f;
+        const int pb = (ti - 1) & 1;
+        if (!__all_sync(0xffffffffu, attn_wait(&pvdone[pb], (uint32_t)((ti - 1) >> 1) & 1u, abort_flag, status,
+                                               AW_PV_RESCALE, ti)))
+          break;
+        tc_fence_after();
+        const float f = rescale ? exp2f(m_used - tmax) : 1.f;
 #pragma unroll 1
-          for (int c = 0; c < kAttnD / 16; ++c) {
-            float v[16];
-            tmem_ld16(tmem_o + lane_off + c * 16, v);
+        for (int c = 0; c < kAttnD / 32; ++c) {   // 32 columns at a time: the scores stay in registers
+          float ov[32];
+          tmem_ld32_nowait(tmem_o + lane_off + c * 32, ov);
+          tmem_wait_ld_regs(ov);
 #pragma unroll
-            for (int i = 0; i < 16; ++i) v[i] *= f;
-            tmem_st16(tmem_o + lane_off + c * 16, v);
-          }
-          l_sum *= f;
-          tc_fence_before();
+          for (int i = 0; i < 32; ++i) ov[i] *= f;
+          tmem_st16u(tmem_o + lane_off + c * 32, reinterpret_cast<const uint32_t*>(ov));
+          tmem_st16u(tmem_o + lane_off + c * 32 + 16, reinterpret_cast<const uint32_t*>(ov + 16));
+          tmem_wait_st();
         }
+        l_sum *= f;
       }
       if (move) m_used = tmax;
       // p = 2^(s * scale - m): one FMA and one ex2 per score; a masked score
-      // (-inf) gives 0; a row with nothing unmasked yet (m = -inf) gives 0
+      // (-inf) gives 0, and a row with nothing valid yet (m = -inf) gives 0
       uint32_t pk[kAttnKeys / 2];
       float ps[4] = {0.f, 0.f, 0.f, 0.f};
       const bool live = m_used != -INFINITY;
       const float neg_m = live ? -m_used : 0.f;
 #pragma unroll
       for (int i = 0; i < kAttnKeys; i += 2) {
-        const float p0 = live ? ex2_approx(fmaf(s[i], scale_log2, neg_m)) : 0.f;
-        const float p1 = live ? ex2_approx(fmaf(s[i + 1], scale_log2, neg_m)) : 0.f;
+        const float p0 = live ? ex2_approx(fmaf(sv[i], scale_log2, neg_m)) : 0.f;
+        const float p1 = live ? ex2_approx(fmaf(sv[i + 1], scale_log2, neg_m)) : 0.f;
         const __nv_bfloat162 pp = __floats2bfloat162_rn(p0, p1);
         // the sum uses the rounded weights that P.V multiplies
         ps[(i >> 1) & 3] += __low2float(pp) + __high2float(pp);
         pk[i / 2] = *reinterpret_cast<const uint32_t*>(&pp);
       }
-      const float psum = (ps[0] + ps[1]) + (ps[2] + ps[3]);
-      l_sum += psum;
-      // P buffer b is free once P.V of tile ti - 2 has completed
-      if (!__all_sync(0xffffffffu, attn_wait(&pvdone[b], (use & 1u) ^ 1u, abort_flag, status, AW_PV_FOR_P, ti))) break;
-      // P into TMEM, the P.V MMAs' A operand (key pairs, 32 columns)
-      tmem_st16u(tmem + lane_off + kTmP + b * (kAttnKeys / 2), pk);
-      tmem_st16u(tmem + lane_off + kTmP + b * (kAttnKeys / 2) + 16, pk + 16);
+      l_sum += (ps[0] + ps[1]) + (ps[2] + ps[3]);
+      // slots at or past ctx + T in this tile hold whatever the cache holds
+      // there: zero their V rows (P is 0 for them, but 0 * NaN is not 0)
+      const int n_ok = ctx + T - key0;                   // tile-uniform
+      if (n_ok < kAttnKeys) {
+        if (!__all_sync(0xffffffffu, attn_wait(&vfull[b], use & 1u, abort_flag, status, AW_VZERO, ti))) break;
+        if (lrow >= n_ok) {
+          unsigned char* vt = sm + kOffV + b * kTileBytes + lrow * 128;
+#pragma unroll
+          for (int c = 0; c < 8; ++c) {
+            *reinterpret_cast<uint4*>(vt + c * 16) = make_uint4(0, 0, 0, 0);
+            *reinterpret_cast<uint4*>(vt + kDBlock + c * 16) = make_uint4(0, 0, 0, 0);
+          }
+          fence_async_smem();
+        }
+      }
+      // P over the first 64 columns of S buffer b (S of this tile is read)
+#pragma unroll
+      for (int part = 0; part < 4; ++part) tmem_st16u(tmem + lane_off + kTmS + b * kAttnKeys + part * 16, pk + part * 16);
+      tmem_wait_st();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&pfull[b]);
     }
+    // every role is done with the rings and TMEM once all MMAs have completed
+    attn_wait(odone, 0, abort_flag, status, AW_ODONE, n_tiles);
   }
-
-  // every role is done with the rings once all MMAs have completed
-  if (warp >= 2 && warp <= 5) attn_wait(odone, 0, abort_flag, status, AW_ODONE, n_tiles);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  // this block's unnormalised O rows and (m, l) into its own shared memory
-  float* so = reinterpret_cast<float*>(sm + kOffStage);   // [128][kOLd]
-  float* sml = so + kAttnRows * kOLd;                     // [128][2]
-  if (warp >= 2 && warp <= 5) {
-#pragma unroll 1
-    for (int c = 0; c < kAttnD / 16; ++c) {
-      float v[16];
-      tmem_ld16(tmem_o + lane_off + c * 16, v);
-#pragma unroll
-      for (int i = 0; i < 16; i += 4)
-        *reinterpret_cast<float4*>(so + lrow * kOLd + c * 16 + i) = make_float4(v[i], v[i + 1], v[i + 2], v[i + 3]);
-    }
-    *reinterpret_cast<float2*>(sml + 2 * lrow) = make_float2(*abort_flag ? -INFINITY : m_used, l_sum);
-  }
-  tc_fence_before();
-  cluster_sync();   // every block's partial is in its shared memory
 
-  // block of cluster rank c merges local rows [rows c/S, rows (c+1)/S): first
-  // each row's split weights 2^(m_s - M) / sum_s 2^(m_s - M) l_s, then thread ->
-  // (row, four head dims) sums the splits' O in split order
+  // ------------------------------------------------------------ merge
+  // Each block stages its O row, max and sum of every real row in its own
+  // shared memory (over the K/V ring, idle now), and one thread copies each
+  // owner's rows into slots split * n_max .. of that owner's receive buffer
+  // (bulk copies, completing on the owner's receive barrier).  The owner then
+  // adds the S splits of its rows by log-sum-exp, in split order.
+  float* stage = reinterpret_cast<float*>(sm + kOffStage);   // [row][kMergeLd]
+  const float* recv = reinterpret_cast<const float*>(sm + kOffRecv);
+  float* wgt = reinterpret_cast<float*>(sm + kOffWgt);
+  const bool have_o = n_tiles > 0 && !*abort_flag;   // block-uniform after the barrier
+  if (warp >= 2 && warp <= 5) {
+    float ov[kAttnD];
+    if (have_o) {
+      tmem_ld128(tmem_o + lane_off, ov);
+    } else {
+#pragma unroll
+      for (int i = 0; i < kAttnD; ++i) ov[i] = 0.f;
+    }
+    if (lrow < vrows) {
+      float* row = stage + (size_t)lrow * kMergeLd;
+#pragma unroll
+      for (int i = 0; i < kAttnD; i += 4) *reinterpret_cast<float4*>(row + i) = make_float4(ov[i], ov[i + 1], ov[i + 2], ov[i + 3]);
+      *reinterpret_cast<float4*>(row + kAttnD) = make_float4(have_o ? m_used : -INFINITY, have_o ? l_sum : 0.f, 0.f, 0.f);
+      fence_async_smem();   // the rows are read by the bulk-copy engine
+    }
+  }
+  __syncthreads();
+  cluster_wait_acquire();   // every block of the cluster runs and has armed its receive barrier
+  if (threadIdx.x == 0) {
+    for (int j = 0; j < S; ++j) {
+      const int r0 = (int)((long long)vrows * j / S), r1 = (int)((long long)vrows * (j + 1) / S);
+      if (r1 > r0)
+        bulk_copy_to_peer(dsmem_addr(sm + kOffRecv + (size_t)split * n_max * kMergeRowBytes, (uint32_t)j),
+                          stage + (size_t)r0 * kMergeLd, (uint32_t)((r1 - r0) * kMergeRowBytes),
+                          dsmem_addr(recv_full, (uint32_t)j));
+    }
+    bulk_commit_and_wait_read();   // the staged rows have been read before this block moves on
+  }
+  // this block's rows from every split
+  attn_wait(recv_full, 0, abort_flag, status, AW_RECV, 0);
   {
-    const int S = n_splits;
-    const int c = (int)cluster_rank();
-    const int lr0 = rows * c / S, lr1 = rows * (c + 1) / S;
-    float* sw = sml + 2 * kAttnRows;   // [row - lr0][kMaxAttnSplits], this block only
-    if (threadIdx.x < lr1 - lr0) {
-      const int lr = lr0 + threadIdx.x;
-      float2 ml[kMaxAttnSplits];
+    // split weights of every owned row: 2^(m_s - M) / sum_s 2^(m_s - M) l_s
+    if (threadIdx.x < n_mine) {
+      const int i = threadIdx.x;
       float M = -INFINITY;
-#pragma unroll
-      for (int sp = 0; sp < kMaxAttnSplits; ++sp) {
-        if (sp < S) {
-          ml[sp] = dsmem_ld2(dsmem_addr(sml + 2 * lr, sp));
-          M = fmaxf(M, ml[sp].x);
-        }
-      }
+      for (int s2 = 0; s2 < S; ++s2) M = fmaxf(M, recv[(size_t)(s2 * n_max + i) * kMergeLd + kAttnD]);
       float den = 0.f;
-#pragma unroll
-      for (int sp = 0; sp < kMaxAttnSplits; ++sp) {
-        if (sp < S) {
-          ml[sp].x = ml[sp].x == -INFINITY ? 0.f : exp2f(ml[sp].x - M);
-          den += ml[sp].x * ml[sp].y;
-        }
+      for (int s2 = 0; s2 < S; ++s2) {
+        const float* ml = recv + (size_t)(s2 * n_max + i) * kMergeLd + kAttnD;
+        const float w = ml[0] == -INFINITY ? 0.f : exp2f(ml[0] - M);
+        wgt[i * kMaxSplits + s2] = w;
+        den += w * ml[1];
       }
       const float inv = den > 0.f ? 1.f / den : 0.f;
-#pragma unroll
-      for (int sp = 0; sp < kMaxAttnSplits; ++sp)
-        if (sp < S) sw[threadIdx.x * kMaxAttnSplits + sp] = ml[sp].x * inv;
+      for (int s2 = 0; s2 < S; ++s2) wgt[i * kMaxSplits + s2] *= inv;
     }
     __syncthreads();
-    for (int idx = threadIdx.x; idx < (lr1 - lr0) * (kAttnD / 4); idx += blockDim.x) {
-      const int lr = lr0 + idx / (kAttnD / 4), d4 = (idx % (kAttnD / 4)) * 4;
-      const int node = rb * npc + lr / group;
-      float4 v[kMaxAttnSplits];
-#pragma unroll
-      for (int sp = 0; sp < kMaxAttnSplits; ++sp)
-        if (sp < S) v[sp] = dsmem_ld4(dsmem_addr(so + lr * kOLd + d4, sp));
+    for (int idx = threadIdx.x; idx < n_mine * (kAttnD / 4); idx += blockDim.x) {
+      const int i = idx / (kAttnD / 4), d4 = (idx % (kAttnD / 4)) * 4;
       float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-      for (int sp = 0; sp < kMaxAttnSplits; ++sp) {
-        if (sp < S) {
-          const float wgt = sw[(lr - lr0) * kMaxAttnSplits + sp];
-          acc.x += wgt * v[sp].x;
-          acc.y += wgt * v[sp].y;
-          acc.z += wgt * v[sp].z;
-          acc.w += wgt * v[sp].w;
-        }
+      for (int s2 = 0; s2 < S; ++s2) {
+        const float w = wgt[i * kMaxSplits + s2];
+        const float4 v = *reinterpret_cast<const float4*>(recv + (size_t)(s2 * n_max + i) * kMergeLd + d4);
+        acc.x += w * v.x;
+        acc.y += w * v.y;
+        acc.z += w * v.z;
+        acc.w += w * v.w;
       }
-      if (node < T) {
-        const size_t grow = (size_t)node * nq + g * group + lr % group;
-        store_act4(out, grow * kAttnD + d4, out_lo_off, acc);
-      }
+      const int lr = lr0_mine + i;
+      const size_t grow = (size_t)(node0 + lr / G) * nq + g * G + lr % G;
+      store_act4(a.out, grow * kAttnD + d4, a.out_lo_off, acc);
     }
   }
-  cluster_sync();   // no block leaves while another may still read its shared memory
+  tc_fence_before();
+  __syncthreads();
   if (warp == 2) {
     tc_fence_after();
     tmem_dealloc(tmem, kAttnTmemCols);
@@ -605,14 +635,15 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
 // ------------------------------------------------------------ fp32 path
 __global__ void __launch_bounds__(128) k_attn_f32(const float* __restrict__ q, const float* __restrict__ kc,
                                                   const float* __restrict__ vc, const unsigned long long* __restrict__ anc,
-                                                  int T, int nq, int nkv, int d, int ctx, float scale,
-                                                  float* __restrict__ out) {
+                                                  int T, int nq, int nkv, int d, const int32_t* __restrict__ ctx_dev,
+                                                  float scale, float* __restrict__ out) {
   __shared__ float qs[128];
   __shared__ float ps[128];
   __shared__ int kpos[128];
   __shared__ float red[32];
-  pdl_trigger();
   pdl_wait();
+  pdl_trigger();
+  const int ctx = *ctx_dev;
   const int i = blockIdx.x, h = blockIdx.y, g = h / (nq / nkv), tid = threadIdx.x;
   if (tid < d) qs[tid] = q[((size_t)i * nq + h) * d + tid];
   const unsigned long long w0 = anc[2 * i], w1 = anc[2 * i + 1];
@@ -656,23 +687,10 @@ __global__ void __launch_bounds__(128) k_attn_f32(const float* __restrict__ q, c
 
 int attn_nodes_per_block(int group) { return group >= kAttnRows ? 1 : kAttnRows / group; }
 
-bool attn_encode_q_maps(Model& m) {
-  const auto& c = m.cfg;
-  const int group = c.n_q_heads / c.n_kv_heads;
-  // q [node][nq][d] viewed as (d, head in group, kv head, node); a box is the
-  // (node, head in group) rows of one kv head, 64 of d at a time
-  const uint64_t dims[4] = {(uint64_t)kAttnD, (uint64_t)group, (uint64_t)c.n_kv_heads, (uint64_t)kMaxT};
-  const uint64_t strides[3] = {(uint64_t)kAttnD * 2, (uint64_t)group * kAttnD * 2, (uint64_t)c.n_q_heads * kAttnD * 2};
-  const uint32_t box[4] = {64, (uint32_t)group, 1, (uint32_t)attn_nodes_per_block(group)};
-  const __nv_bfloat16* q = (const __nv_bfloat16*)m.ws.q;
-  return encode_bf16_map(&m.qmap_hi, q, 4, dims, strides, box) &&
-         encode_bf16_map(&m.qmap_lo, q + (size_t)kMaxT * c.n_q_heads * kAttnD, 4, dims, strides, box);
-}
-
 // clusters of `sp` attention blocks resident at once on this device (occupancy query, cached)
 static int attn_max_clusters(int sp) {
-  static int cached[kMaxAttnSplits + 1] = {0};
-  if (sp < 1 || sp > kMaxAttnSplits) return 0;
+  static int cached[kMaxSplits + 1] = {0};
+  if (sp < 1 || sp > kMaxSplits) return 0;
   if (cached[sp] == 0) {
     cudaLaunchConfig_t lc = {};
     lc.gridDim = dim3(1, 1, sp);
@@ -687,32 +705,48 @@ static int attn_max_clusters(int sp) {
     lc.numAttrs = 1;
     int n = 0;
     cached[sp] = cudaOccupancyMaxActiveClusters(&n, (const void*)k_attn_tc, &lc) == cudaSuccess && n > 0 ? n : -1;
+    cudaGetLastError();
   }
   return cached[sp];
 }
 
 cudaError_t attn_setup() {
-  return cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmem);
+  cudaError_t e = cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmem);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+  return e;
 }
 
-cudaError_t launch_attention(Model& m, int layer, const void* kc, const void* vc, int ctx, int T, cudaStream_t st) {
+int attn_splits(Model& m, int ctx_hint, int T) {
+  const auto& c = m.cfg;
+  const int npc = attn_nodes_per_block(c.n_q_heads / c.n_kv_heads);
+  const int pairs = c.n_kv_heads * ((T + npc - 1) / npc);
+  const int tiles = (ctx_hint + T + kAttnKeys - 1) / kAttnKeys;
+  // the most splits (one cluster of them per row block and kv head) such that
+  // every cluster is resident at once -- one wave -- and no block is without a tile
+  for (int sp = kMaxSplits; sp >= 1; --sp) {
+    if (sp > tiles || pairs * sp > m.num_sms) continue;
+    if (attn_max_clusters(sp) >= pairs) return sp;
+  }
+  return 1;
+}
+
+cudaError_t launch_attention(Model& m, int layer, const void* kc, const void* vc, int capacity, int ctx, int T,
+                             cudaStream_t st) {
   const auto& c = m.cfg;
   if (c.dtype != OOS_DTYPE_BF16) {
     return launch(m.pdl, k_attn_f32, dim3(T, c.n_q_heads), dim3(128), 0, st, (const float*)m.ws.q, (const float*)kc,
-                  (const float*)vc, (const unsigned long long*)m.ws.anc, T, c.n_q_heads, c.n_kv_heads, c.head_dim, ctx,
-                  1.0f / sqrtf((float)c.head_dim), (float*)m.ws.attn);
+                  (const float*)vc, (const unsigned long long*)m.ws.anc, T, c.n_q_heads, c.n_kv_heads, c.head_dim,
+                  (const int32_t*)m.ws.ctx, 1.0f / sqrtf((float)c.head_dim), (float*)m.ws.attn);
   }
   AttnArgs a;
   memset(&a, 0, sizeof(a));
-  a.qhi = m.qmap_hi;
-  a.qlo = m.qmap_lo;
-  // this call's cache, (d, kv head, position) over the ctx + T valid positions:
-  // a tile reaching past them reads zeros (and masks them)
+  // this layer's cache over its whole capacity, (d, kv head, slot); encoded
+  // again only when the cache buffers change
   {
     if ((int)m.kv_maps.size() != c.n_layers) m.kv_maps.assign(c.n_layers, Model::KvMaps());
     Model::KvMaps& km = m.kv_maps[layer];
-    if (km.k != kc || km.v != vc || km.extent != ctx + T) {
-      const uint64_t dims[3] = {(uint64_t)kAttnD, (uint64_t)c.n_kv_heads, (uint64_t)(ctx + T)};
+    if (km.k != kc || km.v != vc || km.extent != capacity) {
+      const uint64_t dims[3] = {(uint64_t)kAttnD, (uint64_t)c.n_kv_heads, (uint64_t)capacity};
       const uint64_t strides[2] = {(uint64_t)kAttnD * 2, (uint64_t)c.n_kv_heads * kAttnD * 2};
       const uint32_t box[3] = {64, 1, (uint32_t)kAttnKeys};
       if (!encode_bf16_map(&km.kmap, kc, 3, dims, strides, box) ||
@@ -722,33 +756,21 @@ cudaError_t launch_attention(Model& m, int layer, const void* kc, const void* vc
       }
       km.k = kc;
       km.v = vc;
-      km.extent = ctx + T;
+      km.extent = capacity;
     }
     a.kmap = km.kmap;
     a.vmap = km.vmap;
   }
+  a.q = (const __nv_bfloat16*)m.ws.q;
+  a.q_lo_off = (size_t)kMaxT * c.n_q_heads * kAttnD;
   a.anc = m.ws.anc;
+  a.ctx_dev = m.ws.ctx;
   a.T = T;
   a.nq = c.n_q_heads;
-  a.nkv = c.n_kv_heads;
   a.group = c.n_q_heads / c.n_kv_heads;
   a.npc = attn_nodes_per_block(a.group);
-  a.ctx = ctx;
-  a.cache_blocks = (ctx + kAttnKeys - 1) / kAttnKeys;
-  a.tiles = a.cache_blocks + (T + kAttnKeys - 1) / kAttnKeys;
   const int RB = (T + a.npc - 1) / a.npc;
-  // The most splits (one cluster of them per row block and kv head) such that
-  // every cluster is resident at once -- one wave -- and no block is without a tile.
-  const int pairs = a.nkv * RB;
-  int splits = 1;
-  for (int sp = kMaxAttnSplits; sp >= 1; --sp) {
-    if (sp > a.tiles || pairs * sp > m.num_sms) continue;
-    if (attn_max_clusters(sp) >= pairs) {
-      splits = sp;
-      break;
-    }
-  }
-  a.splits = splits;
+  a.splits = attn_splits(m, ctx, T);
   a.scale_log2 = 1.4426950408889634f / sqrtf((float)kAttnD);
   a.out = (__nv_bfloat16*)m.ws.attn;
   a.out_lo_off = (size_t)kMaxT * c.n_q_heads * kAttnD;
@@ -758,7 +780,7 @@ cudaError_t launch_attention(Model& m, int layer, const void* kc, const void* vc
   a.pf_bytes = (size_t)c.hidden * c.n_q_heads * kAttnD * 2;
 
   cudaLaunchConfig_t lc = {};
-  lc.gridDim = dim3(RB, a.nkv, splits);
+  lc.gridDim = dim3(RB, c.n_kv_heads, a.splits);
   lc.blockDim = dim3(kAttnThreads);
   lc.dynamicSmemBytes = (size_t)kAttnSmem;
   lc.stream = st;
@@ -766,7 +788,7 @@ cudaError_t launch_attention(Model& m, int layer, const void* kc, const void* vc
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 1;
   attr[0].val.clusterDim.y = 1;
-  attr[0].val.clusterDim.z = splits;
+  attr[0].val.clusterDim.z = a.splits;
   attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   lc.attrs = attr;

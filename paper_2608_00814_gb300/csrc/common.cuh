@@ -15,8 +15,16 @@ enum : uint32_t {
   ST_TIMEOUT = 2u,   // a pipeline wait gave up
 };
 
-// limit of every spin-wait in these kernels (nanoseconds of %globaltimer)
+// Default limit of every pipeline wait in these kernels (nanoseconds of
+// %globaltimer).  The limit in force is a per-handle value kept in the step's
+// status block (words kStatusWaitLimit, +1: a 64-bit count of nanoseconds),
+// set to this default by oos_model_create; waits that only drain a CTA's own
+// copies or MMAs after an abort always use the default.
 constexpr unsigned long long kWaitLimitNs = 2000000000ull;
+constexpr int kStatusWaitLimit = 8;
+OOS_DEV unsigned long long wait_limit(const uint32_t* status) {
+  return *reinterpret_cast<const volatile unsigned long long*>(status + kStatusWaitLimit);
+}
 
 OOS_DEV unsigned long long globaltimer() {
   unsigned long long t;
@@ -139,18 +147,21 @@ OOS_DEV void record_timeout(uint32_t* status, uint32_t site, int phase, long lon
   }
 }
 
-// Wait for the phase with `parity` to complete.  Gives up after kWaitLimitNs or
-// when *abort becomes nonzero (another role gave up); returns false then and
-// records ST_TIMEOUT in *status (only for a genuine timeout).  Between checks of
-// the abort flag the thread sleeps on the barrier (at most 20 us at a time).
+// Wait for the phase with `parity` to complete.  Gives up after the handle's
+// wait limit or when *abort becomes nonzero (another role gave up); returns
+// false then and records ST_TIMEOUT in *status (only for a genuine timeout).
+// Between checks of the abort flag the thread sleeps on the barrier (at most
+// 20 us, and at most the limit, at a time).
 OOS_DEV bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort, uint32_t* status) {
   const uint32_t addr = smem_addr(bar);
   if (mbar_test(addr, parity)) return true;
   const unsigned long long t0 = globaltimer();
+  const unsigned long long limit = wait_limit(status);
+  const uint32_t hint = limit < 20000ull ? (uint32_t)limit : 20000u;
   while (true) {
-    if (mbar_test_sleep(addr, parity, 20000u)) return true;
+    if (mbar_test_sleep(addr, parity, hint)) return true;
     if (*abort) return false;
-    if (globaltimer() - t0 > kWaitLimitNs) {
+    if (globaltimer() - t0 > limit) {
       *abort = 1;
       atomicOr(status, ST_TIMEOUT);
       return false;

@@ -69,7 +69,7 @@ struct GemmArgs {
   const __nv_bfloat16 *bq, *bk, *bv, *gq, *gk;
   const float2* rope;   // [kMaxT][64] (cos, sin) of the step's positions
   __nv_bfloat16 *q_out, *kc, *vc;
-  int ctx;
+  const int32_t* ctx;   // committed length of the step (device; K/V of node t go to slot *ctx + t)
   // EPI_RESID
   float* x;
   const __nv_bfloat16* gain;
@@ -273,6 +273,7 @@ OOS_DEV void finish_qkv(const GemmArgs& a, int n_part, int tile, int nc, const f
   const __nv_bfloat16* gn = kind == 0 ? a.gq : kind == 1 ? a.gk : nullptr;
   const float4 b4 = bias ? bf16x4(bias + h * kTile + 4 * l) : make_float4(0.f, 0.f, 0.f, 0.f);
   const float4 g4 = gn ? bf16x4(gn + 4 * l) : make_float4(1.f, 1.f, 1.f, 1.f);
+  const int ctx = *a.ctx;
   const int m0 = 4 * (l & 15);      // rotary frequency index of this lane's first feature
   const bool first_half = l < 16;   // features 0..63 pair with 64..127 held by lane ^ 16
   for (int t0 = tb; t0 < te; t0 += nw * kFinRows) {
@@ -304,7 +305,7 @@ OOS_DEV void finish_qkv(const GemmArgs& a, int n_part, int tile, int nc, const f
         store_act4(a.q_out, ((size_t)t * a.nq + h) * kTile + 4 * l, (size_t)kMaxT * a.nq * kTile,
                    make_float4(v[0], v[1], v[2], v[3]));
       } else {           // K/V in the cache's bf16 format
-        __nv_bfloat16* dst = (kind == 1 ? a.kc : a.vc) + ((size_t)(a.ctx + t) * a.nkv + h) * kTile;
+        __nv_bfloat16* dst = (kind == 1 ? a.kc : a.vc) + ((size_t)(ctx + t) * a.nkv + h) * kTile;
         __nv_bfloat16 o[4];
 #pragma unroll
         for (int c = 0; c < 4; ++c) o[c] = __float2bfloat16_rn(v[c]);
@@ -385,7 +386,6 @@ __global__ void __launch_bounds__(192, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *tmem_slot;
-  pdl_trigger();
 
   if (warp == 0) {
     // ------------------------------------------------------------ TMA producer
@@ -433,6 +433,7 @@ __global__ void __launch_bounds__(192, 1)
         load_w(j, j);
       }
       pdl_wait();
+      pdl_trigger();
       for (int j = 0; j < n_pre; ++j) load_x(j, j);
       int stage = n_pre % S;
       uint32_t phase = (n_pre == S) ? 1u : 0u;
@@ -548,6 +549,7 @@ __global__ void __launch_bounds__(192, 1)
   } else {
     // ------------------------------------------------------------ epilogue (warps 2..5)
     pdl_wait();
+    pdl_trigger();
     const int q = warp & 3;               // TMEM lane quarter this warp may access
     const int row = q * 32 + lane;
     const int e = threadIdx.x - 64;       // 0..127
@@ -718,6 +720,7 @@ __global__ void __launch_bounds__(192, 1)
         const bool two = wt1 >= 0;
         if (e == 0) {
           const unsigned long long t0 = globaltimer();
+          const unsigned long long limit = wait_limit(a.status);
           for (int i = 0; i < (two ? 2 : 1) && !*abort_flag; ++i) {
             const int wt = i ? wt1 : wt0, nc = i ? nc1 : nc0;
             while (*(volatile int*)&a.cnt[wt] < nc) {
@@ -725,7 +728,7 @@ __global__ void __launch_bounds__(192, 1)
                 *abort_flag = 1;
                 break;
               }
-              if (globaltimer() - t0 > kWaitLimitNs) {
+              if (globaltimer() - t0 > limit) {
                 atomicOr(a.status, ST_TIMEOUT);
                 *abort_flag = 1;
                 break;
@@ -912,8 +915,7 @@ static GemmArgs base_args(Model& m, const GemmW& g, int T, int* cnt) {
   return a;
 }
 
-cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int ctx, int T, const GemmW* next,
-                            cudaStream_t st) {
+cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int T, const GemmW* next, cudaStream_t st) {
   const auto& c = m.cfg;
   const oos_layer_weights& L = m.layers[layer];
   GemmArgs a = base_args(m, m.g_qkv[layer], T, gemm_counters(m, layer, 0));
@@ -928,7 +930,7 @@ cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int ctx, in
   a.q_out = (__nv_bfloat16*)m.ws.q;
   a.kc = (__nv_bfloat16*)kc;
   a.vc = (__nv_bfloat16*)vc;
-  a.ctx = ctx;
+  a.ctx = m.ws.ctx;
   return dispatch_tc<EPI_QKV>(m, m.g_qkv[layer], m.amap_xn, T, m.g_qkv[layer].plan.grid, a, next, st);
 }
 
@@ -972,8 +974,8 @@ cudaError_t launch_lm_head_tc(Model& m, int T, cudaStream_t st) {
 __global__ void __launch_bounds__(128) k_gemm_f32(const float* __restrict__ w0, const float* __restrict__ w1,
                                                   const float* __restrict__ w2, int r0, int r1, int r2, int K,
                                                   const float* __restrict__ x, int T, float* __restrict__ part) {
-  pdl_trigger();
   pdl_wait();
+  pdl_trigger();
   const int N = r0 + r1 + r2;
   const int f = blockIdx.x * 4 + (threadIdx.x >> 5);
   const int lane = threadIdx.x & 31;
@@ -1002,8 +1004,8 @@ __global__ void __launch_bounds__(128) k_lm_head_f32(const float* __restrict__ W
                                                      const float* __restrict__ x, int T, float* am_v1, int32_t* am_i,
                                                      float* am_v2) {
   __shared__ Top2s st[4][kMaxT];
-  pdl_trigger();
   pdl_wait();
+  pdl_trigger();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int t = lane; t < T; t += 32) st[warp][t] = Top2s{-INFINITY, 0x7fffffff, -INFINITY};
   const int r_begin = blockIdx.x * rows_per_block;

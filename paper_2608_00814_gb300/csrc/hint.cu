@@ -30,12 +30,16 @@ namespace oos {
 constexpr int kHintMaxN = 7;        // longest suffix tried
 constexpr int kHintThreads = 256;   // threads of both kernels
 
+// prefix_len_dev: the prefix length in device memory (the decode loop's
+// committed length), or nullptr to use prefix_len
 __global__ void __launch_bounds__(kHintThreads) k_hint_match(const int32_t* __restrict__ bank, int N, int eos,
                                                              const int32_t* __restrict__ prefix, int prefix_len,
+                                                             const int32_t* __restrict__ prefix_len_dev,
                                                              uint8_t* __restrict__ mlen, uint8_t* __restrict__ cmax,
                                                              int* __restrict__ smax, int* __restrict__ best) {
   __shared__ int suf[kHintMaxN];
   __shared__ int wmax[kHintThreads / 32];
+  if (prefix_len_dev) prefix_len = *prefix_len_dev;
   const int nmax = prefix_len < kHintMaxN ? prefix_len : kHintMaxN;
   // suf[nmax - 1] is y's last token, suf[nmax - 1 - j] the one j before it
   if (threadIdx.x < nmax) suf[threadIdx.x] = prefix[prefix_len - nmax + threadIdx.x];
@@ -131,7 +135,8 @@ __global__ void __launch_bounds__(kHintThreads) k_hint_pack(const int32_t* __res
                                                             const int32_t* __restrict__ native,
                                                             const int32_t* __restrict__ native_len, int n_native,
                                                             int native_stride, int max_lanes, int depth,
-                                                            int max_nodes, int32_t* out_tok, int32_t* out_par,
+                                                            int max_nodes, const int32_t* __restrict__ prefix_len_dev,
+                                                            int pad_to, int32_t* out_tok, int32_t* out_par,
                                                             int32_t* out_T, int32_t* out_info) {
   __shared__ int32_t s_tok[kMaxT], s_par[kMaxT];
   __shared__ int32_t s_pos[kHintThreads];     // occurrences in the chunk being visited, in bank order
@@ -142,6 +147,7 @@ __global__ void __launch_bounds__(kHintThreads) k_hint_pack(const int32_t* __res
   __shared__ int s_n, s_nc, s_ns, s_done;
   const int warp = threadIdx.x >> 5, lane_id = threadIdx.x & 31;
   const int n = *best;
+  if (prefix_len_dev) prefix_len = *prefix_len_dev;
   int T = 1, lanes = 0, hint_lanes = 0;       // warp 0's copies are the authoritative ones
   if (threadIdx.x == 0) {
     s_tok[0] = prefix[prefix_len - 1];
@@ -209,6 +215,13 @@ __global__ void __launch_bounds__(kHintThreads) k_hint_pack(const int32_t* __res
       out_tok[i] = s_tok[i];
       out_par[i] = s_par[i];
     }
+    // padding up to a fixed node count (the decode loop verifies a fixed T):
+    // leaves under the root carrying the root's token; the verifier is told
+    // the real node count and never accepts them
+    for (int i = T + lane_id; i < pad_to; i += 32) {
+      out_tok[i] = s_tok[0];
+      out_par[i] = 0;
+    }
     if (lane_id == 0) {
       *out_T = T;
       out_info[0] = n;
@@ -227,9 +240,10 @@ size_t hint_workspace_bytes(long long bank_len) {
 }
 
 cudaError_t launch_hint_tree(const int32_t* bank, int N, int eos, const int32_t* prefix, int prefix_len,
-                             const int32_t* native, const int32_t* native_len, int n_native, int native_stride,
-                             int max_lanes, int depth, int max_nodes, void* ws, int32_t* out_tok, int32_t* out_par,
-                             int32_t* out_T, int32_t* out_info, cudaStream_t st) {
+                             const int32_t* prefix_len_dev, const int32_t* native, const int32_t* native_len,
+                             int n_native, int native_stride, int max_lanes, int depth, int max_nodes, int pad_to,
+                             void* ws, int32_t* out_tok, int32_t* out_par, int32_t* out_T, int32_t* out_info,
+                             cudaStream_t st) {
   int* best = (int*)ws;
   uint8_t* mlen = (uint8_t*)ws + 256;
   const long long n_chunks = ((long long)N + kHintThreads - 1) / kHintThreads;
@@ -243,12 +257,13 @@ cudaError_t launch_hint_tree(const int32_t* bank, int N, int eos, const int32_t*
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int grid = (int)(n_chunks < (long long)sms * 8 ? n_chunks : (long long)sms * 8);
-  k_hint_match<<<grid, kHintThreads, 0, st>>>(bank, N, eos, prefix, prefix_len, mlen, cmax, smax, best);
+  k_hint_match<<<grid, kHintThreads, 0, st>>>(bank, N, eos, prefix, prefix_len, prefix_len_dev, mlen, cmax, smax,
+                                              best);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   k_hint_pack<<<1, kHintThreads, 0, st>>>(bank, N, eos, prefix, prefix_len, mlen, cmax, smax, best, native,
-                                          native_len, n_native, native_stride, max_lanes, depth, max_nodes, out_tok,
-                                          out_par, out_T, out_info);
+                                          native_len, n_native, native_stride, max_lanes, depth, max_nodes,
+                                          prefix_len_dev, pad_to, out_tok, out_par, out_T, out_info);
   return cudaGetLastError();
 }
 
@@ -269,9 +284,9 @@ int oos_hint_tree(const int32_t* bank, int32_t bank_len, int32_t eos, const int3
   if (depth < 1 || depth > kMaxT || max_nodes < 1 || max_nodes > kMaxT) return OOS_EINVAL;
   if (!out_tokens || !out_parent || !out_T || !out_info) return OOS_EINVAL;
   if (!workspace || ((uintptr_t)workspace & 255) || ws_bytes < hint_workspace_bytes(bank_len)) return OOS_EWORKSPACE;
-  return launch_hint_tree(bank, bank_len, eos, prefix, prefix_len, native, native_len, n_native, native_stride,
-                          max_lanes, depth, max_nodes, workspace, out_tokens, out_parent, out_T, out_info,
-                          (cudaStream_t)stream) == cudaSuccess
+  return launch_hint_tree(bank, bank_len, eos, prefix, prefix_len, nullptr, native, native_len, n_native,
+                          native_stride, max_lanes, depth, max_nodes, 0, workspace, out_tokens, out_parent, out_T,
+                          out_info, (cudaStream_t)stream) == cudaSuccess
              ? OOS_OK
              : OOS_ECUDA;
 }

@@ -17,7 +17,6 @@ constexpr int kTile = 128;          // weight rows per MMA (tcgen05 M)
 constexpr int kWorkRowsWide = 256;  // weight rows per work tile of the gate/up GEMM and LM head
 constexpr int kBK = 64;             // reduction elements per pipeline stage (128 bytes of bf16)
 constexpr int kMaxLayers = 128;
-constexpr int kMaxAttnSplits = 8;   // key ranges per row block (one cluster, portable size)
 constexpr int kMaxGridCTAs = 1024;  // upper bound on CTAs of a stream-K GEMM / LM head
 constexpr int kMaxSsChunks = 64;    // hidden <= 8192: RMSNorm partial sums per 128 features
 constexpr int kCntPer = 256;        // arrival counters per (layer, GEMM kind): one per work tile
@@ -70,6 +69,7 @@ struct GemmW {
 
 struct Workspace {
   uint32_t* status;
+  int32_t* ctx;              // committed length of the current step (written by tree preparation)
   int32_t* depth;
   int32_t* pos;
   unsigned long long* anc;   // [kMaxT][2]
@@ -120,9 +120,8 @@ struct Model {
   std::vector<GemmW> g_qkv, g_o, g_gu, g_down;
   GemmW g_lm;
   CUtensorMap amap_xn[4], amap_attn[4], amap_act[4];  // per N-tile variant 16/32/64/128
-  CUtensorMap qmap_hi, qmap_lo;   // attention: q rows of one kv head, (d, head in group, kv head, node)
-  // attention: the last K/V cache maps encoded per layer (re-encoded only when
-  // the cache pointers or the valid extent change)
+  // attention: the K/V cache maps encoded per layer over the whole capacity
+  // (re-encoded only when the cache buffers change)
   struct KvMaps {
     const void* k = nullptr;
     const void* v = nullptr;
@@ -160,20 +159,21 @@ inline cudaError_t launch(bool pdl, void (*kernel)(KArgs...), dim3 grid, dim3 bl
 }
 
 // ---- small kernels (small.cu)
+// ctx from the host, or from device memory when ctx_dev is not null
 cudaError_t launch_tree_prep(Model& m, const int32_t* tokens, const int32_t* parent, int T, int ctx,
-                             cudaStream_t st);
+                             const int32_t* ctx_dev, cudaStream_t st);
 cudaError_t launch_embed_norm(Model& m, const int32_t* tokens, int T, cudaStream_t st);
 cudaError_t launch_embed_tc(Model& m, const int32_t* tokens, int T, cudaStream_t st);
 cudaError_t launch_final_hidden(Model& m, float* hidden, int T, cudaStream_t st);
-cudaError_t launch_qkv_post(Model& m, int layer, const StreamK& plan, void* kc, void* vc, int ctx, int T,
-                            cudaStream_t st);
+cudaError_t launch_qkv_post(Model& m, int layer, const StreamK& plan, void* kc, void* vc, int T, cudaStream_t st);
 cudaError_t launch_resid_norm(Model& m, const StreamK& plan, const void* gain, float* hidden_out, int T,
                               cudaStream_t st);
 cudaError_t launch_silu_mul(Model& m, const StreamK& plan, int T, cudaStream_t st);
-cudaError_t launch_argmax_accept(Model& m, const int32_t* tokens, const int32_t* parent, int T, int n_parts,
-                                 int32_t* len, int32_t* nodes, int32_t* toks, int32_t* bonus,
+// n_valid: DEVICE count of real nodes (the rest is padding, never accepted), or nullptr for T
+cudaError_t launch_argmax_accept(Model& m, const int32_t* tokens, const int32_t* parent, int T, const int32_t* n_valid,
+                                 int n_parts, int32_t* len, int32_t* nodes, int32_t* toks, int32_t* bonus,
                                  int32_t* dbg_argmax, float* dbg_top1, float* dbg_top2, cudaStream_t st);
-cudaError_t launch_kv_compact(Model& m, const oos_kv_cache& kv, int ctx, const int32_t* nodes,
+cudaError_t launch_kv_compact(Model& m, const oos_kv_cache& kv, int ctx, const int32_t* ctx_dev, const int32_t* nodes,
                               const int32_t* len, int max_len, cudaStream_t st);
 cudaError_t compact_setup();
 cudaError_t launch_accept_walk(const int32_t* tokens, const int32_t* parent, const int32_t* argmax, int T,
@@ -191,7 +191,7 @@ int bn_index(int T);   // N-tile variant for T tree nodes: 0..3 -> 16/32/64/128
 cudaError_t gemm_setup();
 // `next`: the weight GEMM that follows; its first stages are prefetched into L2
 // during this GEMM's tail (nullptr: none)
-cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int ctx, int T, const GemmW* next, cudaStream_t st);
+cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int T, const GemmW* next, cudaStream_t st);
 cudaError_t launch_gemm_o(Model& m, int layer, int T, const GemmW* next, cudaStream_t st);
 cudaError_t launch_gemm_gu(Model& m, int layer, int T, const GemmW* next, cudaStream_t st);
 cudaError_t launch_gemm_down(Model& m, int layer, int T, const GemmW* next, cudaStream_t st);
@@ -201,10 +201,33 @@ cudaError_t launch_gemm_f32(Model& m, const void* w0, const void* w1, const void
                             int rows2, int K, const void* x, int T, cudaStream_t st);
 cudaError_t launch_lm_head_f32(Model& m, int T, cudaStream_t st);
 
+// ---- verify step with the committed length and the count of real nodes in
+// device memory (oos_api.cu): tokens/parent hold T nodes of which *n_valid are
+// real (the rest is padding that is never accepted); ctx_dev may be anything
+// up to the cache capacity minus T
+int enqueue_verify_dev(Model& m, const oos_kv_cache* kv, const int32_t* ctx_dev, const int32_t* tokens,
+                       const int32_t* parent, int T, const int32_t* n_valid, int32_t* len, int32_t* nodes,
+                       int32_t* toks, int32_t* bonus, cudaStream_t st);
+
+// ---- hint-bank candidate step (hint.cu)
+size_t hint_workspace_bytes(long long bank_len);
+// prefix_len_dev: DEVICE prefix length (or nullptr for prefix_len); pad_to: write
+// padding nodes up to this count (0: none)
+cudaError_t launch_hint_tree(const int32_t* bank, int N, int eos, const int32_t* prefix, int prefix_len,
+                             const int32_t* prefix_len_dev, const int32_t* native, const int32_t* native_len,
+                             int n_native, int native_stride, int max_lanes, int depth, int max_nodes, int pad_to,
+                             void* ws, int32_t* out_tok, int32_t* out_par, int32_t* out_T, int32_t* out_info,
+                             cudaStream_t st);
+
 // ---- attention (attn.cu)
 cudaError_t attn_setup();
 int attn_nodes_per_block(int group);   // tree nodes per attention block (x group q heads <= 128 rows)
-bool attn_encode_q_maps(Model& m);     // TMA maps of the q buffer (bf16 path), at model creation
-cudaError_t launch_attention(Model& m, int layer, const void* kc, const void* vc, int ctx, int T, cudaStream_t st);
+// the step's ctx comes from the workspace; ctx here only sizes the key splits
+cudaError_t launch_attention(Model& m, int layer, const void* kc, const void* vc, int capacity, int ctx, int T,
+                             cudaStream_t st);
+int attn_splits(Model& m, int ctx_hint, int T);
 
 }  // namespace oos
+
+// the C handle of include/oos.h is the host-side model
+struct oos_model : public oos::Model {};

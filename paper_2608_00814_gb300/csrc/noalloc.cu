@@ -29,6 +29,9 @@ struct StaticScratch {
 };
 static __device__ __align__(256) StaticScratch g_argmax_scratch;
 
+// Merge of two running top-2 states.  Order independent for finite logits (and
+// infinities); a NaN logit compares false everywhere, so rows whose logits
+// contain NaN get a layout-dependent result.
 OOS_DEV StaticTop2 st_merge(StaticTop2 a, StaticTop2 b) {
   StaticTop2 r;
   if (a.v1 > b.v1 || (a.v1 == b.v1 && a.i1 <= b.i1)) {
@@ -45,7 +48,7 @@ OOS_DEV StaticTop2 st_merge(StaticTop2 a, StaticTop2 b) {
 // Block b scans vocabulary rows [b*rows, (b+1)*rows): warp w takes rows
 // w, w+4, ..., lanes stride over the hidden dimension; every row's logit for
 // each of the T hidden rows updates that warp's running top-2.  The last block
-// to finish merges all blocks' states (the merge is order independent).
+// to finish merges all blocks' states, in block order.
 template <typename E>
 __global__ void __launch_bounds__(128) k_lm_argmax_static(const E* __restrict__ W, int V, int H, int rows_per_block,
                                                           const float* __restrict__ hidden, int T, StaticScratch* sc,
@@ -54,6 +57,7 @@ __global__ void __launch_bounds__(128) k_lm_argmax_static(const E* __restrict__ 
   __shared__ int s_last;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   for (int t = lane; t < T; t += 32) st[warp][t] = StaticTop2{-INFINITY, 0x7fffffff, -INFINITY};
+  __syncwarp();   // lane 0 below reads states the other lanes initialised
   const int r_begin = blockIdx.x * rows_per_block;
   const int r_end = min(V, r_begin + rows_per_block);
   for (int r = r_begin + warp; r < r_end; r += 4) {
@@ -94,15 +98,22 @@ __global__ void __launch_bounds__(128) k_lm_argmax_static(const E* __restrict__ 
   if (threadIdx.x == 0) sc->arrived = 0;   // the next call starts from zero
 }
 
-// device address of the scratch array, looked up once per device
+// Device address of the scratch array.  In host code g_argmax_scratch names a
+// host-side stand-in, not device memory, so the kernel is given the address
+// cudaGetSymbolAddress returns for the current device.  Outside stream
+// capture it is looked up on every call (cheap, and right again after a
+// cudaDeviceReset reloads the module); a call made while its stream is being
+// captured uses the address cached by the last uncaptured call on the device.
 static std::mutex g_scratch_mu;
 static StaticScratch* g_scratch_ptr[64];
 
-static StaticScratch* scratch_for_current_device() {
+static StaticScratch* scratch_for_current_device(cudaStream_t st) {
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return nullptr;
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(st, &cs) != cudaSuccess) return nullptr;
   std::lock_guard<std::mutex> lock(g_scratch_mu);
-  if (!g_scratch_ptr[dev]) {
+  if (cs == cudaStreamCaptureStatusNone) {
     void* p = nullptr;
     if (cudaGetSymbolAddress(&p, g_argmax_scratch) != cudaSuccess) return nullptr;
     g_scratch_ptr[dev] = static_cast<StaticScratch*>(p);
@@ -121,11 +132,11 @@ extern "C" int oos_lm_head_argmax_static(int32_t dtype, int32_t vocab, int32_t h
   if (dtype != OOS_DTYPE_F32 && dtype != OOS_DTYPE_BF16) return OOS_EINVAL;
   if (vocab < 1 || hidden_dim < 1) return OOS_EINVAL;
   if (T < 1 || T > kStaticMaxT) return OOS_EINVAL;   // the scratch array holds kStaticMaxT rows
-  StaticScratch* sc = scratch_for_current_device();
+  cudaStream_t st = (cudaStream_t)stream;
+  StaticScratch* sc = scratch_for_current_device(st);
   if (!sc) return OOS_ECUDA;
   const int blocks = vocab < kStaticBlocks ? vocab : kStaticBlocks;
   const int rows = (vocab + blocks - 1) / blocks;
-  cudaStream_t st = (cudaStream_t)stream;
   if (dtype == OOS_DTYPE_BF16)
     k_lm_argmax_static<__nv_bfloat16><<<blocks, 128, 0, st>>>((const __nv_bfloat16*)lm_head, vocab, hidden_dim, rows,
                                                              hidden, T, sc, out_argmax, out_top1, out_top2);

@@ -12,8 +12,6 @@
 #include "common.cuh"
 #include "internal.h"
 
-struct oos_model : public oos::Model {};
-
 namespace oos {
 
 static size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
@@ -55,6 +53,7 @@ size_t carve_workspace(const oos_model_config& c, int n_sms, uint8_t* base, Work
   const size_t kvd = (size_t)c.n_kv_heads * c.head_dim;
   Workspace w;
   w.status = (uint32_t*)take(256);
+  w.ctx = (int32_t*)take(256);
   w.depth = (int32_t*)take(kMaxT * 4);
   w.pos = (int32_t*)take(kMaxT * 4);
   w.anc = (unsigned long long*)take(kMaxT * 16);
@@ -167,13 +166,16 @@ static unsigned long long kv_hash(const oos_kv_cache* kv) {
   } while (0)
 
 // tree prep, embedding and every decoder layer of a tree on stream st: the
-// K/V of the T nodes land in slots ctx.., the final-norm input in ws.x
-static int enqueue_layers(Model& m, const oos_kv_cache* kv, int ctx, const int32_t* tokens, const int32_t* parent,
-                          int T, float* hidden, cudaStream_t st) {
+// K/V of the T nodes land in slots ctx.., the final-norm input in ws.x.  The
+// committed length ctx comes from the host, or from device memory when ctx_dev
+// is not null (then any value up to the cache capacity is allowed).
+static int enqueue_layers(Model& m, const oos_kv_cache* kv, int ctx, const int32_t* ctx_dev, const int32_t* tokens,
+                          const int32_t* parent, int T, float* hidden, cudaStream_t st) {
   const auto& c = m.cfg;
   const int L = c.n_layers;
   const int qd = c.n_q_heads * c.head_dim, kvd = c.n_kv_heads * c.head_dim;
-  OOS_TRY(launch_tree_prep(m, tokens, parent, T, ctx, st));
+  const int ctx_hint = ctx_dev ? kv->capacity - T : ctx;   // sizes the attention's key splits
+  OOS_TRY(launch_tree_prep(m, tokens, parent, T, ctx, ctx_dev, st));
   if (c.dtype == OOS_DTYPE_BF16) OOS_TRY(launch_embed_tc(m, tokens, T, st));
   else OOS_TRY(launch_embed_norm(m, tokens, T, st));
   for (int l = 0; l < L; ++l) {
@@ -183,15 +185,15 @@ static int enqueue_layers(Model& m, const oos_kv_cache* kv, int ctx, const int32
     if (c.dtype == OOS_DTYPE_BF16) {
       // five kernels per layer; every elementwise step runs in a GEMM epilogue
       const GemmW* after_down = (l + 1 < L) ? &m.g_qkv[l + 1] : &m.g_lm;
-      OOS_TRY(launch_gemm_qkv(m, l, kv->k[l], kv->v[l], ctx, T, &m.g_o[l], st));
-      OOS_TRY(launch_attention(m, l, kv->k[l], kv->v[l], ctx, T, st));
+      OOS_TRY(launch_gemm_qkv(m, l, kv->k[l], kv->v[l], T, &m.g_o[l], st));
+      OOS_TRY(launch_attention(m, l, kv->k[l], kv->v[l], kv->capacity, ctx_hint, T, st));
       OOS_TRY(launch_gemm_o(m, l, T, &m.g_gu[l], st));
       OOS_TRY(launch_gemm_gu(m, l, T, &m.g_down[l], st));
       OOS_TRY(launch_gemm_down(m, l, T, after_down, st));
     } else {
       OOS_TRY(launch_gemm_f32(m, W.w_q, W.w_k, W.w_v, qd, kvd, kvd, c.hidden, m.ws.xn, T, st));
-      OOS_TRY(launch_qkv_post(m, l, m.p_qkv, kv->k[l], kv->v[l], ctx, T, st));
-      OOS_TRY(launch_attention(m, l, kv->k[l], kv->v[l], ctx, T, st));
+      OOS_TRY(launch_qkv_post(m, l, m.p_qkv, kv->k[l], kv->v[l], T, st));
+      OOS_TRY(launch_attention(m, l, kv->k[l], kv->v[l], kv->capacity, ctx_hint, T, st));
       OOS_TRY(launch_gemm_f32(m, W.w_o, nullptr, nullptr, c.hidden, 0, 0, qd, m.ws.attn, T, st));
       OOS_TRY(launch_resid_norm(m, m.p_o, W.mlp_norm, nullptr, T, st));
       OOS_TRY(launch_gemm_f32(m, W.w_gate, W.w_up, nullptr, c.intermediate, c.intermediate, 0, c.hidden, m.ws.xn, T,
@@ -204,12 +206,13 @@ static int enqueue_layers(Model& m, const oos_kv_cache* kv, int ctx, const int32
   return OOS_OK;
 }
 
-// the whole verify step on stream st
-static int enqueue_verify(Model& m, const oos_kv_cache* kv, int ctx, const int32_t* tokens, const int32_t* parent,
-                          int T, int32_t* len, int32_t* nodes, int32_t* toks, int32_t* bonus, float* hidden,
-                          int32_t* dbg_arg, float* dbg_t1, float* dbg_t2, cudaStream_t st) {
+// the whole verify step on stream st (ctx_dev, n_valid: see enqueue_verify_dev)
+static int enqueue_verify(Model& m, const oos_kv_cache* kv, int ctx, const int32_t* ctx_dev, const int32_t* tokens,
+                          const int32_t* parent, int T, const int32_t* n_valid, int32_t* len, int32_t* nodes,
+                          int32_t* toks, int32_t* bonus, float* hidden, int32_t* dbg_arg, float* dbg_t1,
+                          float* dbg_t2, cudaStream_t st) {
   const auto& c = m.cfg;
-  const int rc = enqueue_layers(m, kv, ctx, tokens, parent, T, hidden, st);
+  const int rc = enqueue_layers(m, kv, ctx, ctx_dev, tokens, parent, T, hidden, st);
   if (rc != OOS_OK) return rc;
   if (c.dtype == OOS_DTYPE_BF16) {
     if (hidden) OOS_TRY(launch_final_hidden(m, hidden, T, st));
@@ -217,8 +220,16 @@ static int enqueue_verify(Model& m, const oos_kv_cache* kv, int ctx, const int32
   } else {
     OOS_TRY(launch_lm_head_f32(m, T, st));
   }
-  OOS_TRY(launch_argmax_accept(m, tokens, parent, T, m.lm_grid, len, nodes, toks, bonus, dbg_arg, dbg_t1, dbg_t2, st));
+  OOS_TRY(launch_argmax_accept(m, tokens, parent, T, n_valid, m.lm_grid, len, nodes, toks, bonus, dbg_arg, dbg_t1,
+                               dbg_t2, st));
   return OOS_OK;
+}
+
+int enqueue_verify_dev(Model& m, const oos_kv_cache* kv, const int32_t* ctx_dev, const int32_t* tokens,
+                       const int32_t* parent, int T, const int32_t* n_valid, int32_t* len, int32_t* nodes,
+                       int32_t* toks, int32_t* bonus, cudaStream_t st) {
+  return enqueue_verify(m, kv, 0, ctx_dev, tokens, parent, T, n_valid, len, nodes, toks, bonus, nullptr, nullptr,
+                        nullptr, nullptr, st);
 }
 
 // Prefill: the prompt as chains of at most max_T tokens.  In a chain node j's
@@ -232,13 +243,13 @@ static int prefill_impl(Model& m, const oos_kv_cache* kv, int ctx, const int32_t
   int32_t* sc = m.ws.pf_scratch;
   for (int off = 0; off < n; off += c.max_T) {
     const int T = std::min(c.max_T, n - off);
-    const int rc = enqueue_layers(m, kv, ctx + off, tokens + off, m.ws.chain_parent, T, nullptr, st);
+    const int rc = enqueue_layers(m, kv, ctx + off, nullptr, tokens + off, m.ws.chain_parent, T, nullptr, st);
     if (rc != OOS_OK) return rc;
     if (off + T < n) continue;
     if (c.dtype == OOS_DTYPE_BF16) OOS_TRY(launch_lm_head_tc(m, T, st));
     else OOS_TRY(launch_lm_head_f32(m, T, st));
-    OOS_TRY(launch_argmax_accept(m, tokens + off, m.ws.chain_parent, T, m.lm_grid, sc, sc + 2, sc + 2 + kMaxT,
-                                 sc + 1, nullptr, nullptr, nullptr, st));
+    OOS_TRY(launch_argmax_accept(m, tokens + off, m.ws.chain_parent, T, nullptr, m.lm_grid, sc, sc + 2,
+                                 sc + 2 + kMaxT, sc + 1, nullptr, nullptr, nullptr, st));
     if (next_token) OOS_TRY(cudaMemcpyAsync(next_token, m.ws.argmax + (T - 1), 4, cudaMemcpyDeviceToDevice, st));
   }
   return OOS_OK;
@@ -256,7 +267,8 @@ static int verify_impl(oos_model* mp, const oos_kv_cache* kv, int32_t ctx, const
   if ((long long)ctx + T > kv->capacity) return OOS_ECAPACITY;
   cudaStream_t st = (cudaStream_t)stream;
   if (!m.cfg.use_graph)
-    return enqueue_verify(m, kv, ctx, tokens, parent, T, len, nodes, toks, bonus, hidden, dbg_arg, dbg_t1, dbg_t2, st);
+    return enqueue_verify(m, kv, ctx, nullptr, tokens, parent, T, nullptr, len, nodes, toks, bonus, hidden, dbg_arg,
+                          dbg_t1, dbg_t2, st);
   GraphKey key;
   key.kv_hash = kv_hash(kv);
   key.capacity = kv->capacity;
@@ -267,8 +279,8 @@ static int verify_impl(oos_model* mp, const oos_kv_cache* kv, int32_t ctx, const
   if (!(m.have_graph && key == m.gkey)) {
     cudaGraph_t graph = nullptr;
     OOS_TRY(cudaStreamBeginCapture(m.cap_stream, cudaStreamCaptureModeThreadLocal));
-    int rc = enqueue_verify(m, kv, ctx, tokens, parent, T, len, nodes, toks, bonus, hidden, dbg_arg, dbg_t1, dbg_t2,
-                            m.cap_stream);
+    int rc = enqueue_verify(m, kv, ctx, nullptr, tokens, parent, T, nullptr, len, nodes, toks, bonus, hidden, dbg_arg,
+                            dbg_t1, dbg_t2, m.cap_stream);
     cudaError_t ce = cudaStreamEndCapture(m.cap_stream, &graph);
     if (rc != OOS_OK || ce != cudaSuccess) {
       if (graph) cudaGraphDestroy(graph);
@@ -349,6 +361,11 @@ int oos_model_create(const oos_model_config* cfg, const oos_weights* w, void* wo
   int rc = OOS_OK;
   do {
     if (cudaMemset(workspace, 0, need) != cudaSuccess) { rc = OOS_ECUDA; break; }
+    const unsigned long long limit = kWaitLimitNs;
+    if (cudaMemcpy(m->ws.status + kStatusWaitLimit, &limit, sizeof(limit), cudaMemcpyHostToDevice) != cudaSuccess) {
+      rc = OOS_ECUDA;
+      break;
+    }
     std::vector<double> inv(c.head_dim / 2);
     for (int j = 0; j < c.head_dim / 2; ++j) inv[j] = pow((double)c.rope_theta, -2.0 * j / (double)c.head_dim);
     if (c.rope_factor > 1.f) rope_rescale(inv, c);
@@ -418,7 +435,6 @@ int oos_model_create(const oos_model_config* cfg, const oos_weights* w, void* wo
         ok = encode_act_map(&m->amap_xn[b], m->ws.xn, H, boxes[b]) &&
              encode_act_map(&m->amap_attn[b], m->ws.attn, qd, boxes[b]) &&
              encode_act_map(&m->amap_act[b], m->ws.act, I, boxes[b]);
-      ok = ok && attn_encode_q_maps(*m);
       if (!ok) {
         rc = OOS_ECUDA;
         break;
@@ -485,7 +501,8 @@ int oos_kv_compact(oos_model* m, const oos_kv_cache* kv, int32_t ctx_len, const 
     if (!kv->k[l] || !kv->v[l]) return OOS_EINVAL;
   if (ctx_len < 0 || max_len < 1 || max_len > kMaxT) return OOS_EINVAL;
   if ((long long)ctx_len + max_len > kv->capacity) return OOS_ECAPACITY;
-  if (launch_kv_compact(*m, *kv, ctx_len, accepted_nodes, accepted_len, max_len, (cudaStream_t)stream) != cudaSuccess)
+  if (launch_kv_compact(*m, *kv, ctx_len, nullptr, accepted_nodes, accepted_len, max_len, (cudaStream_t)stream) !=
+      cudaSuccess)
     return OOS_ECUDA;
   return OOS_OK;
 }
@@ -551,8 +568,24 @@ int oos_launch_attention(oos_model* m, const oos_kv_cache* kv, int32_t layer, in
   if (layer < 0 || layer >= m->cfg.n_layers || !kv->k[layer] || !kv->v[layer]) return OOS_EINVAL;
   if (T < 1 || T > m->cfg.max_T || ctx_len < 0) return OOS_EINVAL;
   if ((long long)ctx_len + T > kv->capacity) return OOS_ECAPACITY;
-  return launch_attention(*m, layer, kv->k[layer], kv->v[layer], ctx_len, T, (cudaStream_t)stream) == cudaSuccess ? OOS_OK
-                                                                                                        : OOS_ECUDA;
+  // the kernel reads the step's committed length from the workspace
+  cudaStream_t st = (cudaStream_t)stream;
+  const int32_t c32 = ctx_len;
+  if (cudaMemcpyAsync(m->ws.ctx, &c32, sizeof(c32), cudaMemcpyHostToDevice, st) != cudaSuccess) return OOS_ECUDA;
+  return launch_attention(*m, layer, kv->k[layer], kv->v[layer], kv->capacity, ctx_len, T, st) == cudaSuccess
+             ? OOS_OK
+             : OOS_ECUDA;
+}
+
+int oos_set_wait_limit(oos_model* m, uint64_t limit_ns, void* stream) {
+  if (!m) return OOS_EINVAL;
+  if (limit_ns == 0 || limit_ns > kWaitLimitNs) limit_ns = kWaitLimitNs;
+  const unsigned long long v = limit_ns;
+  cudaStream_t st = (cudaStream_t)stream;
+  if (cudaMemcpyAsync(m->ws.status + kStatusWaitLimit, &v, sizeof(v), cudaMemcpyHostToDevice, st) != cudaSuccess)
+    return OOS_ECUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return OOS_ECUDA;
+  return OOS_OK;
 }
 
 int oos_last_status(oos_model* m, void* stream) {

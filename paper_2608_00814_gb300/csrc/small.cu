@@ -12,15 +12,20 @@ namespace oos {
 // Tree encoding: parents-first numbering (parent[0] = -1, parent[i] < i).  Node
 // i attends to the committed cache and its ancestors (itself included); its
 // RoPE position is ctx + depth(i).  Ancestor sets are 128-bit masks.
+// ctx: the committed length, from the host (ctx_in == nullptr) or from device
+// memory; written to ctx_out, where every later kernel of the step reads it.
 __global__ void __launch_bounds__(kMaxT) k_tree_prep(const int32_t* __restrict__ tokens,
                                                      const int32_t* __restrict__ parent, int T, int ctx,
+                                                     const int32_t* __restrict__ ctx_in, int32_t* ctx_out,
                                                      int vocab, uint32_t* status, int32_t* depth_out,
                                                      int32_t* pos_out, unsigned long long* anc_out) {
   __shared__ int s_parent[kMaxT];
   __shared__ int s_bad;
-  pdl_trigger();
   pdl_wait();
+  pdl_trigger();
+  if (ctx_in) ctx = *ctx_in;
   const int i = threadIdx.x;
+  if (i == 0) *ctx_out = ctx;
   if (i == 0) s_bad = 0;
   __syncthreads();
   if (i < T) {
@@ -53,12 +58,15 @@ __global__ void __launch_bounds__(kMaxT) k_tree_prep(const int32_t* __restrict__
 
 // The first kernel of a step is launched without programmatic serialisation:
 // it starts only after all earlier work on the stream (the previous step's
-// compaction, the caller's cache writes) has completed, so later kernels of
-// the step may read cache positions < ctx before their own dependency wait.
+// compaction, the caller's cache writes) has completed.  Every kernel of the
+// step lets its dependents launch only after its own dependency wait, so a
+// kernel that starts finds the kernel two launches back, and all before it,
+// complete: later kernels may read cache positions < ctx, and ctx itself,
+// before their own dependency wait.
 cudaError_t launch_tree_prep(Model& m, const int32_t* tokens, const int32_t* parent, int T, int ctx,
-                             cudaStream_t st) {
-  return launch(false, k_tree_prep, dim3(1), dim3(kMaxT), 0, st, tokens, parent, T, ctx, m.cfg.vocab,
-                m.ws.status, m.ws.depth, m.ws.pos, m.ws.anc);
+                             const int32_t* ctx_dev, cudaStream_t st) {
+  return launch(false, k_tree_prep, dim3(1), dim3(kMaxT), 0, st, tokens, parent, T, ctx, ctx_dev, m.ws.ctx,
+                m.cfg.vocab, m.ws.status, m.ws.depth, m.ws.pos, m.ws.anc);
 }
 
 // ============================================================ embedding + first RMSNorm
@@ -68,8 +76,8 @@ __global__ void __launch_bounds__(256) k_embed_norm(const int32_t* __restrict__ 
                                                     const E* __restrict__ gain, int H, int vocab, float eps,
                                                     float* __restrict__ x, E* __restrict__ xn) {
   __shared__ float red[32];
-  pdl_trigger();
   pdl_wait();
+  pdl_trigger();
   const int t = blockIdx.x;
   int tok = tokens[t];
   tok = tok < 0 ? 0 : (tok >= vocab ? vocab - 1 : tok);   // invalid trees are flagged by tree_prep
@@ -110,8 +118,8 @@ __global__ void __launch_bounds__(128) k_embed_tc(const int32_t* __restrict__ to
                                                   const double* __restrict__ inv_freq, int half_d,
                                                   float2* __restrict__ rope, int* __restrict__ cnt, int n_cnt) {
   __shared__ float red[32];
-  pdl_trigger();
   pdl_wait();
+  pdl_trigger();
   const int t = blockIdx.x, f = blockIdx.y * 128 + threadIdx.x;
   {   // the step's GEMM arrival counters start from zero
     const int nb = gridDim.x * gridDim.y, b = blockIdx.y * gridDim.x + blockIdx.x;
@@ -149,8 +157,8 @@ cudaError_t launch_embed_tc(Model& m, const int32_t* tokens, int T, cudaStream_t
 __global__ void __launch_bounds__(256) k_final_hidden(const float* __restrict__ x, const float* __restrict__ ss,
                                                       int chunks, const __nv_bfloat16* __restrict__ gain, int H,
                                                       float eps, float* __restrict__ hidden) {
-  pdl_trigger();
   pdl_wait();
+  pdl_trigger();
   const int t = blockIdx.x;
   float s = 0.f;
   for (int c = 0; c < chunks; ++c) s += ss[(size_t)c * kMaxT + t];
@@ -194,14 +202,14 @@ struct QkvPostArgs {
   void* q;
   void* kc;
   void* vc;
-  int ctx;
+  const int32_t* ctx;   // committed length of the step (device)
 };
 
 template <typename E>
 __global__ void k_qkv_post(QkvPostArgs a) {
   __shared__ float red[32];
-  pdl_trigger();
   pdl_wait();
+  pdl_trigger();
   const int t = blockIdx.x, hs = blockIdx.y, j = threadIdx.x, half = a.d / 2;
   const int f0 = hs * a.d + j, f1 = f0 + half;
   float v0 = gather_partial(a.part, a.plan, a.N, t, f0);
@@ -236,13 +244,12 @@ __global__ void k_qkv_post(QkvPostArgs a) {
   }
   E* dst;
   if (kind == 0) dst = (E*)a.q + ((size_t)t * a.nq + h) * a.d;
-  else dst = (E*)(kind == 1 ? a.kc : a.vc) + ((size_t)(a.ctx + t) * a.nkv + h) * a.d;
+  else dst = (E*)(kind == 1 ? a.kc : a.vc) + ((size_t)(*a.ctx + t) * a.nkv + h) * a.d;
   dst[j] = from_f32<E>(v0);
   dst[j + half] = from_f32<E>(v1);
 }
 
-cudaError_t launch_qkv_post(Model& m, int layer, const StreamK& plan, void* kc, void* vc, int ctx, int T,
-                            cudaStream_t st) {
+cudaError_t launch_qkv_post(Model& m, int layer, const StreamK& plan, void* kc, void* vc, int T, cudaStream_t st) {
   const auto& c = m.cfg;
   const auto& L = m.layers[layer];
   QkvPostArgs a;
@@ -263,7 +270,7 @@ cudaError_t launch_qkv_post(Model& m, int layer, const StreamK& plan, void* kc, 
   a.q = m.ws.q;
   a.kc = kc;
   a.vc = vc;
-  a.ctx = ctx;
+  a.ctx = m.ws.ctx;
   dim3 grid(T, c.n_q_heads + 2 * c.n_kv_heads);
   if (c.dtype == OOS_DTYPE_BF16) return launch(m.pdl, k_qkv_post<__nv_bfloat16>, grid, dim3(c.head_dim / 2), 0, st, a);
   return launch(m.pdl, k_qkv_post<float>, grid, dim3(c.head_dim / 2), 0, st, a);
@@ -278,8 +285,8 @@ __global__ void __launch_bounds__(256) k_resid_norm(const float* __restrict__ pa
                                                     const E* __restrict__ gain, float eps, float* __restrict__ x,
                                                     E* __restrict__ xn, float* __restrict__ hidden_out) {
   __shared__ float red[32];
-  pdl_trigger();
   pdl_wait();
+  pdl_trigger();
   const int t = blockIdx.x;
   float* xr = x + (size_t)t * H;
   float ss = 0.f;
@@ -312,8 +319,8 @@ cudaError_t launch_resid_norm(Model& m, const StreamK& plan, const void* gain, f
 template <typename E>
 __global__ void __launch_bounds__(256) k_silu_mul(const float* __restrict__ part, StreamK plan, int I,
                                                   E* __restrict__ act) {
-  pdl_trigger();
   pdl_wait();
+  pdl_trigger();
   const int t = blockIdx.y;
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i < I) {
@@ -357,9 +364,10 @@ OOS_DEV Top2 top2_merge(Top2 a, Top2 b) {
 // Greedy longest-prefix acceptance (Eq. 1; "Verify and commit") by one warp.
 // ok(0) = 1; ok(i) = ok(parent) and token_i == argmax(parent).  The committed
 // path ends at the deepest ok node (lowest id on ties); bonus = its argmax.
+// Nodes at or past n_valid are padding of a fixed-size tree and never ok.
 OOS_DEV void accept_walk_warp(const int32_t* tokens, const int32_t* parent, const int32_t* depth,
-                              const int32_t* argmax, int T, bool bad, int32_t* len_out, int32_t* nodes_out,
-                              int32_t* toks_out, int32_t* bonus_out) {
+                              const int32_t* argmax, int T, int n_valid, bool bad, int32_t* len_out,
+                              int32_t* nodes_out, int32_t* toks_out, int32_t* bonus_out) {
   const int lane = threadIdx.x & 31;
   if (bad) {
     for (int i = lane; i < T; i += 32) {
@@ -374,8 +382,8 @@ OOS_DEV void accept_walk_warp(const int32_t* tokens, const int32_t* parent, cons
   }
   int best_key = 0x7fffffff;  // key = (kMaxT - depth) * 256 + node: min = deepest, then lowest id
   for (int i = lane; i < T; i += 32) {
-    bool ok = true;
-    for (int a = i; a != 0; a = parent[a]) {
+    bool ok = i < n_valid;
+    for (int a = i; ok && a != 0; a = parent[a]) {
       const int p = parent[a];
       if (tokens[a] != argmax[p]) {
         ok = false;
@@ -413,12 +421,13 @@ __global__ void __launch_bounds__(1024) k_argmax_accept(const float* __restrict_
                                                          const int32_t* __restrict__ tokens,
                                                          const int32_t* __restrict__ parent,
                                                          const int32_t* __restrict__ depth, const uint32_t* status,
-                                                         int T, int32_t* argmax_ws, float* top1_ws, float* top2_ws,
+                                                         int T, const int32_t* __restrict__ n_valid_dev,
+                                                         int32_t* argmax_ws, float* top1_ws, float* top2_ws,
                                                          int32_t* len, int32_t* nodes, int32_t* toks, int32_t* bonus,
                                                          int32_t* dbg_argmax, float* dbg_top1, float* dbg_top2) {
   __shared__ int32_t s_tok[kMaxT], s_par[kMaxT], s_dep[kMaxT], s_arg[kMaxT];
-  pdl_trigger();
   pdl_wait();
+  pdl_trigger();
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, nw = blockDim.x >> 5;
   // one warp per node (32 warps); the merge is order independent (max with
   // lowest-id ties, multiset second max), so lanes take CTA states in any order
@@ -452,17 +461,20 @@ __global__ void __launch_bounds__(1024) k_argmax_accept(const float* __restrict_
     s_dep[i] = depth[i];
   }
   __syncthreads();
-  if (threadIdx.x < 32)
-    accept_walk_warp(s_tok, s_par, s_dep, s_arg, T, (*status & ST_TREE) != 0, len, nodes, toks, bonus);
+  if (threadIdx.x < 32) {
+    int n_valid = n_valid_dev ? *n_valid_dev : T;
+    n_valid = n_valid < 1 ? 1 : (n_valid > T ? T : n_valid);
+    accept_walk_warp(s_tok, s_par, s_dep, s_arg, T, n_valid, (*status & ST_TREE) != 0, len, nodes, toks, bonus);
+  }
 }
 
-cudaError_t launch_argmax_accept(Model& m, const int32_t* tokens, const int32_t* parent, int T, int n_parts,
-                                 int32_t* len, int32_t* nodes, int32_t* toks, int32_t* bonus, int32_t* dbg_argmax,
-                                 float* dbg_top1, float* dbg_top2, cudaStream_t st) {
+cudaError_t launch_argmax_accept(Model& m, const int32_t* tokens, const int32_t* parent, int T, const int32_t* n_valid,
+                                 int n_parts, int32_t* len, int32_t* nodes, int32_t* toks, int32_t* bonus,
+                                 int32_t* dbg_argmax, float* dbg_top1, float* dbg_top2, cudaStream_t st) {
   return launch(m.pdl, k_argmax_accept, dim3(1), dim3(1024), 0, st, (const float*)m.ws.lm_v1,
                 (const int32_t*)m.ws.lm_i, (const float*)m.ws.lm_v2, n_parts, tokens, parent,
-                (const int32_t*)m.ws.depth, (const uint32_t*)m.ws.status, T, m.ws.argmax, m.ws.top1, m.ws.top2,
-                len, nodes, toks, bonus, dbg_argmax, dbg_top1, dbg_top2);
+                (const int32_t*)m.ws.depth, (const uint32_t*)m.ws.status, T, n_valid, m.ws.argmax, m.ws.top1,
+                m.ws.top2, len, nodes, toks, bonus, dbg_argmax, dbg_top1, dbg_top2);
 }
 
 // standalone walk: validates the tree itself
@@ -488,7 +500,7 @@ __global__ void k_accept_walk(const int32_t* tokens, const int32_t* parent, cons
     s_dep[i] = d;
   }
   __syncthreads();
-  if (i < 32) accept_walk_warp(s_tok, s_par, s_dep, s_arg, T, s_bad != 0, len, nodes, toks, bonus);
+  if (i < 32) accept_walk_warp(s_tok, s_par, s_dep, s_arg, T, T, s_bad != 0, len, nodes, toks, bonus);
   if (i == 0) *status = s_bad ? OOS_ETREE : OOS_OK;
 }
 
@@ -510,12 +522,13 @@ struct KvPtrs {
 };
 
 template <typename E>
-__global__ void k_kv_compact(KvPtrs p, int nkv, int d, int ctx, const int32_t* __restrict__ nodes,
-                             const int32_t* __restrict__ len_ptr, int max_len) {
+__global__ void k_kv_compact(KvPtrs p, int nkv, int d, int ctx, const int32_t* __restrict__ ctx_dev,
+                             const int32_t* __restrict__ nodes, const int32_t* __restrict__ len_ptr, int max_len) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   E* buf = reinterpret_cast<E*>(smem_raw);
-  pdl_trigger();
   pdl_wait();
+  pdl_trigger();
+  if (ctx_dev) ctx = *ctx_dev;
   const int layer = blockIdx.x, which = blockIdx.y, g = blockIdx.z;
   E* base = (E*)(which == 0 ? p.k[layer] : p.v[layer]);
   int len = *len_ptr;
@@ -541,8 +554,8 @@ cudaError_t compact_setup() {
                               kMaxT * 128 * 2);
 }
 
-cudaError_t launch_kv_compact(Model& m, const oos_kv_cache& kv, int ctx, const int32_t* nodes, const int32_t* len,
-                              int max_len, cudaStream_t st) {
+cudaError_t launch_kv_compact(Model& m, const oos_kv_cache& kv, int ctx, const int32_t* ctx_dev, const int32_t* nodes,
+                              const int32_t* len, int max_len, cudaStream_t st) {
   const auto& c = m.cfg;
   KvPtrs p;
   for (int l = 0; l < c.n_layers; ++l) {
@@ -553,9 +566,9 @@ cudaError_t launch_kv_compact(Model& m, const oos_kv_cache& kv, int ctx, const i
   const size_t smem = (size_t)max_len * c.head_dim * m.esize;
   if (c.dtype == OOS_DTYPE_BF16)
     return launch(m.pdl, k_kv_compact<__nv_bfloat16>, grid, dim3(256), smem, st, p, c.n_kv_heads, c.head_dim, ctx,
-                  nodes, len, max_len);
-  return launch(m.pdl, k_kv_compact<float>, grid, dim3(256), smem, st, p, c.n_kv_heads, c.head_dim, ctx, nodes, len,
-                max_len);
+                  ctx_dev, nodes, len, max_len);
+  return launch(m.pdl, k_kv_compact<float>, grid, dim3(256), smem, st, p, c.n_kv_heads, c.head_dim, ctx, ctx_dev,
+                nodes, len, max_len);
 }
 
 }  // namespace oos

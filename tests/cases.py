@@ -71,7 +71,7 @@ def root_token(cfg, seed):
 
 
 def build_case(name="tiny", seed=0, T=None, recipe=None, plant=None, ctx_len=None,
-               cfg_overrides=None, gain_std=0.0, planted=None, prefill=None, root=None):
+               cfg_overrides=None, gain_std=0.0, planted=None, prefill=None, root=None, tree_key=None):
     """A verify-step case for workload `name` (defaults from its recipe)."""
     w = workload(name)
     cfg = w.model if not cfg_overrides else dataclasses.replace(w.model, **cfg_overrides)
@@ -94,14 +94,34 @@ def build_case(name="tiny", seed=0, T=None, recipe=None, plant=None, ctx_len=Non
             planted, margins = [], []
     else:
         planted, margins = planted
-    tokens, parent, path = trees.make_tree(recipe, T, root, planted, cfg.vocab,
-                                           gen.tensor_key(seed, TREE_SHAPE, T))
+    if tree_key is None:
+        tree_key = gen.tensor_key(seed, TREE_SHAPE, T)
+    tokens, parent, path = trees.make_tree(recipe, T, root, planted, cfg.vocab, tree_key)
     return Case(cfg, model, view, ctx_len, native, k64, v64, tokens, parent, path,
                 list(margins))
+
+
+def with_tree(case, name, root, planted, margins, index):
+    """The same model and cache with another tree: the workload's recipe
+    around root -> planted path, shape drawn from stream `index`."""
+    w = workload(name)
+    T = len(case.tokens)
+    tokens, parent, path = trees.make_tree(w.tree, T, int(root), list(planted), case.cfg.vocab,
+                                           gen.tensor_key(1000 + int(index), TREE_SHAPE, T))
+    return dataclasses.replace(case, tokens=tokens, parent=parent, planted_path=path,
+                               planted_margins=list(margins))
 
 
 def load_planted(name):
     """Planted greedy paths written by golden/make_planted.py (oracle only)."""
     with open(os.path.join(GOLDEN, "planted.json")) as f:
+        d = json.load(f)
+    return d[name]
+
+
+def load_gated_roots(name):
+    """Well-separated roots and their greedy paths, written by
+    golden/make_planted.py --roots (oracle only)."""
+    with open(os.path.join(GOLDEN, "gated_roots.json")) as f:
         d = json.load(f)
     return d[name]

@@ -10,6 +10,14 @@ near-tie could be decided either way by a bf16 verifier, so exact comparison of
 the accept outputs is only meaningful on such well-separated paths.
 
 Usage: python tests/golden/make_planted.py [workload ...]
+       python tests/golden/make_planted.py --roots N workload ...
+
+The second form writes golden/gated_roots.json instead: for each workload,
+the first N roots of the seeded ROOT stream (weights seed 0, the workload's
+own committed cache: a real prefill for the prefilled test models, the
+synthetic cache otherwise) whose greedy continuation of `plant` tokens and
+the bonus is well separated.  Every such root gives the GPU parity tests one
+gated case: a tree around that path whose accept outputs must match exactly.
 """
 
 import json
@@ -25,14 +33,34 @@ sys.path.insert(0, ROOT)
 sys.path.insert(0, os.path.dirname(HERE))
 
 import oracle  # noqa: E402
-from cases import synthetic_cache  # noqa: E402
+from cases import synthetic_cache, tiny_cache  # noqa: E402
 from synth import gen  # noqa: E402
-from synth.configs import WORKLOADS  # noqa: E402
+from synth.configs import WORKLOADS, workload  # noqa: E402
 from synth.model import ROOT as ROOT_KIND, SynthModel  # noqa: E402
 
 OUT = os.environ.get("PLANTED_OUT") or os.path.join(HERE, "planted.json")   # override: write elsewhere
+ROOTS_OUT = os.environ.get("GATED_ROOTS_OUT") or os.path.join(HERE, "gated_roots.json")
 MIN_MARGIN = 0.06       # the tests gate at 0.05
 MAX_ROOTS = 64
+
+
+def _separated_path(view, k64, v64, ctx_len, root, plant):
+    """Greedy decisions after `root` until plant + 1 are found or one is a
+    near-tie: (tokens, margins); complete when len(tokens) == plant + 1."""
+    ck = [np.array(c) for c in k64]
+    cv = [np.array(c) for c in v64]
+    n_pos, tok, toks, margins = ctx_len, root, [], []
+    while len(toks) < plant + 1:
+        _, a, t1, t2, ks, vs = oracle.decode_step(view, ck, cv, n_pos, tok)
+        margins.append(t1 - t2)
+        if t1 - t2 <= MIN_MARGIN:
+            break
+        toks.append(a)
+        ck = [np.concatenate([c, x[None]]) for c, x in zip(ck, ks)]
+        cv = [np.concatenate([c, x[None]]) for c, x in zip(cv, vs)]
+        n_pos += 1
+        tok = a
+    return toks, margins
 
 
 def plant_one(name, seed=0):
@@ -43,19 +71,7 @@ def plant_one(name, seed=0):
     roots = gen.uniform_int(gen.tensor_key(seed, ROOT_KIND), MAX_ROOTS, cfg.vocab)
     for k in range(MAX_ROOTS):
         root = int(roots[k])
-        ck = [np.array(c) for c in k64]
-        cv = [np.array(c) for c in v64]
-        n_pos, tok, toks, margins = w.ctx_len, root, [], []
-        while len(toks) < w.plant + 1:
-            _, a, t1, t2, ks, vs = oracle.decode_step(view, ck, cv, n_pos, tok)
-            margins.append(t1 - t2)
-            if t1 - t2 <= MIN_MARGIN:
-                break
-            toks.append(a)
-            ck = [np.concatenate([c, x[None]]) for c, x in zip(ck, ks)]
-            cv = [np.concatenate([c, x[None]]) for c, x in zip(cv, vs)]
-            n_pos += 1
-            tok = a
+        toks, margins = _separated_path(view, k64, v64, w.ctx_len, root, w.plant)
         print("  %s root #%d: %d/%d decisions above margin" % (name, k, len(toks), w.plant + 1), flush=True)
         if len(toks) == w.plant + 1:
             return dict(seed=seed, ctx_len=w.ctx_len, root_index=k, root=root, planted=toks[:w.plant],
@@ -63,6 +79,33 @@ def plant_one(name, seed=0):
                         note="oracle greedy continuation after the root on the synthetic cache; every margin "
                              "> %.2f" % MIN_MARGIN)
     raise RuntimeError("no well-separated greedy path found for %s" % name)
+
+
+def gated_roots(name, n_cases, seed=0, max_roots=1024):
+    """The first n_cases roots of the seeded ROOT stream whose greedy path
+    (plant tokens and the bonus) is well separated."""
+    w = workload(name)
+    cfg = w.model
+    model = SynthModel(cfg, seed)
+    view = model.oracle_view()
+    if w.prefill:
+        _, k64, v64 = tiny_cache(cfg, model, view, seed, w.ctx_len)
+    else:
+        _, k64, v64 = synthetic_cache(cfg, seed, w.ctx_len)
+    roots = gen.uniform_int(gen.tensor_key(seed, ROOT_KIND), max_roots, cfg.vocab)
+    found = []
+    for k in range(max_roots):
+        root = int(roots[k])
+        toks, margins = _separated_path(view, k64, v64, w.ctx_len, root, w.plant)
+        if len(toks) == w.plant + 1:
+            found.append(dict(root_index=k, root=root, planted=toks[:w.plant], bonus=toks[w.plant],
+                              margins=margins))
+            print("  %s root #%d kept (%d so far)" % (name, k, len(found)), flush=True)
+            if len(found) == n_cases:
+                return dict(seed=seed, ctx_len=w.ctx_len, plant=w.plant, cases=found,
+                            note="roots of the seeded stream whose oracle greedy continuation (plant tokens and "
+                                 "the bonus) has every top-1/top-2 margin > %.2f" % MIN_MARGIN)
+    raise RuntimeError("only %d well-separated roots for %s" % (len(found), name))
 
 
 def main(names):
@@ -79,5 +122,21 @@ def main(names):
             json.dump(data, f, indent=1)
 
 
+def main_roots(n_cases, names):
+    data = {}
+    if os.path.exists(ROOTS_OUT):
+        with open(ROOTS_OUT) as f:
+            data = json.load(f)
+    for name in names:
+        t0 = time.time()
+        data[name] = gated_roots(name, n_cases)
+        print(name, "%d roots" % n_cases, "%.0fs" % (time.time() - t0), flush=True)
+        with open(ROOTS_OUT, "w") as f:
+            json.dump(data, f, indent=1)
+
+
 if __name__ == "__main__":
-    main(sys.argv[1:] or [n for n, w in WORKLOADS.items() if w.model.dtype == "bf16"])
+    if len(sys.argv) > 2 and sys.argv[1] == "--roots":
+        main_roots(int(sys.argv[2]), sys.argv[3:])
+    else:
+        main(sys.argv[1:] or [n for n, w in WORKLOADS.items() if w.model.dtype == "bf16"])

@@ -8,7 +8,7 @@ import pytest
 import torch
 
 import oracle
-from cases import GOLDEN, build_case, load_planted
+from cases import GOLDEN, build_case, load_gated_roots, load_planted, with_tree
 from gpu_util import (GATE, TOL, check_case, check_compaction, gpu_cache, gpu_model, max_rel_err, ok_nodes, run,
                       to_f64)
 from synth import trees
@@ -237,6 +237,8 @@ def _mini(mini_models, seed, **kw):
 
 
 def test_mini_bf16_parity_seeds(mini_models):
+    """Random weight seeds: every tensor at tolerance, accept outputs exact
+    wherever the margin gate holds."""
     gated = 0
     for seed in range(6):
         case, model = _mini(mini_models, seed)
@@ -245,6 +247,42 @@ def test_mini_bf16_parity_seeds(mini_models):
         gated += check_case(case, g, _oracle(case))
         check_compaction(model, kv, case.ctx_len, g)
     assert gated >= 1
+
+
+def _gated_roots_sweep(name, base, model, min_gated):
+    """One case per stored well-separated root (golden/gated_roots.json):
+    the workload's tree recipe around root -> greedy path, every node checked
+    against the full oracle step; counts the cases whose accept outputs were
+    compared exactly (the margin gate)."""
+    roots = load_gated_roots(name)
+    gated, n = 0, 0
+    for k, e in enumerate(roots["cases"]):
+        case = with_tree(base, name, e["root"], e["planted"], e["margins"], e["root_index"])
+        kv = gpu_cache(case, case.ctx_len + len(case.tokens))
+        g = run(model, kv, case.ctx_len, case.tokens, case.parent)
+        r = _oracle(case)
+        ok = check_case(case, g, r)
+        check_compaction(model, kv, case.ctx_len, g)
+        if ok:
+            assert g["accepted_len"] >= len(case.planted_path)
+        gated += ok
+        n += 1
+    print("%s: %d of %d bf16 cases gated (accept outputs compared exactly)" % (name, gated, n))
+    assert gated >= min_gated, "%s: only %d of %d cases passed the margin gate" % (name, gated, n)
+
+
+def test_mini_bf16_gated_roots(mini_models):
+    base, model = _mini(mini_models, 0)
+    _gated_roots_sweep("mini-bf16", base, model, 20)
+
+
+def test_bf16_qwen3_06b_gated_roots():
+    """Full-size Qwen3-0.6B shape: 24 trees around well-separated greedy paths,
+    every node of every tree against the full oracle step."""
+    p = load_planted("qwen3-0.6b")
+    base = build_case("qwen3-0.6b", p["seed"], planted=(p["planted"], p["margins"]), root=p["root"])
+    model, _ = gpu_model(base)
+    _gated_roots_sweep("qwen3-0.6b", base, model, 20)
 
 
 @pytest.mark.parametrize("T,recipe,ctx", [
@@ -283,9 +321,10 @@ def _bf16_case(name, T=None, ctx=None):
     return build_case(name, p["seed"], planted=(p["planted"], p["margins"]), T=T, ctx_len=ctx, root=p["root"])
 
 
-@pytest.mark.parametrize("name", ["qwen3-0.6b"])
+@pytest.mark.parametrize("name", ["qwen3-0.6b", "qwen3-8b"])
 def test_bf16_full_size_every_node(name):
-    """Full-size parity: every node, every layer, at the workload's shape."""
+    """Full-size parity: every node, every layer, at the workload's shape
+    (qwen3-8b: the benchmark's own workload, T=64 over 2048 cached positions)."""
     case = _bf16_case(name)
     model, _ = gpu_model(case)
     kv = gpu_cache(case, case.ctx_len + case.tokens.shape[0])
