@@ -31,7 +31,7 @@ import numpy as np  # noqa: E402
 
 from synth import gen, trees  # noqa: E402
 from synth.configs import WORKLOADS  # noqa: E402
-from synth.model import TREE_SHAPE, SynthModel, synthetic_kv  # noqa: E402
+from synth.model import ROOT as ROOT_KIND, TREE_SHAPE, SynthModel, synthetic_kv  # noqa: E402
 
 METRIC = "tree-verify step µs and tree tokens/s at 1 GB300; achieved HBM GB/s vs ~8 TB/s"
 UNIT = "tree tokens/s"
@@ -49,7 +49,9 @@ def workload_tree(name):
     w = WORKLOADS[name]
     cfg = w.model
     with open(PLANTED) as f:
-        p = json.load(f)[name]
+        p = json.load(f).get(name)
+    if p is None:   # no planted path for this shape yet: the tree's tokens are all random
+        p = dict(seed=0, root=int(gen.uniform_int(gen.tensor_key(0, ROOT_KIND), 1, cfg.vocab)[0]), planted=[])
     seed, root = p["seed"], p["root"]
     tokens, parent, path = trees.make_tree(w.tree, w.T, root, p["planted"], cfg.vocab,
                                            gen.tensor_key(seed, TREE_SHAPE, w.T))
@@ -220,6 +222,79 @@ def reduce_step_time(ms, world, dist=None, device="cuda"):
 def job_throughput(T, ms, world):
     """Tree tokens verified per second by all ranks together."""
     return world * T / (ms * 1e-3)
+
+
+# ---------------------------------------------------------------- decode loop
+
+def decode_leg(B, cfg, weights, native_cache, T, stream, n_vanilla=96, n_rounds=12, eos=2):
+    """Committed tokens/s of the device decode loop and of vanilla decoding."""
+    import torch
+    from synth.device import upload_cache
+    seed, ctx = native_cache
+    cap = ctx + max(n_vanilla * T, n_rounds * T) + 8   # the plain T-node run below commits one token per T slots
+    native = [(synthetic_kv(cfg, seed, l, ctx, "native", "k"), synthetic_kv(cfg, seed, l, ctx, "native", "v"))
+              for l in range(cfg.n_layers)]
+    k, v = upload_cache(cfg, native, cap)
+    del native
+    kv = B.KVCache(k, v)
+    # the planted root: its first greedy decisions are well separated (golden/planted.json)
+    with open(PLANTED) as f:
+        p = json.load(f).get(cfg.name)
+    root = int(p["root"]) if p else int(gen.uniform_int(gen.tensor_key(seed, ROOT_KIND), 1, cfg.vocab)[0])
+    state = torch.zeros(3, dtype=torch.int32, device="cuda")
+
+    def run(model, bank, max_nodes, rounds, depth=16, lanes=8):
+        committed = torch.zeros(1 + rounds * max_nodes, dtype=torch.int32, device="cuda")
+        committed[0] = root
+        mat = torch.zeros(rounds, dtype=torch.int32, device="cuda")
+        ws = torch.empty(B.oos_decode_workspace_bytes(int(bank.numel())) + 256, dtype=torch.uint8, device="cuda")
+        wsa = ws[(-ws.data_ptr()) % 256:]
+        B.oos_decode(model, kv, ctx, committed, 1, bank, eos, lanes, depth, max_nodes, rounds, mat, state, wsa,
+                     stream)   # warm (capture, first touch)
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        B.oos_decode(model, kv, ctx, committed, 1, bank, eos, lanes, depth, max_nodes, rounds, mat, state, wsa,
+                     stream)
+        b.record(stream)
+        torch.cuda.synchronize()
+        if B.oos_last_status(model) != B.OOS_OK:
+            raise RuntimeError("decode status %s" % B.oos_status_string(B.oos_last_status(model)))
+        n_tok = int(state[1].item()) - 1
+        return committed[1:1 + n_tok].cpu().tolist(), mat.cpu().tolist(), a.elapsed_time(b) * 1e-3
+
+    # vanilla: a bank of EOS only never matches, so every tree is the root alone (T = 1)
+    eos_bank = torch.full((64,), eos, dtype=torch.int32, device="cuda")
+    m1 = B.OosModel(cfg, weights, max_T=1, use_graph=True)
+    van_toks, van_mat, van_s = run(m1, eos_bank, 1, n_vanilla)
+    m1.close()
+    # the continuation the bank is built from: the same loop on trees of T nodes
+    # holding the root alone, so that it is computed by the kernels the
+    # speculative run uses (a random-init model has near-tied greedy decisions,
+    # which a different tree size can decide the other way)
+    mT = B.OosModel(cfg, weights, max_T=T, use_graph=True)
+    ref_toks, _, _ = run(mT, eos_bank, T, n_vanilla)
+    seq = [root] + ref_toks
+    rng = np.random.default_rng(seed)
+    bank = []
+    for a in range(0, len(seq) - 24, 12):
+        view = list(seq[a:a + 28])
+        for j in range(7, len(view), 8):
+            view[j] = 3 + (view[j] + 11) % (cfg.vocab - 3)
+        bank += rng.integers(3, cfg.vocab, size=16).tolist() + [eos] + view + [eos]
+    spec_toks, spec_mat, spec_s = run(mT, torch.as_tensor(np.asarray(bank, np.int32), device="cuda"), T, n_rounds)
+    mT.close()
+    k_same = 0
+    while k_same < min(len(spec_toks), len(ref_toks)) and spec_toks[k_same] == ref_toks[k_same]:
+        k_same += 1
+    return {"rounds": n_rounds, "tree_nodes": T, "mat": spec_mat, "mat_mean": sum(spec_mat) / len(spec_mat),
+            "tokens_per_s": len(spec_toks) / spec_s, "vanilla_rounds": n_vanilla,
+            "vanilla_tokens_per_s": len(van_toks) / van_s, "speedup": (len(spec_toks) / spec_s) / (len(van_toks) / van_s),
+            "tokens_equal_plain": k_same, "bank_tokens": len(bank),
+            "note": "device loop: hint-bank suffix match -> tree -> verify -> compaction -> commit per round, one "
+                    "captured graph per round; vanilla = trees of the root alone (T=1); bank = views of the plain "
+                    "greedy continuation (root-only trees of T nodes) with every 8th token altered; "
+                    "tokens_equal_plain = leading committed tokens identical to that continuation"}
 
 
 # ---------------------------------------------------------------- GPU arm
@@ -406,6 +481,15 @@ def run_ours(args):
                 "tree_nodes": tn, "request_bank_tokens": res["request"][0], "request_us": res["request"][1]}
         del bank, ws
 
+    # ---- multi-step decode loop on the device (hint-bank tree -> verify -> compaction -> commit,
+    # no host round trip between rounds), against vanilla decoding (T = 1: the root alone) on the
+    # same model.  The bank holds views of the target's own continuation (found by the vanilla run)
+    # with every 8th token altered, so that acceptance stops inside the views the way a hint bank
+    # that is only partly right makes it stop; tokens committed per call is the paper's #MAT.
+    decode = None
+    if not args.no_decode:
+        decode = decode_leg(B, cfg, weights, native_cache=(seed, ctx), T=T, stream=stream)
+
     # ---- CPU checker on the host cores (rank 0, N = 1 only)
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
@@ -441,6 +525,7 @@ def run_ours(args):
             "clocks": clk,
             "prefill": prefill,
             "hint": hint,
+            "decode": decode,
         }), flush=True)
     model.close()
     if world > 1:
@@ -458,6 +543,7 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-prefill", action="store_true", help="skip the prefill measurement")
     ap.add_argument("--no-hint", action="store_true", help="skip the hint-bank step measurement")
+    ap.add_argument("--no-decode", action="store_true", help="skip the decode-loop measurement")
     ap.add_argument("--layers", type=int, default=0,
                     help="profiling captures only: keep the first N layers of the workload's model")
     args = ap.parse_args()

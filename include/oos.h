@@ -107,6 +107,13 @@ typedef struct {
     float rope_low_freq_factor;
     float rope_high_freq_factor;
     int32_t rope_orig_max_pos;
+    /* Nonzero: the KV cache holds IEEE binary16 (round to nearest even)
+     * instead of the model dtype -- the FP16 cache backend of the paper's
+     * Qwen2.5 and Llama runs ("Targets, Workloads, and Protocol").  bf16
+     * models only (OOS_EUNSUPPORTED otherwise).  Every K/V a node attends to,
+     * cached or written by the tree pass, is then binary16, and the attention
+     * products run in f16. */
+    int32_t kv_f16;
 } oos_model_config;
 
 /* Per-layer weights, all DEVICE pointers. */
@@ -136,7 +143,8 @@ typedef struct {
 
 /* Committed KV cache: per layer one K and one V buffer of `capacity` slots.
  * Slot p holds the post-RoPE K (resp. V) of committed position p for all
- * kv heads: layout [capacity][nkv][d], element type = model dtype.  During
+ * kv heads: layout [capacity][nkv][d], element type = model dtype, or
+ * binary16 with oos_model_config.kv_f16.  During
  * oos_tree_verify the tree's K/V are written to slots ctx_len .. ctx_len+T-1;
  * oos_kv_compact then moves the accepted path to ctx_len .. ctx_len+len-1. */
 typedef struct {

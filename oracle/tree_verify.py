@@ -28,7 +28,8 @@ What the paper leaves open, and the reading taken here:
     rescaling published with that model (rope_inv_freq); the paper runs
     Llama-3.1-8B and does not restate it.
   * K and V are stored in the cache's format before anything attends to them
-    (bf16 for the bf16 models): the tree's own K/V go through the cache too.
+    (bf16 for the bf16 models, binary16 for an FP16 cache): the tree's own K/V
+    go through the cache too.
   * "Longest prefix" is the deepest accepted node, lowest node id on ties;
     argmax ties go to the lowest vocabulary id.
   * The decoder is a pre-norm Llama/Qwen block: RMSNorm, q/k/v projections
@@ -165,6 +166,13 @@ def cache_format(x, dtype):
     return (u.astype(np.uint32) << 16).view(np.float32).astype(np.float64).reshape(np.shape(x))
 
 
+def kv_format(cfg):
+    """Element type of the model's KV cache: cfg.cache_dtype when set (the
+    FP16 cache backend of the paper's Qwen2.5 and Llama runs, "Targets,
+    Workloads, and Protocol"), else the model dtype."""
+    return getattr(cfg, "cache_dtype", "") or cfg.dtype
+
+
 def attend(q, keys, values):
     """softmax(keys q / sqrt(d)) @ values for one query vector."""
     d = q.shape[-1]
@@ -260,8 +268,8 @@ def verify_tree(m, cache_k, cache_v, ctx_len, tokens, parent, only=None):
         v = np.full((T, nkv, d), np.nan)
         for r, i in enumerate(nodes):
             q[i] = rope(q_s[r], ctx_len + depth[i], cfg.rope_theta, rope_scaling(cfg))
-            k[i] = cache_format(rope(k_s[r], ctx_len + depth[i], cfg.rope_theta, rope_scaling(cfg)), cfg.dtype)
-            v[i] = cache_format(v_s[r], cfg.dtype)
+            k[i] = cache_format(rope(k_s[r], ctx_len + depth[i], cfg.rope_theta, rope_scaling(cfg)), kv_format(cfg))
+            v[i] = cache_format(v_s[r], kv_format(cfg))
         tree_k.append(k)
         tree_v.append(v)
         o = np.zeros((T, nq, d))
@@ -356,8 +364,8 @@ def decode_step(m, cache_k, cache_v, n_pos, token):
         h = rms_norm(x, W["attn_norm"], cfg.rms_eps)
         q, k, v = qkv(W, cfg, h)
         q = rope(q[0], n_pos, cfg.rope_theta, rope_scaling(cfg))
-        k = cache_format(rope(k[0], n_pos, cfg.rope_theta, rope_scaling(cfg)), cfg.dtype)
-        v = cache_format(v[0], cfg.dtype)
+        k = cache_format(rope(k[0], n_pos, cfg.rope_theta, rope_scaling(cfg)), kv_format(cfg))
+        v = cache_format(v[0], kv_format(cfg))
         ks.append(k)
         vs.append(v)
         o = np.zeros((nq, d))

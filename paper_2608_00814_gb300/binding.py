@@ -37,7 +37,7 @@ class OosModelConfig(ctypes.Structure):
                 ("qk_norm", c_i32), ("qkv_bias", c_i32), ("rms_eps", ctypes.c_float),
                 ("rope_theta", ctypes.c_float), ("max_T", c_i32), ("use_graph", c_i32),
                 ("rope_factor", ctypes.c_float), ("rope_low_freq_factor", ctypes.c_float),
-                ("rope_high_freq_factor", ctypes.c_float), ("rope_orig_max_pos", c_i32)]
+                ("rope_high_freq_factor", ctypes.c_float), ("rope_orig_max_pos", c_i32), ("kv_f16", c_i32)]
 
 
 LAYER_FIELDS = ("attn_norm", "w_q", "w_k", "w_v", "b_q", "b_k", "b_v", "q_norm", "k_norm", "w_o",
@@ -137,7 +137,8 @@ def make_config(cfg, max_T, use_graph=True):
                           int(use_graph), float(getattr(cfg, "rope_factor", 0.0) or 0.0),
                           float(getattr(cfg, "rope_low_freq_factor", 1.0)),
                           float(getattr(cfg, "rope_high_freq_factor", 4.0)),
-                          int(getattr(cfg, "rope_orig_max_pos", 8192)))
+                          int(getattr(cfg, "rope_orig_max_pos", 8192)),
+                          int(getattr(cfg, "cache_dtype", "") == "f16"))
 
 
 def oos_workspace_bytes(c_cfg):
@@ -159,7 +160,8 @@ class KVCache:
 
     @staticmethod
     def empty(cfg, capacity, device="cuda"):
-        dt = torch.bfloat16 if cfg.dtype == "bf16" else torch.float32
+        dt = torch.float16 if getattr(cfg, "cache_dtype", "") == "f16" else \
+            (torch.bfloat16 if cfg.dtype == "bf16" else torch.float32)
         k = [torch.zeros(capacity, cfg.n_kv_heads, cfg.head_dim, dtype=dt, device=device) for _ in range(cfg.n_layers)]
         v = [torch.zeros_like(t) for t in k]
         return KVCache(k, v)

@@ -66,6 +66,8 @@ constexpr int kOffRecv = kOffV + kKvStages * kTileBytes;  // merge: rows copied 
 constexpr int kOffWgt = kOffRecv + kRecvRows * kMergeRowBytes;   // merge weights [owned row][split]
 constexpr int kOffBar = kOffWgt + kAttnRows * kMaxSplits * 4;
 static_assert(kAttnRows * kMergeRowBytes <= kKvStages * 2 * kTileBytes, "merge staging");
+static_assert(4 * kAttnRows * 128 <= kRecvRows * kMergeRowBytes, "q staging in the receive buffer");
+static_assert((kOffRecv & 1023) == 0, "swizzled q staging is 1024-aligned");
 constexpr int kAttnSmem = kOffBar + 256 + 1024;           // + barriers + alignment slack
 constexpr int kAttnThreads = 224;                         // 7 warps, roles below
 static_assert(kAttnSmem <= 227 * 1024, "shared memory per block");
@@ -81,8 +83,7 @@ static_assert(kTmQ + kAttnD == kAttnTmemCols, "TMEM columns");
 
 struct AttnArgs {
   CUtensorMap kmap, vmap;   // cache [capacity][nkv][d] as (d, kv head, slot)
-  const __nv_bfloat16* q;   // [kMaxT][nq][d] hi halves; lo halves at q_lo_off
-  size_t q_lo_off;
+  CUtensorMap qhi, qlo;     // q [node][nq][d] as (d, head in group, kv head, node), hi and lo halves
   const unsigned long long* anc;
   const int* ctx_dev;       // committed positions of the step (written by tree preparation)
   int T, nq, group;
@@ -101,7 +102,8 @@ OOS_DEV uint32_t cluster_rank() {
   asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
   return r;
 }
-OOS_DEV void cluster_arrive_release() { asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory"); }
+// not .aligned: the threads of a warp may arrive at different points
+OOS_DEV void cluster_arrive_release() { asm volatile("barrier.cluster.arrive.release;" ::: "memory"); }
 OOS_DEV void cluster_wait_acquire() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
 // address of the same shared-memory location in block `rank` of the cluster
 OOS_DEV uint32_t dsmem_addr(const void* p, uint32_t rank) {
@@ -139,6 +141,9 @@ OOS_DEV float ex2_approx(float x) {
   asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
   return y;
 }
+// 16-byte chunk c of row r of a 128-byte-swizzled tile (rows 128 bytes apart,
+// 8-row / 1024-byte swizzle atoms, tile base 1024-aligned)
+OOS_DEV uint32_t sw128(int r, int c) { return (uint32_t)(r * 128 + ((c ^ (r & 7)) << 4)); }
 // 32 lanes x 32 bit, 16 consecutive columns per thread, TMEM <- raw words
 OOS_DEV void tmem_st16u(uint32_t taddr, const uint32_t* v) {
   asm volatile(
@@ -224,6 +229,9 @@ OOS_DEV void drain_wait(uint64_t* bar, uint32_t parity) {
 // layouts); warp 1 lane 0 issues the S MMAs, warp 6 lane 0 the P.V MMAs;
 // warps 2..5 load q into TMEM and run the softmax (thread = query row = TMEM
 // lane); all warps take part in the merge.
+// F16: the KV cache (and q) are IEEE binary16 -- every product runs in f16;
+// otherwise bf16.
+template <bool F16>
 __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_constant__ AttnArgs a) {
   extern __shared__ __align__(1024) unsigned char smem_raw[];
   unsigned char* sm = reinterpret_cast<unsigned char*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -238,9 +246,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
   uint64_t* qtm = bar + 14;       // 4 softmax warps: q rows are in TMEM
   uint64_t* odone = bar + 15;     // both MMA issuers done
   uint64_t* recv_full = bar + 16; // merge: every split's rows for this block copied in (transaction bytes)
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar + 17);
+  uint64_t* qfull = bar + 17;     // q tile landed (transaction bytes)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(bar + 18);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
-  static_assert(17 * 8 + 8 <= 256, "barrier block");
+  static_assert(18 * 8 + 8 <= 256, "barrier block");
 
   const int T = a.T, nq = a.nq, G = a.group, npc = a.npc, S = a.splits;
   const float scale_log2 = a.scale_log2;
@@ -278,6 +287,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
     mbar_init(qtm, 4);
     mbar_init(odone, 2);
     mbar_init(recv_full, 1);
+    mbar_init(qfull, 1);
     // every split copies its rows of this block in: S * n_mine merge rows
     mbar_arrive_expect_tx(recv_full, (uint32_t)(S * n_mine * kMergeRowBytes));
     *abort_flag = 0;
@@ -287,10 +297,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  // Another block may copy into this block's shared memory only once the
-  // block runs and its receive barrier is armed: arrive now, and every block
-  // waits for the whole cluster before its merge copies.
-  cluster_arrive_release();
+  // Another block may copy into this block's receive buffer only once the
+  // block runs, its receive barrier is armed and the q tile staged in that
+  // buffer has gone to TMEM: every thread arrives on the cluster barrier when
+  // it is past that point (the q rows' threads after their copy, the others
+  // now), and every block waits for the whole cluster before its merge copies.
+  if (warp < 2 || warp > 5) cluster_arrive_release();
   const uint32_t tmem = *tmem_slot;
   const uint32_t tmem_o = tmem + kTmO;
 
@@ -320,6 +332,19 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
       }
       pdl_wait();
       pdl_trigger();
+      // q rows of the block's nodes, hi and lo halves, two 64-wide d blocks
+      // each, staged in the (still unused) receive buffer
+      tma_prefetch_desc(&a.qhi);
+      tma_prefetch_desc(&a.qlo);
+      {
+        const uint64_t pol_q = policy_evict_last();
+        unsigned char* qs = sm + kOffRecv;
+        mbar_arrive_expect_tx(qfull, (uint32_t)(4 * rows * 128));
+        tma_load_4d(qs, &a.qhi, qfull, 0, 0, g, node0, pol_q);
+        tma_load_4d(qs + kAttnRows * 128, &a.qhi, qfull, 64, 0, g, node0, pol_q);
+        tma_load_4d(qs + 2 * kAttnRows * 128, &a.qlo, qfull, 0, 0, g, node0, pol_q);
+        tma_load_4d(qs + 3 * kAttnRows * 128, &a.qlo, qfull, 64, 0, g, node0, pol_q);
+      }
       for (int ti = nk; ti < n_tiles; ++ti) {
         const int st = ti & 1;
         const uint32_t use = (uint32_t)(ti >> 1);
@@ -357,7 +382,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
     // Descriptors: the start address is the low field (16-byte units), so a
     // byte offset o inside an operand region is added as o >> 4.
     if (lane == 0 && warp == 1) {
-      constexpr uint32_t idesc_s = idesc_bf16_f32(kAttnRows, kAttnKeys);
+      constexpr uint32_t idesc_s = F16 ? idesc_f16_f32(kAttnRows, kAttnKeys) : idesc_bf16_f32(kAttnRows, kAttnKeys);
       bool ok = attn_wait(qtm, 0, abort_flag, status, AW_QTM, 0);
       tc_fence_after();
       const uint64_t kdesc0 = smem_desc_sw128(smem_addr(sm + kOffK));
@@ -387,7 +412,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
       }
       tc_commit(odone);
     } else if (lane == 0 && warp == 6) {
-      constexpr uint32_t idesc_pv = idesc_bf16_f32(kAttnRows, kAttnD) | (1u << 16);   // B (V) MN-major
+      constexpr uint32_t idesc_pv =
+          (F16 ? idesc_f16_f32(kAttnRows, kAttnD) : idesc_bf16_f32(kAttnRows, kAttnD)) | (1u << 16);   // B (V) MN-major
       // V tile: d blocks of 64 (kDBlock apart) along N, 16 keys (2 KB) per MMA along K
       const uint64_t vdesc0 = smem_desc_sw128_mn(smem_addr(sm + kOffV), kDBlock);
       for (int ti = 0; ti < n_tiles; ++ti) {
@@ -421,28 +447,33 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
     pdl_wait();
     pdl_trigger();
     const unsigned long long anc0 = a.anc[2 * node], anc1 = a.anc[2 * node + 1];
-    {
-      // this thread's q row (hi then lo, 64 columns each as bf16 pairs) into
-      // TMEM, the S MMAs' A operand; rows of padding nodes are zero
-      const __nv_bfloat16* qh = a.q + ((size_t)node * nq + g * G + (real ? lrow % G : 0)) * kAttnD;
-      uint4 w[2][16];
+    // this thread's q row (hi then lo, 64 columns each as bf16 pairs) from the
+    // staged swizzled tile into TMEM, the S MMAs' A operand; rows of padding
+    // nodes are zero
+    const bool qok = __all_sync(0xffffffffu, attn_wait(qfull, 0, abort_flag, status, AW_QTM, 0));
+    if (qok) {
+      const unsigned char* qs = sm + kOffRecv;
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const uint4* src = reinterpret_cast<const uint4*>(h ? qh + a.q_lo_off : qh);
+      for (int part = 0; part < 8; ++part) {   // (hi/lo, 64-wide d block, half of its 8 chunks)
+        const unsigned char* qb = qs + (part >> 1) * (kAttnRows * 128);
+        uint32_t w[16];
 #pragma unroll
-        for (int c = 0; c < 16; ++c) w[h][c] = real ? __ldcg(src + c) : make_uint4(0, 0, 0, 0);
+        for (int c = 0; c < 4; ++c) {
+          const uint4 v = real ? *reinterpret_cast<const uint4*>(qb + sw128(lrow, (part & 1) * 4 + c))
+                               : make_uint4(0, 0, 0, 0);
+          w[4 * c] = v.x;
+          w[4 * c + 1] = v.y;
+          w[4 * c + 2] = v.z;
+          w[4 * c + 3] = v.w;
+        }
+        tmem_st16u(tmem + lane_off + kTmQ + part * 16, w);
       }
-#pragma unroll
-      for (int h = 0; h < 2; ++h)
-#pragma unroll
-        for (int part = 0; part < 4; ++part)
-          tmem_st16u(tmem + lane_off + kTmQ + h * (kAttnD / 2) + part * 16,
-                     reinterpret_cast<const uint32_t*>(&w[h][part * 4]));
       tmem_wait_st();
     }
     tc_fence_before();
     __syncwarp();
     if (lane == 0) mbar_arrive(qtm);
+    cluster_arrive_release();   // this thread is done with the staged q
     for (int ti = 0; ti < n_tiles; ++ti) {
       const int b = ti & 1;
       const uint32_t use = (uint32_t)(ti >> 1);
@@ -515,10 +546,16 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
       for (int i = 0; i < kAttnKeys; i += 2) {
         const float p0 = live ? ex2_approx(fmaf(sv[i], scale_log2, neg_m)) : 0.f;
         const float p1 = live ? ex2_approx(fmaf(sv[i + 1], scale_log2, neg_m)) : 0.f;
-        const __nv_bfloat162 pp = __floats2bfloat162_rn(p0, p1);
-        // the sum uses the rounded weights that P.V multiplies
-        ps[(i >> 1) & 3] += __low2float(pp) + __high2float(pp);
-        pk[i / 2] = *reinterpret_cast<const uint32_t*>(&pp);
+        // P in the operand format of V; the sum uses the rounded weights that P.V multiplies
+        if constexpr (F16) {
+          const __half2 pp = __floats2half2_rn(p0, p1);
+          ps[(i >> 1) & 3] += __low2float(pp) + __high2float(pp);
+          pk[i / 2] = *reinterpret_cast<const uint32_t*>(&pp);
+        } else {
+          const __nv_bfloat162 pp = __floats2bfloat162_rn(p0, p1);
+          ps[(i >> 1) & 3] += __low2float(pp) + __high2float(pp);
+          pk[i / 2] = *reinterpret_cast<const uint32_t*>(&pp);
+        }
       }
       l_sum += (ps[0] + ps[1]) + (ps[2] + ps[3]);
       // slots at or past ctx + T in this tile hold whatever the cache holds
@@ -687,6 +724,20 @@ __global__ void __launch_bounds__(128) k_attn_f32(const float* __restrict__ q, c
 
 int attn_nodes_per_block(int group) { return group >= kAttnRows ? 1 : kAttnRows / group; }
 
+bool attn_encode_q_maps(Model& m) {
+  const auto& c = m.cfg;
+  const int group = c.n_q_heads / c.n_kv_heads;
+  // q [node][nq][d] viewed as (d, head in group, kv head, node); a box is the
+  // (node, head in group) rows of one kv head, 64 of d at a time
+  const uint64_t dims[4] = {(uint64_t)kAttnD, (uint64_t)group, (uint64_t)c.n_kv_heads, (uint64_t)kMaxT};
+  const uint64_t strides[3] = {(uint64_t)kAttnD * 2, (uint64_t)group * kAttnD * 2, (uint64_t)c.n_q_heads * kAttnD * 2};
+  const uint32_t box[4] = {64, (uint32_t)group, 1, (uint32_t)attn_nodes_per_block(group)};
+  const __nv_bfloat16* q = (const __nv_bfloat16*)m.ws.q;
+  const bool f16 = c.kv_f16 != 0;
+  return encode_bf16_map(&m.qmap_hi, q, 4, dims, strides, box, f16) &&
+         encode_bf16_map(&m.qmap_lo, q + (size_t)kMaxT * c.n_q_heads * kAttnD, 4, dims, strides, box, f16);
+}
+
 // clusters of `sp` attention blocks resident at once on this device (occupancy query, cached)
 static int attn_max_clusters(int sp) {
   static int cached[kMaxSplits + 1] = {0};
@@ -704,16 +755,22 @@ static int attn_max_clusters(int sp) {
     lc.attrs = attr;
     lc.numAttrs = 1;
     int n = 0;
-    cached[sp] = cudaOccupancyMaxActiveClusters(&n, (const void*)k_attn_tc, &lc) == cudaSuccess && n > 0 ? n : -1;
+    cached[sp] = cudaOccupancyMaxActiveClusters(&n, (const void*)k_attn_tc<false>, &lc) == cudaSuccess && n > 0 ? n : -1;
     cudaGetLastError();
   }
   return cached[sp];
 }
 
-cudaError_t attn_setup() {
-  cudaError_t e = cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmem);
-  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_attn_tc, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+template <bool F16>
+static cudaError_t attn_setup_one() {
+  cudaError_t e = cudaFuncSetAttribute(k_attn_tc<F16>, cudaFuncAttributeMaxDynamicSharedMemorySize, kAttnSmem);
+  if (e == cudaSuccess) e = cudaFuncSetAttribute(k_attn_tc<F16>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
   return e;
+}
+
+cudaError_t attn_setup() {
+  cudaError_t e = attn_setup_one<false>();
+  return e == cudaSuccess ? attn_setup_one<true>() : e;
 }
 
 int attn_splits(Model& m, int ctx_hint, int T) {
@@ -749,8 +806,8 @@ cudaError_t launch_attention(Model& m, int layer, const void* kc, const void* vc
       const uint64_t dims[3] = {(uint64_t)kAttnD, (uint64_t)c.n_kv_heads, (uint64_t)capacity};
       const uint64_t strides[2] = {(uint64_t)kAttnD * 2, (uint64_t)c.n_kv_heads * kAttnD * 2};
       const uint32_t box[3] = {64, 1, (uint32_t)kAttnKeys};
-      if (!encode_bf16_map(&km.kmap, kc, 3, dims, strides, box) ||
-          !encode_bf16_map(&km.vmap, vc, 3, dims, strides, box)) {
+      if (!encode_bf16_map(&km.kmap, kc, 3, dims, strides, box, c.kv_f16 != 0) ||
+          !encode_bf16_map(&km.vmap, vc, 3, dims, strides, box, c.kv_f16 != 0)) {
         km.k = km.v = nullptr;
         return cudaErrorInvalidValue;
       }
@@ -761,8 +818,8 @@ cudaError_t launch_attention(Model& m, int layer, const void* kc, const void* vc
     a.kmap = km.kmap;
     a.vmap = km.vmap;
   }
-  a.q = (const __nv_bfloat16*)m.ws.q;
-  a.q_lo_off = (size_t)kMaxT * c.n_q_heads * kAttnD;
+  a.qhi = m.qmap_hi;
+  a.qlo = m.qmap_lo;
   a.anc = m.ws.anc;
   a.ctx_dev = m.ws.ctx;
   a.T = T;
@@ -793,7 +850,7 @@ cudaError_t launch_attention(Model& m, int layer, const void* kc, const void* vc
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   lc.attrs = attr;
   lc.numAttrs = m.pdl ? 2 : 1;
-  return cudaLaunchKernelEx(&lc, k_attn_tc, a);
+  return c.kv_f16 ? cudaLaunchKernelEx(&lc, k_attn_tc<true>, a) : cudaLaunchKernelEx(&lc, k_attn_tc<false>, a);
 }
 
 }  // namespace oos

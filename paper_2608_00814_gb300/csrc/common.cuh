@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -56,6 +57,21 @@ OOS_DEV void store_act4(__nv_bfloat16* p, size_t i, size_t lo_off, float4 v) {
   for (int c = 0; c < 4; ++c) {
     hi[c] = __float2bfloat16_rn(a[c]);
     lo[c] = __float2bfloat16_rn(a[c] - __bfloat162float(hi[c]));
+  }
+  *reinterpret_cast<uint2*>(p + i) = *reinterpret_cast<const uint2*>(hi);
+  *reinterpret_cast<uint2*>(p + i + lo_off) = *reinterpret_cast<const uint2*>(lo);
+}
+
+// The same split into IEEE binary16 halves (hi = fp16(v), lo = fp16(v - hi)):
+// the query layout of a model whose KV cache is binary16, so that the
+// attention products multiply f16 by f16.
+OOS_DEV void store_act4_h(__half* p, size_t i, size_t lo_off, float4 v) {
+  const float a[4] = {v.x, v.y, v.z, v.w};
+  __half hi[4], lo[4];
+#pragma unroll
+  for (int c = 0; c < 4; ++c) {
+    hi[c] = __float2half_rn(a[c]);
+    lo[c] = __float2half_rn(a[c] - __half2float(hi[c]));
   }
   *reinterpret_cast<uint2*>(p + i) = *reinterpret_cast<const uint2*>(hi);
   *reinterpret_cast<uint2*>(p + i + lo_off) = *reinterpret_cast<const uint2*>(lo);
@@ -253,6 +269,11 @@ OOS_DEV uint64_t smem_desc_sw128(uint32_t saddr) {
 //   15/16 A/B major (0 = K), 17-22 N >> 3, 24-28 M >> 4
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
   return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+
+// Same for f16 A and B (format 0 in both fields), fp32 D.
+__host__ __device__ constexpr uint32_t idesc_f16_f32(int M, int N) {
+  return (1u << 4) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
 }
 
 // D[tmem] (+)= A[smem] * B[smem]^T, one elected thread issues

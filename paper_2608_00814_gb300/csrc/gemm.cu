@@ -70,6 +70,7 @@ struct GemmArgs {
   const float2* rope;   // [kMaxT][64] (cos, sin) of the step's positions
   __nv_bfloat16 *q_out, *kc, *vc;
   const int32_t* ctx;   // committed length of the step (device; K/V of node t go to slot *ctx + t)
+  int kv_f16;           // the KV cache (and so q) are binary16 instead of bf16
   // EPI_RESID
   float* x;
   const __nv_bfloat16* gain;
@@ -130,6 +131,7 @@ OOS_DEV Top2s t2_merge(Top2s a, Top2s b) {
 
 OOS_DEV void epi_bar() { asm volatile("bar.sync 1, 128;" ::: "memory"); }
 
+
 // Finishing a subtile: warp w of the four epilogue warps owns token rows
 // t = t0 + 4k + w, lane l owns the four features 4l..4l+3 of the subtile, so a
 // token's 128 features sit in one warp (RMSNorm sums, q/k norm and the RoPE
@@ -140,15 +142,24 @@ constexpr int kFinRows = 4;    // token rows per warp per pass (16 tokens per pa
 OOS_DEV float4 f4_add(float4 a, float4 b) { return make_float4(a.x + b.x, a.y + b.y, a.z + b.z, a.w + b.w); }
 OOS_DEV float4 f4_ldcg(const float* p) { return __ldcg(reinterpret_cast<const float4*>(p)); }
 
+// Where a finishing pass reads the partial sums of output (token t, feature f)
+// from: partial s of nc, the stream-K slices in global memory,
+// [slice][kMaxT][n_part] (feature f of the stacked weight).
+struct GSrc {
+  const float* p;
+  size_t slice;
+  int ld;
+  OOS_DEV float4 ld4(int s, int t, int f) const { return f4_ldcg(p + (size_t)s * slice + (size_t)t * ld + f); }
+};
+
 // acc[k] = (init ? init row : 0) + sum over nc slices of the partial tile rows,
 // rows t = t0 + nw k + w below T (the end of the token range; w is this warp's
 // index among the nw warps finishing the tile).  Slices are
 // fetched BATCH at a time -- every load of a group is issued before any is
 // added -- and added in slice order, so the sum is the same for every finisher.
-template <int R, int BATCH>
-OOS_DEV void load_tile_rows(float4 (&acc)[R], const float* __restrict__ part, int nc, size_t slice, int n_part,
-                            int col, int t0, int T, const float* __restrict__ init, int init_ld, int init_col, int w,
-                            int nw) {
+template <int R, int BATCH, typename Src>
+OOS_DEV void load_tile_rows(float4 (&acc)[R], const Src& src, int nc, int col, int t0, int T,
+                            const float* __restrict__ init, int init_ld, int init_col, int w, int nw) {
 #pragma unroll
   for (int k = 0; k < R; ++k) {
     const int t = t0 + nw * k + w;
@@ -159,11 +170,10 @@ OOS_DEV void load_tile_rows(float4 (&acc)[R], const float* __restrict__ part, in
     float4 v[BATCH][R];
 #pragma unroll
     for (int q = 0; q < BATCH; ++q) {
-      const float* base = part + (size_t)(s0 + q) * slice + col;
 #pragma unroll
       for (int k = 0; k < R; ++k) {
         const int t = t0 + nw * k + w;
-        v[q][k] = (s0 + q < nc && t < T) ? f4_ldcg(base + (size_t)t * n_part) : make_float4(0.f, 0.f, 0.f, 0.f);
+        v[q][k] = (s0 + q < nc && t < T) ? src.ld4(s0 + q, t, col) : make_float4(0.f, 0.f, 0.f, 0.f);
       }
     }
 #pragma unroll
@@ -174,22 +184,21 @@ OOS_DEV void load_tile_rows(float4 (&acc)[R], const float* __restrict__ part, in
 }
 
 // gate (col) and up (col + up_off) rows of a SwiGLU pair, two slices per batch
-template <int R>
-OOS_DEV void load_pair_rows(float4 (&g)[R], float4 (&u)[R], const float* __restrict__ part, int nc, size_t slice,
-                            int n_part, int col, int up_off, int t0, int T, int w, int nw) {
+template <int R, typename Src>
+OOS_DEV void load_pair_rows(float4 (&g)[R], float4 (&u)[R], const Src& src, int nc, int col, int up_off, int t0,
+                            int T, int w, int nw) {
 #pragma unroll
   for (int k = 0; k < R; ++k) g[k] = u[k] = make_float4(0.f, 0.f, 0.f, 0.f);
   for (int s0 = 0; s0 < nc; s0 += 2) {
     float4 vg[2][R], vu[2][R];
 #pragma unroll
     for (int q = 0; q < 2; ++q) {
-      const float* base = part + (size_t)(s0 + q) * slice + col;
 #pragma unroll
       for (int k = 0; k < R; ++k) {
         const int t = t0 + nw * k + w;
         const bool ok = s0 + q < nc && t < T;
-        vg[q][k] = ok ? f4_ldcg(base + (size_t)t * n_part) : make_float4(0.f, 0.f, 0.f, 0.f);
-        vu[q][k] = ok ? f4_ldcg(base + (size_t)t * n_part + up_off) : make_float4(0.f, 0.f, 0.f, 0.f);
+        vg[q][k] = ok ? src.ld4(s0 + q, t, col) : make_float4(0.f, 0.f, 0.f, 0.f);
+        vu[q][k] = ok ? src.ld4(s0 + q, t, col + up_off) : make_float4(0.f, 0.f, 0.f, 0.f);
       }
     }
 #pragma unroll
@@ -210,14 +219,14 @@ OOS_DEV float4 bf16x4(const __nv_bfloat16* p) {
 
 // EPI_RESID on 128-row tile `tile`, tokens [tb, te), by warp w of nw: x += W.a;
 // y = g (.) x; per-tile sums of x^2
-OOS_DEV void finish_resid(const GemmArgs& a, int n_part, int tile, int nc, int tb, int te, int w, int nw) {
+template <typename Src>
+OOS_DEV void finish_resid(const GemmArgs& a, const Src& src, int tile, int nc, int tb, int te, int w, int nw) {
   const int l = threadIdx.x & 31;
-  const size_t slice = (size_t)kMaxT * n_part;
   const int f = tile * kTile + 4 * l;
   const float4 g = bf16x4(a.gain + f);
   for (int t0 = tb; t0 < te; t0 += nw * kFinRows) {
     float4 acc[kFinRows];
-    load_tile_rows<kFinRows, 8>(acc, a.part, nc, slice, n_part, f, t0, te, a.x, a.N, f, w, nw);   // x + sum of slices
+    load_tile_rows<kFinRows, 8>(acc, src, nc, f, t0, te, a.x, a.N, f, w, nw);   // x + sum of the partials
 #pragma unroll
     for (int k = 0; k < kFinRows; ++k) {
       const int t = t0 + nw * k + w;
@@ -234,16 +243,16 @@ OOS_DEV void finish_resid(const GemmArgs& a, int n_part, int tile, int nc, int t
 
 // EPI_SILU on work tile wt (subtile 0 = gate rows of block wt, subtile 1 = up
 // rows), tokens [tb, te), by warp w of nw
-OOS_DEV void finish_silu(const GemmArgs& a, int n_part, int wt, int nc, const float* rms, int tb, int te, int w,
+template <typename Src>
+OOS_DEV void finish_silu(const GemmArgs& a, const Src& src, int wt, int nc, const float* rms, int tb, int te, int w,
                          int nw) {
   const int l = threadIdx.x & 31;
-  const size_t slice = (size_t)kMaxT * n_part;
   const int i = wt * kTile + 4 * l;
   constexpr int R = 8;   // 8 token rows per warp per pass
   for (int t0 = tb; t0 < te; t0 += nw * R) {
     float4 gv[R], uv[R];
     // gate and up slices of a pass in one batch of loads
-    load_pair_rows<R>(gv, uv, a.part, nc, slice, n_part, 2 * wt * kTile + 4 * l, kTile, t0, te, w, nw);
+    load_pair_rows<R>(gv, uv, src, nc, 2 * wt * kTile + 4 * l, kTile, t0, te, w, nw);
 #pragma unroll
     for (int k = 0; k < R; ++k) {
       const int t = t0 + nw * k + w;
@@ -261,10 +270,10 @@ OOS_DEV void finish_silu(const GemmArgs& a, int n_part, int wt, int nc, const fl
 
 // EPI_QKV on 128-row tile `tile` = one head (q heads, then k heads, then v
 // heads), tokens [tb, te), by warp w of nw
-OOS_DEV void finish_qkv(const GemmArgs& a, int n_part, int tile, int nc, const float* rms, int tb, int te, int w,
+template <typename Src>
+OOS_DEV void finish_qkv(const GemmArgs& a, const Src& src, int tile, int nc, const float* rms, int tb, int te, int w,
                         int nw) {
   const int l = threadIdx.x & 31;
-  const size_t slice = (size_t)kMaxT * n_part;
   int kind, h;
   if (tile < a.nq) { kind = 0; h = tile; }
   else if (tile < a.nq + a.nkv) { kind = 1; h = tile - a.nq; }
@@ -278,7 +287,7 @@ OOS_DEV void finish_qkv(const GemmArgs& a, int n_part, int tile, int nc, const f
   const bool first_half = l < 16;   // features 0..63 pair with 64..127 held by lane ^ 16
   for (int t0 = tb; t0 < te; t0 += nw * kFinRows) {
     float4 acc[kFinRows];
-    load_tile_rows<kFinRows, 8>(acc, a.part, nc, slice, n_part, tile * kTile + 4 * l, t0, te, nullptr, 0, 0, w, nw);
+    load_tile_rows<kFinRows, 8>(acc, src, nc, tile * kTile + 4 * l, t0, te, nullptr, 0, 0, w, nw);
 #pragma unroll
     for (int k = 0; k < kFinRows; ++k) {
       const int t = t0 + nw * k + w;
@@ -301,15 +310,25 @@ OOS_DEV void finish_qkv(const GemmArgs& a, int n_part, int tile, int nc, const f
           v[c] = first_half ? v[c] * cs.x - other * cs.y : v[c] * cs.x + other * cs.y;
         }
       }
-      if (kind == 0) {   // q as hi/lo bf16 halves: the attention product sees ~16-bit q
-        store_act4(a.q_out, ((size_t)t * a.nq + h) * kTile + 4 * l, (size_t)kMaxT * a.nq * kTile,
-                   make_float4(v[0], v[1], v[2], v[3]));
-      } else {           // K/V in the cache's bf16 format
+      if (kind == 0) {   // q as hi/lo halves in the cache's 16-bit format: the attention product sees ~16-bit q
+        const size_t qi = ((size_t)t * a.nq + h) * kTile + 4 * l, lo_off = (size_t)kMaxT * a.nq * kTile;
+        if (a.kv_f16) store_act4_h(reinterpret_cast<__half*>(a.q_out), qi, lo_off, make_float4(v[0], v[1], v[2], v[3]));
+        else store_act4(a.q_out, qi, lo_off, make_float4(v[0], v[1], v[2], v[3]));
+      } else {           // K/V in the cache's format (bf16, or binary16)
         __nv_bfloat16* dst = (kind == 1 ? a.kc : a.vc) + ((size_t)(ctx + t) * a.nkv + h) * kTile;
-        __nv_bfloat16 o[4];
+        uint2 o;
+        if (a.kv_f16) {
+          __half hv[4];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) o[c] = __float2bfloat16_rn(v[c]);
-        *reinterpret_cast<uint2*>(dst + 4 * l) = *reinterpret_cast<const uint2*>(o);
+          for (int c = 0; c < 4; ++c) hv[c] = __float2half_rn(v[c]);
+          o = *reinterpret_cast<const uint2*>(hv);
+        } else {
+          __nv_bfloat16 bv[4];
+#pragma unroll
+          for (int c = 0; c < 4; ++c) bv[c] = __float2bfloat16_rn(v[c]);
+          o = *reinterpret_cast<const uint2*>(bv);
+        }
+        *reinterpret_cast<uint2*>(dst + 4 * l) = o;
       }
     }
   }
@@ -743,15 +762,16 @@ __global__ void __launch_bounds__(192, 1)
         const int nw = two ? 2 : 4, w = two ? (ew & 1) : ew;
         const int wt = second ? wt1 : wt0, nc = second ? nc1 : nc0, tb = second ? tb1 : tb0, te = second ? te1 : te0;
         if (tb < te) {
+          const GSrc src{a.part, (size_t)kMaxT * n_part, n_part};
           if (EPI == EPI_SILU) {
-            finish_silu(a, n_part, wt, nc, rms, tb, te, w, nw);
+            finish_silu(a, src, wt, nc, rms, tb, te, w, nw);
           } else {
 #pragma unroll 1
             for (int sub = 0; sub < kSub; ++sub) {
               const int tile = wt * kSub + sub;
               if (tile >= a.n_tiles) break;
-              if (EPI == EPI_RESID) finish_resid(a, n_part, tile, nc, tb, te, w, nw);
-              else finish_qkv(a, n_part, tile, nc, rms, tb, te, w, nw);
+              if (EPI == EPI_RESID) finish_resid(a, src, tile, nc, tb, te, w, nw);
+              else finish_qkv(a, src, tile, nc, rms, tb, te, w, nw);
             }
           }
         }
@@ -805,7 +825,7 @@ static bool encode_2d(CUtensorMap* map, const void* ptr, int rows, int K, int bo
 }
 
 bool encode_bf16_map(CUtensorMap* map, const void* ptr, int rank, const uint64_t* dims, const uint64_t* strides,
-                     const uint32_t* box) {
+                     const uint32_t* box, bool f16) {
   EncodeTiledFn enc = get_encode();
   if (!enc || rank < 1 || rank > 5) return false;
   memset(map, 0, sizeof(*map));
@@ -817,7 +837,8 @@ bool encode_bf16_map(CUtensorMap* map, const void* ptr, int rank, const uint64_t
     estr[i] = 1;
     if (i + 1 < rank) gstride[i] = strides[i];
   }
-  CUresult r = enc(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank, const_cast<void*>(ptr), gdim, gstride, bx,
+  CUresult r = enc(map, f16 ? CU_TENSOR_MAP_DATA_TYPE_FLOAT16 : CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank,
+                   const_cast<void*>(ptr), gdim, gstride, bx,
                    estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
   return r == CUDA_SUCCESS;
@@ -834,9 +855,11 @@ int bn_index(int T) { return T <= 16 ? 0 : T <= 32 ? 1 : T <= 64 ? 2 : 3; }
 
 template <int BN, int EPI>
 static cudaError_t set_smem() {
-  return cudaFuncSetAttribute(k_gemm_tc<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                              TcCfg<BN, SubOf<EPI>::v>::SMEM);
+  cudaError_t e = cudaFuncSetAttribute(k_gemm_tc<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       TcCfg<BN, SubOf<EPI>::v>::SMEM);
+  return e;
 }
+
 
 template <int BN>
 static cudaError_t set_smem_all() {
@@ -870,6 +893,7 @@ static cudaError_t launch_tc(Model& m, const GemmW& g, const CUtensorMap& amap, 
 template <int EPI>
 static cudaError_t dispatch_tc(Model& m, const GemmW& g, const CUtensorMap* amaps, int T, int grid, GemmArgs& a,
                                const GemmW* next, cudaStream_t st) {
+  const int bi = bn_index(T);
   if (next) {
     // about 64 KB of the next GEMM's weights per CTA index
     a.pf_units = 4 / next->sub;
@@ -883,7 +907,6 @@ static cudaError_t dispatch_tc(Model& m, const GemmW& g, const CUtensorMap* amap
     a.pf_round_robin = next->round_robin;
     for (int s = 0; s < 3; ++s) a.pf_seg_tiles[s] = next->seg_tiles[s < next->n_seg ? s : next->n_seg - 1];
   }
-  const int bi = bn_index(T);
   switch (bi) {
     case 0: return launch_tc<16, EPI>(m, g, amaps[0], grid, a, next, st);
     case 1: return launch_tc<32, EPI>(m, g, amaps[1], grid, a, next, st);
@@ -931,6 +954,7 @@ cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int T, cons
   a.kc = (__nv_bfloat16*)kc;
   a.vc = (__nv_bfloat16*)vc;
   a.ctx = m.ws.ctx;
+  a.kv_f16 = c.kv_f16 ? 1 : 0;
   return dispatch_tc<EPI_QKV>(m, m.g_qkv[layer], m.amap_xn, T, m.g_qkv[layer].plan.grid, a, next, st);
 }
 

@@ -120,6 +120,7 @@ struct Model {
   std::vector<GemmW> g_qkv, g_o, g_gu, g_down;
   GemmW g_lm;
   CUtensorMap amap_xn[4], amap_attn[4], amap_act[4];  // per N-tile variant 16/32/64/128
+  CUtensorMap qmap_hi, qmap_lo;   // attention: q rows of one kv head, (d, head in group, kv head, node)
   // attention: the K/V cache maps encoded per layer over the whole capacity
   // (re-encoded only when the cache buffers change)
   struct KvMaps {
@@ -182,10 +183,11 @@ cudaError_t launch_accept_walk(const int32_t* tokens, const int32_t* parent, con
 
 // ---- GEMMs (gemm.cu)
 bool encode_weight_map(CUtensorMap* map, const void* ptr, int rows, int K);
-// bf16 tensor map with 128-byte swizzle: dims[0] contiguous, strides[i] = bytes
-// between consecutive indices of dim i + 1, box[] elements per dim
+// 16-bit (bf16, or binary16 when f16) tensor map with 128-byte swizzle: dims[0]
+// contiguous, strides[i] = bytes between consecutive indices of dim i + 1, box[]
+// elements per dim
 bool encode_bf16_map(CUtensorMap* map, const void* ptr, int rank, const uint64_t* dims, const uint64_t* strides,
-                     const uint32_t* box);
+                     const uint32_t* box, bool f16 = false);
 bool encode_act_map(CUtensorMap* map, const void* ptr, int K, int box_rows);
 int bn_index(int T);   // N-tile variant for T tree nodes: 0..3 -> 16/32/64/128
 cudaError_t gemm_setup();
@@ -222,6 +224,7 @@ cudaError_t launch_hint_tree(const int32_t* bank, int N, int eos, const int32_t*
 // ---- attention (attn.cu)
 cudaError_t attn_setup();
 int attn_nodes_per_block(int group);   // tree nodes per attention block (x group q heads <= 128 rows)
+bool attn_encode_q_maps(Model& m);     // TMA maps of the q buffer (bf16 path), at model creation
 // the step's ctx comes from the workspace; ctx here only sizes the key splits
 cudaError_t launch_attention(Model& m, int layer, const void* kc, const void* vc, int capacity, int ctx, int T,
                              cudaStream_t st);

@@ -131,6 +131,7 @@ static bool config_ok(const oos_model_config* c) {
 }
 
 static bool shape_supported(const oos_model_config* c) {
+  if (c->kv_f16 && c->dtype != OOS_DTYPE_BF16) return false;   // FP16 caches: bf16 models only
   if (c->dtype == OOS_DTYPE_BF16) {
     if (c->head_dim != 128 || c->hidden % 128 || c->intermediate % 128) return false;
     if (c->hidden / 128 > kMaxSsChunks) return false;
@@ -435,6 +436,7 @@ int oos_model_create(const oos_model_config* cfg, const oos_weights* w, void* wo
         ok = encode_act_map(&m->amap_xn[b], m->ws.xn, H, boxes[b]) &&
              encode_act_map(&m->amap_attn[b], m->ws.attn, qd, boxes[b]) &&
              encode_act_map(&m->amap_act[b], m->ws.act, I, boxes[b]);
+      ok = ok && attn_encode_q_maps(*m);
       if (!ok) {
         rc = OOS_ECUDA;
         break;

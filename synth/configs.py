@@ -31,6 +31,9 @@ class ModelConfig:
     qkv_bias: bool        # Qwen2.5: bias on the q, k, v projections
     tied: bool            # LM head shares the embedding matrix
     init_std: float = 0.02
+    # element type of the KV cache when it differs from `dtype` ("f16": the
+    # FP16 cache backend the paper's Qwen2.5 and Llama runs use); "" = dtype
+    cache_dtype: str = ""
     # Llama 3.1 rotary frequency rescaling (factor <= 1: none)
     rope_factor: float = 0.0
     rope_low_freq_factor: float = 1.0
@@ -44,6 +47,10 @@ class ModelConfig:
     @property
     def kv_dim(self):
         return self.n_kv_heads * self.head_dim
+
+    @property
+    def kv_dtype(self):
+        return self.cache_dtype or self.dtype
 
     def as_dict(self):
         return asdict(self)
@@ -78,7 +85,7 @@ QWEN3_8B = ModelConfig("qwen3-8b", n_layers=36, hidden=4096, n_q_heads=32,
                        vocab=151936, rms_eps=1e-6, rope_theta=1e6,
                        dtype="bf16", qk_norm=True, qkv_bias=False, tied=False)
 
-# Qwen3 targets of the paper's scaling study (4B .. 32B with one frozen sidecar)
+# Qwen3 targets of the paper's scaling study (4B, 8B, 14B, 32B with one frozen sidecar)
 QWEN3_4B = ModelConfig("qwen3-4b", n_layers=36, hidden=2560, n_q_heads=32,
                        n_kv_heads=8, head_dim=128, intermediate=9728,
                        vocab=151936, rms_eps=1e-6, rope_theta=1e6,
@@ -86,6 +93,11 @@ QWEN3_4B = ModelConfig("qwen3-4b", n_layers=36, hidden=2560, n_q_heads=32,
 
 QWEN3_14B = ModelConfig("qwen3-14b", n_layers=40, hidden=5120, n_q_heads=40,
                         n_kv_heads=8, head_dim=128, intermediate=17408,
+                        vocab=151936, rms_eps=1e-6, rope_theta=1e6,
+                        dtype="bf16", qk_norm=True, qkv_bias=False, tied=False)
+
+QWEN3_32B = ModelConfig("qwen3-32b", n_layers=64, hidden=5120, n_q_heads=64,
+                        n_kv_heads=8, head_dim=128, intermediate=25600,
                         vocab=151936, rms_eps=1e-6, rope_theta=1e6,
                         dtype="bf16", qk_norm=True, qkv_bias=False, tied=False)
 
@@ -115,6 +127,8 @@ WORKLOADS = {
     "qwen3-4b": Workload(QWEN3_4B, ctx_len=2048, T=64, plant=10,
                          tree=dict(kind="branch", bmin=1, bmax=4, max_depth=12)),
     "qwen3-14b": Workload(QWEN3_14B, ctx_len=2048, T=64, plant=10,
+                          tree=dict(kind="branch", bmin=1, bmax=4, max_depth=12)),
+    "qwen3-32b": Workload(QWEN3_32B, ctx_len=2048, T=64, plant=10,
                           tree=dict(kind="branch", bmin=1, bmax=4, max_depth=12)),
 }
 

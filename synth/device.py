@@ -63,8 +63,9 @@ def upload_model(sm, device="cuda"):
 def upload_cache(cfg, native_layers, capacity, device="cuda"):
     """K and V device tensors [capacity, nkv, d] per layer; slots past the
     given prefix are zero."""
-    bf16 = cfg.dtype == "bf16"
-    dt = torch.bfloat16 if bf16 else torch.float32
+    f16 = getattr(cfg, "cache_dtype", "") == "f16"
+    bf16 = cfg.dtype == "bf16" or f16
+    dt = torch.float16 if f16 else (torch.bfloat16 if bf16 else torch.float32)
     ks, vs = [], []
     for k_np, v_np in native_layers:
         n = k_np.shape[0]
@@ -73,7 +74,7 @@ def upload_cache(cfg, native_layers, capacity, device="cuda"):
             t = torch.zeros(capacity, cfg.n_kv_heads, cfg.head_dim, dtype=dt, device=device)
             if n:
                 src = torch.from_numpy(np.ascontiguousarray(arr).view(np.int16) if bf16 else np.ascontiguousarray(arr))
-                t[:n].copy_((src.view(torch.bfloat16) if bf16 else src).to(device))
+                t[:n].copy_((src.view(dt) if bf16 else src).to(device))
             pair.append(t)
         ks.append(pair[0])
         vs.append(pair[1])

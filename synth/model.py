@@ -156,6 +156,11 @@ def synthetic_kv(cfg, seed, layer, n_pos, fmt="native", which="k"):
     kind = KV_K if which == "k" else KV_V
     key = gen.tensor_key(seed, kind, layer)
     n = n_pos * cfg.kv_dim
+    if getattr(cfg, "cache_dtype", "") == "f16":
+        # fp32 deviates rounded to IEEE binary16 (nearest even): uint16 bits or their fp64 values
+        h = gen.normal(key, n, 1.0, "f32").astype(np.float16)
+        out = h.view(np.uint16) if fmt == "native" else h.astype(np.float64)
+        return out.reshape(n_pos, cfg.n_kv_heads, cfg.head_dim)
     bf16 = cfg.dtype == "bf16"
     if fmt == "native":
         out = gen.normal(key, n, 1.0, "bf16" if bf16 else "f32")

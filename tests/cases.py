@@ -36,6 +36,9 @@ class Case:
 
 def round_cache(cfg, arr64):
     """Round a fp64 cache to the storage type; return (native, widened fp64)."""
+    if cfg.kv_dtype == "f16":
+        h = np.asarray(arr64, np.float32).astype(np.float16)
+        return h.view(np.uint16), h.astype(np.float64)
     if cfg.dtype == "f32":
         a32 = np.asarray(arr64, np.float32)
         return a32, a32.astype(np.float64)

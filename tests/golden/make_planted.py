@@ -10,7 +10,7 @@ near-tie could be decided either way by a bf16 verifier, so exact comparison of
 the accept outputs is only meaningful on such well-separated paths.
 
 Usage: python tests/golden/make_planted.py [workload ...]
-       python tests/golden/make_planted.py --roots N workload ...
+       python tests/golden/make_planted.py --roots N [--known i,j,...] workload ...
 
 The second form writes golden/gated_roots.json instead: for each workload,
 the first N roots of the seeded ROOT stream (weights seed 0, the workload's
@@ -81,9 +81,11 @@ def plant_one(name, seed=0):
     raise RuntimeError("no well-separated greedy path found for %s" % name)
 
 
-def gated_roots(name, n_cases, seed=0, max_roots=1024):
+def gated_roots(name, n_cases, seed=0, max_roots=1024, known=(), on_found=None):
     """The first n_cases roots of the seeded ROOT stream whose greedy path
-    (plant tokens and the bonus) is well separated."""
+    (plant tokens and the bonus) is well separated.  `known`: root indices
+    already found to qualify (checked again, and the search resumes after the
+    last of them); on_found(result) is called after every qualifying root."""
     w = workload(name)
     cfg = w.model
     model = SynthModel(cfg, seed)
@@ -94,17 +96,27 @@ def gated_roots(name, n_cases, seed=0, max_roots=1024):
         _, k64, v64 = synthetic_cache(cfg, seed, w.ctx_len)
     roots = gen.uniform_int(gen.tensor_key(seed, ROOT_KIND), max_roots, cfg.vocab)
     found = []
-    for k in range(max_roots):
+    known = sorted(int(k) for k in known)
+    order = known + list(range(known[-1] + 1 if known else 0, max_roots))
+
+    def result():
+        return dict(seed=seed, ctx_len=w.ctx_len, plant=w.plant, cases=list(found),
+                    note="roots of the seeded stream whose oracle greedy continuation (plant tokens and "
+                         "the bonus) has every top-1/top-2 margin > %.2f" % MIN_MARGIN)
+
+    for k in order:
         root = int(roots[k])
         toks, margins = _separated_path(view, k64, v64, w.ctx_len, root, w.plant)
         if len(toks) == w.plant + 1:
             found.append(dict(root_index=k, root=root, planted=toks[:w.plant], bonus=toks[w.plant],
                               margins=margins))
             print("  %s root #%d kept (%d so far)" % (name, k, len(found)), flush=True)
+            if on_found:
+                on_found(result())
             if len(found) == n_cases:
-                return dict(seed=seed, ctx_len=w.ctx_len, plant=w.plant, cases=found,
-                            note="roots of the seeded stream whose oracle greedy continuation (plant tokens and "
-                                 "the bonus) has every top-1/top-2 margin > %.2f" % MIN_MARGIN)
+                return result()
+        elif k in known:
+            raise RuntimeError("root #%d of %s no longer qualifies" % (k, name))
     raise RuntimeError("only %d well-separated roots for %s" % (len(found), name))
 
 
@@ -122,21 +134,31 @@ def main(names):
             json.dump(data, f, indent=1)
 
 
-def main_roots(n_cases, names):
+def main_roots(n_cases, names, known=()):
     data = {}
     if os.path.exists(ROOTS_OUT):
         with open(ROOTS_OUT) as f:
             data = json.load(f)
-    for name in names:
-        t0 = time.time()
-        data[name] = gated_roots(name, n_cases)
-        print(name, "%d roots" % n_cases, "%.0fs" % (time.time() - t0), flush=True)
+
+    def save(name, r):
+        data[name] = r
         with open(ROOTS_OUT, "w") as f:
             json.dump(data, f, indent=1)
+
+    for name in names:
+        t0 = time.time()
+        save(name, gated_roots(name, n_cases, known=known, on_found=lambda r: save(name, r)))
+        print(name, "%d roots" % n_cases, "%.0fs" % (time.time() - t0), flush=True)
 
 
 if __name__ == "__main__":
     if len(sys.argv) > 2 and sys.argv[1] == "--roots":
-        main_roots(int(sys.argv[2]), sys.argv[3:])
+        # --roots N [--known i,j,...] workload ...
+        args = sys.argv[3:]
+        known = ()
+        if args and args[0] == "--known":
+            known = [int(x) for x in args[1].split(",")]
+            args = args[2:]
+        main_roots(int(sys.argv[2]), args, known)
     else:
         main(sys.argv[1:] or [n for n, w in WORKLOADS.items() if w.model.dtype == "bf16"])

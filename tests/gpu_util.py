@@ -32,7 +32,7 @@ def to_f64(cfg, t):
 
 
 def _bits(t):
-    return t.view(torch.int16) if t.dtype == torch.bfloat16 else t.view(torch.int32)
+    return t.view(torch.int16) if t.element_size() == 2 else t.view(torch.int32)
 
 
 def run(model, kv, ctx, tokens, parent):
@@ -144,5 +144,4 @@ def check_compaction(model, kv, ctx, g):
             exp = snap.clone()
             for j, src in enumerate(path):
                 exp[ctx + j] = snap[ctx + src]
-            assert torch.equal(exp.view(torch.int16) if exp.dtype == torch.bfloat16 else exp.view(torch.int32),
-                               cur.view(torch.int16) if cur.dtype == torch.bfloat16 else cur.view(torch.int32))
+            assert torch.equal(_bits(exp), _bits(cur))

@@ -61,9 +61,10 @@ def _bank(seq, vocab, seed, n_views=8):
     return np.asarray(out, np.int32)
 
 
-@pytest.mark.parametrize("name,n_rounds,max_nodes", [("tiny", 12, 16), ("mini-bf16", 8, 32)])
-def test_decode_loop_matches_oracle_and_greedy(name, n_rounds, max_nodes):
-    case = build_case(name, 0)
+@pytest.mark.parametrize("name,n_rounds,max_nodes,overrides", [("tiny", 12, 16, None), ("mini-bf16", 8, 32, None),
+                                                                ("mini-bf16", 6, 24, dict(cache_dtype="f16"))])
+def test_decode_loop_matches_oracle_and_greedy(name, n_rounds, max_nodes, overrides):
+    case = build_case(name, 0, cfg_overrides=overrides)
     cfg = case.cfg
     gate = GATE[cfg.dtype]
     n_ref = n_rounds * max_nodes

@@ -314,6 +314,41 @@ def test_mini_bf16_variants(mini_models, overrides, gain_std):
     check_case(case, g, _oracle(case))
 
 
+@pytest.mark.parametrize("T,recipe,ctx", [
+    (7, dict(kind="uniform", max_depth=4), 200),
+    (50, dict(kind="uniform", max_depth=12), 65),
+    (128, dict(kind="branch", bmin=1, bmax=3, max_depth=30), 4600),
+    (12, dict(kind="uniform", max_depth=5), 0),
+])
+def test_mini_f16_cache_shapes(mini_models, T, recipe, ctx):
+    """FP16 KV cache under bf16 weights (the paper's Qwen2.5 / Llama backend):
+    the cache, the tree's K/V and the attention operands are binary16."""
+    case, model = _mini(mini_models, 1, T=T, recipe=recipe, ctx_len=ctx, plant=min(3, T - 1),
+                        cfg_overrides=dict(cache_dtype="f16"))
+    kv = gpu_cache(case, ctx + T)
+    assert kv.k[0].dtype == torch.float16
+    g = run(model, kv, ctx, case.tokens, case.parent)
+    check_case(case, g, _oracle(case))
+    check_compaction(model, kv, ctx, g)
+
+
+def test_mini_f16_cache_gated_seeds(mini_models):
+    gated = 0
+    for seed in range(4):
+        case, model = _mini(mini_models, seed, cfg_overrides=dict(cache_dtype="f16"))
+        kv = gpu_cache(case, case.ctx_len + 16)
+        g = run(model, kv, case.ctx_len, case.tokens, case.parent)
+        gated += check_case(case, g, _oracle(case))
+    assert gated >= 1
+
+
+def test_fp16_cache_rejected_for_fp32_models():
+    case = build_case("tiny", 0, cfg_overrides=dict(cache_dtype="f16"))
+    with pytest.raises(B.OosError) as e:
+        gpu_model(case)
+    assert e.value.code == B.OOS_EUNSUPPORTED
+
+
 # ------------------------------------------------------------------ bf16 decoders at the workload shapes
 
 def _bf16_case(name, T=None, ctx=None):
@@ -377,6 +412,44 @@ def test_bf16_qwen3_scaling_targets_sampled(name):
     """Qwen3 targets of the paper's scaling study: 4B (tied head, q width 4096
     over hidden 2560) and 14B (40/8 heads, hidden 5120)."""
     _sampled_check(name)
+
+
+def test_llama31_8b_fp16_cache_sampled():
+    """Llama-3.1-8B shape with the FP16 cache the paper runs it with: T=128 wide
+    tree over 8192 cached binary16 positions, sampled nodes against the oracle
+    (tensors at tolerance, argmax and accept outputs where the margins gate)."""
+    p = load_planted("llama3.1-8b")
+    case = build_case("llama3.1-8b", p["seed"], planted=(p["planted"], p["margins"]), root=p["root"],
+                      cfg_overrides=dict(cache_dtype="f16"))
+    model, _ = gpu_model(case)
+    kv = gpu_cache(case, case.ctx_len + case.tokens.shape[0])
+    assert kv.k[0].dtype == torch.float16
+    g = run(model, kv, case.ctx_len, case.tokens, case.parent)
+    T = len(case.tokens)
+    leaves = [i for i in range(T) if i not in set(case.parent[1:].tolist())]
+    rng = np.random.default_rng(9)
+    sample = [case.planted_path[-1]] + list(rng.choice(leaves, size=2, replace=False))
+    r = _oracle(case, only=sample)
+    check_case(case, g, r, rows=r["nodes"])
+    check_compaction(model, kv, case.ctx_len, g)
+
+
+def test_bf16_qwen3_32b_sampled():
+    """Qwen3-32B shape of the paper's scaling study (64 layers, hidden 5120,
+    64/8 heads, q/k norm, SwiGLU 25600; about 63 GB of bf16 weights): a random
+    tree of 64 nodes, sampled nodes against the oracle (tensors at tolerance,
+    argmax and accept outputs where the margins gate)."""
+    case = build_case("qwen3-32b", 0, plant=0)
+    model, _ = gpu_model(case)
+    kv = gpu_cache(case, case.ctx_len + case.tokens.shape[0])
+    g = run(model, kv, case.ctx_len, case.tokens, case.parent)
+    T = len(case.tokens)
+    leaves = [i for i in range(T) if i not in set(case.parent[1:].tolist())]
+    rng = np.random.default_rng(3)
+    sample = list(rng.choice(leaves, size=3, replace=False))
+    r = _oracle(case, only=sample)
+    check_case(case, g, r, rows=r["nodes"])
+    check_compaction(model, kv, case.ctx_len, g)
 
 
 def test_bf16_qwen25_32b_sampled():

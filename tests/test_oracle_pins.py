@@ -447,3 +447,51 @@ def test_bf16_layer0_tree_k_matches_library_restatement():
     k_rot = torch.cat([kc.real, kc.imag], dim=-1)
     ref = k_rot.to(torch.float32).to(torch.bfloat16).to(torch.float64).numpy()
     np.testing.assert_allclose(r["tree_k"][0], ref, rtol=0, atol=0)
+
+
+def _mini_f16_case(seed, T=7, ctx_len=12):
+    return build_case("mini-bf16", seed, T=T, recipe=dict(kind="uniform", max_depth=3), ctx_len=ctx_len, plant=0,
+                      cfg_overrides=dict(cache_dtype="f16"))
+
+
+def test_f16_cache_tree_kv_and_tree_equals_causal_decoding():
+    """FP16 cache (the paper's Qwen2.5 / Llama backend) under bf16 weights: the
+    cache and every K/V a node attends to are binary16, the tree pass equals
+    causal decoding along every path, and layer-0 K equals the library
+    restatement rounded by torch's own fp32 -> fp16 conversion."""
+    c = _mini_f16_case(7)
+    assert oracle.kv_format(c.cfg) == "f16" and c.cfg.dtype == "bf16"
+    for l in range(c.cfg.n_layers):   # the committed cache is binary16 values
+        np.testing.assert_array_equal(c.cache_k64[l].astype(np.float16).astype(np.float64), c.cache_k64[l])
+    r = oracle.verify_tree(c.view, c.cache_k64, c.cache_v64, c.ctx_len, c.tokens, c.parent)
+    for l in range(c.cfg.n_layers):
+        np.testing.assert_array_equal(r["tree_k"][l].astype(np.float16).astype(np.float64), r["tree_k"][l])
+        np.testing.assert_array_equal(r["tree_v"][l].astype(np.float16).astype(np.float64), r["tree_v"][l])
+    _, paths = oracle.tree_structure(c.parent)
+    leaves = [i for i in range(len(c.parent)) if i not in set(c.parent[1:].tolist())]
+    for leaf in leaves:
+        path = paths[leaf]
+        steps, _, _ = oracle.decode_sequence(c.view, c.cache_k64, c.cache_v64, c.ctx_len, c.tokens[path])
+        for j, node in enumerate(path):
+            np.testing.assert_allclose(r["final_hidden"][node], steps[j]["final_hidden"], rtol=1e-10, atol=1e-10)
+            for l in range(c.cfg.n_layers):
+                np.testing.assert_array_equal(r["tree_k"][l][node], steps[j]["k"][l])
+    W = c.view.layer(0)
+    cfg = c.cfg
+    depth, _ = oracle.tree_structure(c.parent)
+    x = torch.from_numpy(c.view.embed_rows(c.tokens))
+    h = F.rms_norm(x, (cfg.hidden,), torch.from_numpy(W["attn_norm"]), eps=cfg.rms_eps)
+    v = (h @ torch.from_numpy(W["w_v"]).T).reshape(len(c.tokens), cfg.n_kv_heads, cfg.head_dim)
+    np.testing.assert_array_equal(r["tree_v"][0], v.to(torch.float32).to(torch.float16).to(torch.float64).numpy())
+
+
+def test_f16_and_bf16_caches_differ_only_by_the_cache_rounding():
+    """Same weights, same tree: the two cache formats give final hiddens that
+    differ (the cache rounding changes), but by far less than the bf16
+    tolerance."""
+    a = _mini_case(9)
+    b = _mini_f16_case(9)
+    ra = oracle.verify_tree(a.view, a.cache_k64, a.cache_v64, a.ctx_len, a.tokens, a.parent)
+    rb = oracle.verify_tree(b.view, b.cache_k64, b.cache_v64, b.ctx_len, b.tokens, b.parent)
+    d = np.abs(ra["final_hidden"] - rb["final_hidden"]).max() / max(1.0, np.abs(ra["final_hidden"]).max())
+    assert 0.0 < d < 2e-2
