@@ -224,6 +224,60 @@ def job_throughput(T, ms, world):
     return world * T / (ms * 1e-3)
 
 
+# ---------------------------------------------------------------- other workloads
+
+OTHER_WORKLOADS = ("qwen3-0.6b", "llama3.1-8b", "qwen2.5-32b", "qwen3-4b", "qwen3-14b", "qwen3-32b")
+
+
+def time_workload(B, name, steps, warmup, peak):
+    """µs per verify + compaction step of another workload (graph replay,
+    inputs resident, weights far larger than L2 except for the 0.6B model,
+    whose 1.2 GB still exceed it)."""
+    import torch
+    from synth.device import upload_cache, upload_model
+    w = WORKLOADS[name]
+    cfg, T, ctx = w.model, w.T, w.ctx_len
+    seed, tokens_np, parent_np, _ = workload_tree(name)
+    weights = upload_model(SynthModel(cfg, seed))
+    native = [(synthetic_kv(cfg, seed, l, ctx, "native", "k"), synthetic_kv(cfg, seed, l, ctx, "native", "v"))
+              for l in range(cfg.n_layers)]
+    k, v = upload_cache(cfg, native, ctx + T)
+    del native
+    kv = B.KVCache(k, v)
+    model = B.OosModel(cfg, weights, max_T=T, use_graph=True)
+    stream = torch.cuda.current_stream()
+    tok = torch.as_tensor(tokens_np, dtype=torch.int32, device="cuda")
+    par = torch.as_tensor(parent_np, dtype=torch.int32, device="cuda")
+    outs = B.VerifyOutputs(T)
+
+    def step():
+        B.oos_tree_verify(model, kv, ctx, tok, par, T, outs.accepted_len, outs.accepted_nodes, outs.accepted_tokens,
+                          outs.bonus, stream)
+        B.oos_kv_compact(model, kv, ctx, outs.accepted_nodes, outs.accepted_len, T, stream)
+
+    for _ in range(max(warmup, 3)):
+        step()
+    torch.cuda.synchronize()
+    if B.oos_last_status(model) != B.OOS_OK:
+        raise RuntimeError("%s: verify status %s" % (name, B.oos_status_string(B.oos_last_status(model))))
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        step()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / steps
+    acc = int(outs.accepted_len.item())
+    model.close()
+    b = step_bytes(cfg, ctx, T)
+    res = {"config": "%s T=%d ctx_len=%d%s" % (name, T, ctx, " kv=f16" if cfg.kv_dtype == "f16" else ""),
+           "us_per_step": ms * 1e3, "tree_tokens_per_s": T / (ms * 1e-3), "step_gbs": b / (ms * 1e-3) / 1e9,
+           "step_frac_of_measured_hbm": b / (ms * 1e-3) / 1e9 / peak, "accepted_len": acc}
+    del weights, kv, k, v, model
+    torch.cuda.empty_cache()
+    return res
+
+
 # ---------------------------------------------------------------- decode loop
 
 def decode_leg(B, cfg, weights, native_cache, T, stream, n_vanilla=96, n_rounds=12, eos=2):
@@ -490,6 +544,14 @@ def run_ours(args):
     if not args.no_decode:
         decode = decode_leg(B, cfg, weights, native_cache=(seed, ctx), T=T, stream=stream)
 
+    # ---- the other workload shapes, one after another (N = 1 only)
+    workloads = None
+    if world == 1 and not args.no_workloads:
+        workloads = {}
+        for name in OTHER_WORKLOADS:
+            workloads[name] = time_workload(B, name, 10, 3, peak)
+            log("%s: %.1f us/step" % (name, workloads[name]["us_per_step"]))
+
     # ---- CPU checker on the host cores (rank 0, N = 1 only)
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
@@ -526,6 +588,7 @@ def run_ours(args):
             "prefill": prefill,
             "hint": hint,
             "decode": decode,
+            "workloads": workloads,
         }), flush=True)
     model.close()
     if world > 1:
@@ -544,6 +607,7 @@ def main():
     ap.add_argument("--no-prefill", action="store_true", help="skip the prefill measurement")
     ap.add_argument("--no-hint", action="store_true", help="skip the hint-bank step measurement")
     ap.add_argument("--no-decode", action="store_true", help="skip the decode-loop measurement")
+    ap.add_argument("--no-workloads", action="store_true", help="skip timing the other workload shapes")
     ap.add_argument("--layers", type=int, default=0,
                     help="profiling captures only: keep the first N layers of the workload's model")
     args = ap.parse_args()

@@ -211,7 +211,7 @@ OOS_DEV void shl128(unsigned long long lo, unsigned long long hi, int s, unsigne
 
 // sites of the bounded waits (recorded on the status word when one expires)
 enum { AW_KEMPTY = 21, AW_VEMPTY, AW_QTM, AW_KFULL, AW_SFREE, AW_PFULL, AW_VFULL, AW_SFULL, AW_PV_RESCALE,
-       AW_VZERO, AW_ODONE, AW_RECV };
+       AW_VZERO };
 OOS_DEV bool attn_wait(uint64_t* bar, uint32_t parity, volatile int* abort, uint32_t* status, uint32_t site, int ti) {
   if (mbar_wait(bar, parity, abort, status)) return true;
   if (*(volatile uint32_t*)(status + 1) == 0u && (*(volatile uint32_t*)status & ST_TIMEOUT))
@@ -368,11 +368,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
           asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(a.pf + o), "r"(len & ~15u) : "memory");
         }
       }
-      if (*abort_flag) {
-        // let this block's copies in flight land before it moves on
-        for (int ti = nk > 2 ? nk - 2 : 0; ti < nk; ++ti) drain_wait(&kfull[ti & 1], (uint32_t)(ti >> 1) & 1u);
-        for (int ti = nv > 2 ? nv - 2 : 0; ti < nv; ++ti) drain_wait(&vfull[ti & 1], (uint32_t)(ti >> 1) & 1u);
-      }
+      // every copy this thread issued has landed before the block can exit,
+      // whoever gave up (immediate on the normal path, where all were consumed)
+      for (int ti = nk > 2 ? nk - 2 : 0; ti < nk; ++ti) drain_wait(&kfull[ti & 1], (uint32_t)(ti >> 1) & 1u);
+      for (int ti = nv > 2 ? nv - 2 : 0; ti < nv; ++ti) drain_wait(&vfull[ti & 1], (uint32_t)(ti >> 1) & 1u);
+      drain_wait(qfull, 0);
     }
   } else if (warp == 1 || warp == 6) {
     // ------------------------------------------------------------ MMA issuers
@@ -581,8 +581,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
       __syncwarp();
       if (lane == 0) mbar_arrive(&pfull[b]);
     }
-    // every role is done with the rings and TMEM once all MMAs have completed
-    attn_wait(odone, 0, abort_flag, status, AW_ODONE, n_tiles);
+    // every role is done with the rings and TMEM once all MMAs have completed;
+    // both issuers always commit this barrier, and TMEM must not be released
+    // under a running MMA, so the wait is not cut short by the handle's limit
+    drain_wait(odone, 0);
   }
   tc_fence_before();
   __syncthreads();
@@ -626,8 +628,10 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
     }
     bulk_commit_and_wait_read();   // the staged rows have been read before this block moves on
   }
-  // this block's rows from every split
-  attn_wait(recv_full, 0, abort_flag, status, AW_RECV, 0);
+  // this block's rows from every split.  Every block copies its rows even
+  // after an abort, so this wait ends; it is not cut short by the handle's
+  // limit, because the block must not exit while copies into it are in flight.
+  drain_wait(recv_full, 0);
   {
     // split weights of every owned row: 2^(m_s - M) / sum_s 2^(m_s - M) l_s
     if (threadIdx.x < n_mine) {

@@ -286,6 +286,15 @@ OOS_DEV void finish_qkv(const GemmArgs& a, const Src& src, int tile, int nc, con
   const int m0 = 4 * (l & 15);      // rotary frequency index of this lane's first feature
   const bool first_half = l < 16;   // features 0..63 pair with 64..127 held by lane ^ 16
   for (int t0 = tb; t0 < te; t0 += nw * kFinRows) {
+    // the pass's rotary factors, loaded ahead of (and so together with) the partial sums
+    float2 cs[kFinRows][4];
+#pragma unroll
+    for (int k = 0; k < kFinRows; ++k) {
+      const int t = t0 + nw * k + w;
+#pragma unroll
+      for (int c = 0; c < 4; ++c)
+        cs[k][c] = (kind < 2 && t < te) ? __ldcg(a.rope + t * (kTile / 2) + m0 + c) : make_float2(1.f, 0.f);
+    }
     float4 acc[kFinRows];
     load_tile_rows<kFinRows, 8>(acc, src, nc, tile * kTile + 4 * l, t0, te, nullptr, 0, 0, w, nw);
 #pragma unroll
@@ -306,8 +315,7 @@ OOS_DEV void finish_qkv(const GemmArgs& a, const Src& src, int tile, int nc, con
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
           const float other = __shfl_xor_sync(0xffffffffu, v[c], 16);
-          const float2 cs = a.rope[t * (kTile / 2) + m0 + c];
-          v[c] = first_half ? v[c] * cs.x - other * cs.y : v[c] * cs.x + other * cs.y;
+          v[c] = first_half ? v[c] * cs[k][c].x - other * cs[k][c].y : v[c] * cs[k][c].x + other * cs[k][c].y;
         }
       }
       if (kind == 0) {   // q as hi/lo halves in the cache's 16-bit format: the attention product sees ~16-bit q
@@ -500,8 +508,9 @@ __global__ void __launch_bounds__(192, 1)
           }
         }
       }
-      if (*abort_flag) {
-        // let this CTA's copies in flight land before the CTA exits
+      {
+        // every copy this thread issued has landed before the CTA can exit,
+        // whoever gave up (immediate on the normal path, where all were consumed)
         const int first = issued - S > 0 ? issued - S : 0;
         for (int j = first; j < issued; ++j) {
           const unsigned long long t0 = globaltimer();
@@ -624,11 +633,31 @@ __global__ void __launch_bounds__(192, 1)
         for (int sub = 0; sub < kSub; ++sub) {
           float* dst = a.part + (size_t)(cta - c0) * kMaxT * n_part + (size_t)(wt * kSub + sub) * kTile + q * 32 +
                        (lane & ~3);
+          // the subtile's accumulator row in batches of TMEM loads (up to 64
+          // tokens, hi and lo products when paired), one wait per batch
+          constexpr int NG = BN / 16 < 4 ? BN / 16 : 4;   // 16-token chunks per batch
 #pragma unroll 1
-          for (int cc = 0; cc < BN / 16; ++cc) {
+          for (int c0g = 0; c0g < BN / 16; c0g += NG) {
+            if (c0g * 16 >= a.T) break;
+            float vv[NG][16], ww[C::PAIRED ? NG : 1][16];
+#pragma unroll
+            for (int k = 0; k < NG; ++k) {
+              tmem_ld16_nowait(taddr0 + sub * C::SUB_COLS + (c0g + k) * 16, vv[k]);
+              if (C::PAIRED) tmem_ld16_nowait(taddr0 + sub * C::SUB_COLS + BN + (c0g + k) * 16, ww[C::PAIRED ? k : 0]);
+            }
+            tmem_wait_ld();
+#pragma unroll
+            for (int k = 0; k < NG; ++k) {
+              reg_fence(vv[k]);
+              if (C::PAIRED) reg_fence(ww[C::PAIRED ? k : 0]);
+            }
+#pragma unroll
+          for (int k = 0; k < NG; ++k) {
+            const int cc = c0g + k;
             if (cc * 16 >= a.T) break;
             float v[16];
-            acc16(sub, cc, v);
+#pragma unroll
+            for (int i = 0; i < 16; ++i) v[i] = C::PAIRED ? vv[k][i] + ww[C::PAIRED ? k : 0][i] : vv[k][i];
 #pragma unroll
             for (int b = 0; b < 4; ++b) {
               float x0 = v[4 * b], x1 = v[4 * b + 1], x2 = v[4 * b + 2], x3 = v[4 * b + 3];
@@ -653,6 +682,7 @@ __global__ void __launch_bounds__(192, 1)
               const int t = cc * 16 + 4 * b + li;   // rows (lane & ~3) .. +3 of token t
               if (t < a.T) *reinterpret_cast<float4*>(dst + (size_t)t * n_part) = make_float4(x0, x1, x2, x3);
             }
+          }
           }
         }
         // accumulators drained: hand the TMEM buffer back to the MMA issuer

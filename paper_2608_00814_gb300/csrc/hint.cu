@@ -10,11 +10,10 @@
 // bank order, cut at the lane depth or before an EOS; a lane counts towards
 // the budget only when it creates a node.
 //
-// k_hint_match: one thread per bank position (a block per 256-position chunk,
-// grid-stride over chunks) computes the longest n whose suffix ends there, 0
-// when nothing follows, as one byte; the maximum of each chunk and of each run
-// of 256 chunks (a "span") is kept too, and the block maxima give the n of the
-// call.  k_hint_pack: one block descends the two summaries in bank order --
+// k_hint_match: for every bank position the longest n whose suffix ends
+// there (0 when nothing, or EOS, follows), as one byte; a warp per 256-position
+// chunk, 8 positions per lane; the maximum of each chunk and of each run of 256
+// chunks (a "span") is kept too, and the warp maxima give the n of the call.  k_hint_pack: one block descends the two summaries in bank order --
 // spans, then their chunks, then positions, 256 at a time, each level's hits
 // gathered in order by warp ballots -- so only spans and chunks that hold an
 // occurrence are read, and warp 0 inserts each lane into the tree held in
@@ -31,44 +30,81 @@ constexpr int kHintMaxN = 7;        // longest suffix tried
 constexpr int kHintThreads = 256;   // threads of both kernels
 
 // prefix_len_dev: the prefix length in device memory (the decode loop's
-// committed length), or nullptr to use prefix_len
+// committed length), or nullptr to use prefix_len.  Each warp takes one
+// 256-position chunk at a time (grid-stride over chunks), each lane 8
+// consecutive positions: the lane reads bank[p0 - 8, p0 + 16) (vector loads
+// when the bank is 16-byte aligned), computes the 8 match lengths, stores
+// them as 8 bytes, and the chunk maximum is a warp reduction -- no block
+// barrier.  vec: the bank address is 16-byte aligned.
 __global__ void __launch_bounds__(kHintThreads) k_hint_match(const int32_t* __restrict__ bank, int N, int eos,
                                                              const int32_t* __restrict__ prefix, int prefix_len,
-                                                             const int32_t* __restrict__ prefix_len_dev,
+                                                             const int32_t* __restrict__ prefix_len_dev, int vec,
                                                              uint8_t* __restrict__ mlen, uint8_t* __restrict__ cmax,
                                                              int* __restrict__ smax, int* __restrict__ best) {
   __shared__ int suf[kHintMaxN];
-  __shared__ int wmax[kHintThreads / 32];
   if (prefix_len_dev) prefix_len = *prefix_len_dev;
   const int nmax = prefix_len < kHintMaxN ? prefix_len : kHintMaxN;
-  // suf[nmax - 1] is y's last token, suf[nmax - 1 - j] the one j before it
-  if (threadIdx.x < nmax) suf[threadIdx.x] = prefix[prefix_len - nmax + threadIdx.x];
+  // suf[j] is the token j places before y's last token
+  if (threadIdx.x < nmax) suf[threadIdx.x] = prefix[prefix_len - 1 - threadIdx.x];
   __syncthreads();
-  const long long n_chunks = ((long long)N + kHintThreads - 1) / kHintThreads;
-  int bmax = 0;   // thread 0: this block's maximum
-  for (long long c = blockIdx.x; c < n_chunks; c += gridDim.x) {
-    const long long p = c * kHintThreads + threadIdx.x;
-    int m = 0;
-    // the next bank token must exist and not be EOS
-    if (p + 1 < N && bank[p + 1] != eos) {
-      while (m < nmax && p - m >= 0 && bank[p - m] == suf[nmax - 1 - m]) ++m;
-    }
-    if (p < N) mlen[p] = (uint8_t)m;
-    int cm = m;
+  int sfx[kHintMaxN];
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) cm = max(cm, __shfl_xor_sync(0xffffffffu, cm, o));
-    if ((threadIdx.x & 31) == 0) wmax[threadIdx.x >> 5] = cm;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      int b = 0;
-      for (int w = 0; w < kHintThreads / 32; ++w) b = max(b, wmax[w]);
-      cmax[c] = (uint8_t)b;
-      if (b > 0) atomicMax(&smax[c / kHintThreads], b);
-      bmax = max(bmax, b);
+  for (int j = 0; j < kHintMaxN; ++j) sfx[j] = j < nmax ? suf[j] : 0;
+  const int lane = threadIdx.x & 31;
+  const long long n_chunks = ((long long)N + kHintThreads - 1) / kHintThreads;
+  const long long n_warps = (long long)gridDim.x * (kHintThreads / 32);
+  int wbest = 0;
+  for (long long c = (long long)blockIdx.x * (kHintThreads / 32) + (threadIdx.x >> 5); c < n_chunks; c += n_warps) {
+    const long long p0 = c * kHintThreads + lane * 8;
+    int w[24];   // bank[p0 - 8 + i]; positions outside [0, N) are never compared
+    if (vec && p0 >= 8 && p0 + 16 <= N) {
+      const int4* src = reinterpret_cast<const int4*>(bank + p0 - 8);
+#pragma unroll
+      for (int q = 0; q < 6; ++q) {
+        const int4 v = __ldcs(src + q);
+        w[4 * q] = v.x;
+        w[4 * q + 1] = v.y;
+        w[4 * q + 2] = v.z;
+        w[4 * q + 3] = v.w;
+      }
+    } else {
+#pragma unroll
+      for (int i = 0; i < 24; ++i) {
+        const long long q = p0 - 8 + i;
+        w[i] = (q >= 0 && q < N) ? bank[q] : 0;
+      }
     }
-    __syncthreads();
+    uint32_t packed[2] = {0u, 0u};
+    int lmax = 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const long long p = p0 + i;
+      int m = 0;
+      // the next bank token must exist and not be EOS
+      if (p + 1 < N && w[9 + i] != eos) {
+#pragma unroll
+        for (int j = 0; j < kHintMaxN; ++j) {
+          if (m < j || j >= nmax || p - j < 0 || w[8 + i - j] != sfx[j]) break;
+          m = j + 1;
+        }
+      }
+      packed[i >> 2] |= (uint32_t)m << (8 * (i & 3));
+      lmax = m > lmax ? m : lmax;
+    }
+    if (p0 + 8 <= N) {
+      *reinterpret_cast<uint2*>(mlen + p0) = make_uint2(packed[0], packed[1]);
+    } else {
+      for (int i = 0; i < 8 && p0 + i < N; ++i) mlen[p0 + i] = (uint8_t)((packed[i >> 2] >> (8 * (i & 3))) & 255u);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) lmax = max(lmax, __shfl_xor_sync(0xffffffffu, lmax, o));
+    if (lane == 0) {
+      cmax[c] = (uint8_t)lmax;
+      if (lmax > 0) atomicMax(&smax[c / kHintThreads], lmax);
+    }
+    wbest = max(wbest, lmax);
   }
-  if (threadIdx.x == 0 && bmax > 0) atomicMax(best, bmax);
+  if (lane == 0 && wbest > 0) atomicMax(best, wbest);
 }
 
 // Whole block: the values of the threads whose `has` is set, in thread order,
@@ -256,8 +292,11 @@ cudaError_t launch_hint_tree(const int32_t* bank, int N, int eos, const int32_t*
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
   cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const int grid = (int)(n_chunks < (long long)sms * 8 ? n_chunks : (long long)sms * 8);
-  k_hint_match<<<grid, kHintThreads, 0, st>>>(bank, N, eos, prefix, prefix_len, prefix_len_dev, mlen, cmax, smax,
+  // one warp per 256-position chunk; enough blocks for every SM to hold several
+  const long long want = (n_chunks + kHintThreads / 32 - 1) / (kHintThreads / 32);
+  const int grid = (int)(want < (long long)sms * 8 ? want : (long long)sms * 8);
+  const int vec = ((uintptr_t)bank & 15) == 0 ? 1 : 0;
+  k_hint_match<<<grid, kHintThreads, 0, st>>>(bank, N, eos, prefix, prefix_len, prefix_len_dev, vec, mlen, cmax, smax,
                                               best);
   e = cudaGetLastError();
   if (e != cudaSuccess) return e;

@@ -464,7 +464,9 @@ __global__ void __launch_bounds__(1024) k_argmax_accept(const float* __restrict_
   if (threadIdx.x < 32) {
     int n_valid = n_valid_dev ? *n_valid_dev : T;
     n_valid = n_valid < 1 ? 1 : (n_valid > T ? T : n_valid);
-    accept_walk_warp(s_tok, s_par, s_dep, s_arg, T, n_valid, (*status & ST_TREE) != 0, len, nodes, toks, bonus);
+    // a malformed tree or a pipeline wait that gave up: no accepted path
+    accept_walk_warp(s_tok, s_par, s_dep, s_arg, T, n_valid, (*status & (ST_TREE | ST_TIMEOUT)) != 0, len, nodes,
+                     toks, bonus);
   }
 }
 
