@@ -93,8 +93,6 @@ struct AttnArgs {
   __nv_bfloat16* out;       // [T][nq*d] hi rows, lo rows at out_lo_off
   size_t out_lo_off;
   uint32_t* status;         // step status word (pipeline waits that give up)
-  const unsigned char* pf;  // bytes to warm in L2 meanwhile (the next GEMM's weights; may be null)
-  size_t pf_bytes;
 };
 
 OOS_DEV uint32_t cluster_rank() {
@@ -354,19 +352,6 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
         if (!attn_wait(&vempty[st], (use & 1u) ^ 1u, abort_flag, status, AW_VEMPTY, ti)) break;
         load(ti, true);
         ++nv;
-      }
-      // HBM is nearly idle for the rest of the attention: pull this block's
-      // share of the next GEMM's weights into L2 (after this block's own loads)
-      if (a.pf && !*abort_flag) {
-        const size_t nb = (size_t)gridDim.x * gridDim.y * gridDim.z;
-        const size_t bid = blockIdx.x + (size_t)gridDim.x * (blockIdx.y + (size_t)gridDim.y * blockIdx.z);
-        const size_t per = ((a.pf_bytes + nb - 1) / nb + 4095) & ~(size_t)4095;
-        const size_t b0 = bid * per;
-        const size_t b1 = b0 + per < a.pf_bytes ? b0 + per : a.pf_bytes;
-        for (size_t o = b0; o < b1; o += 65536) {
-          const uint32_t len = (uint32_t)((b1 - o) < 65536 ? (b1 - o) : 65536);
-          asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(a.pf + o), "r"(len & ~15u) : "memory");
-        }
       }
       // every copy this thread issued has landed before the block can exit,
       // whoever gave up (immediate on the normal path, where all were consumed)
@@ -836,9 +821,6 @@ cudaError_t launch_attention(Model& m, int layer, const void* kc, const void* vc
   a.out = (__nv_bfloat16*)m.ws.attn;
   a.out_lo_off = (size_t)kMaxT * c.n_q_heads * kAttnD;
   a.status = m.ws.status;
-  // the O-projection weights of this layer, [H][nq*d] bf16, contiguous
-  a.pf = (const unsigned char*)m.layers[layer].w_o;
-  a.pf_bytes = (size_t)c.hidden * c.n_q_heads * kAttnD * 2;
 
   cudaLaunchConfig_t lc = {};
   lc.gridDim = dim3(RB, c.n_kv_heads, a.splits);

@@ -226,11 +226,6 @@ OOS_DEV void tma_load_4d(void* smem_dst, const void* tmap, uint64_t* bar, int x,
       "l"(reinterpret_cast<uint64_t>(tmap)), "r"(x), "r"(y), "r"(z), "r"(w), "r"(smem_addr(bar)), "l"(policy)
       : "memory");
 }
-OOS_DEV void tma_prefetch_l2(const void* tmap, int x, int y) {
-  asm volatile("cp.async.bulk.prefetch.tensor.2d.L2.global.tile [%0, {%1, %2}];" ::"l"(reinterpret_cast<uint64_t>(tmap)),
-               "r"(x), "r"(y)
-               : "memory");
-}
 
 // ---- tcgen05 (5th-generation tensor cores, accumulators in TMEM)
 OOS_DEV void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }

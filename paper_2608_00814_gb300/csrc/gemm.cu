@@ -83,10 +83,6 @@ struct GemmArgs {
   float* am_v1;
   int32_t* am_i;
   float* am_v2;
-  // L2 prefetch, during this GEMM's tail, of the next weight GEMM's first units
-  int pf_units;       // units per CTA of the next GEMM (0: no prefetch)
-  int pf_n_tiles, pf_n_work, pf_kbt, pf_total, pf_grid, pf_sub, pf_interleave, pf_round_robin;
-  int pf_seg_tiles[3];
 };
 
 template <int BN, int kSub>
@@ -345,9 +341,7 @@ OOS_DEV void finish_qkv(const GemmArgs& a, const Src& src, int tile, int nc, con
 template <int BN, int EPI>
 __global__ void __launch_bounds__(192, 1)
     k_gemm_tc(const __grid_constant__ CUtensorMap wm0, const __grid_constant__ CUtensorMap wm1,
-              const __grid_constant__ CUtensorMap wm2, const __grid_constant__ CUtensorMap am,
-              const __grid_constant__ CUtensorMap pm0, const __grid_constant__ CUtensorMap pm1,
-              const __grid_constant__ CUtensorMap pm2, GemmArgs a) {
+              const __grid_constant__ CUtensorMap wm2, const __grid_constant__ CUtensorMap am, GemmArgs a) {
   constexpr int kSub = SubOf<EPI>::v;
   using C = TcCfg<BN, kSub>;
   constexpr int S = C::S;
@@ -474,38 +468,6 @@ __global__ void __launch_bounds__(192, 1)
         if (++stage == S) {
           stage = 0;
           phase ^= 1u;
-        }
-      }
-      if (!*abort_flag && a.pf_units > 0) {
-        // HBM goes idle during this GEMM's tail (reductions in L2): warm L2
-        // with the first units the next weight GEMM's CTAs will stream
-        for (int c2 = cta; c2 < a.pf_grid; c2 += G) {
-          const long long v0 = a.pf_round_robin ? 0 : (long long)c2 * a.pf_total / a.pf_grid;
-          const long long v1 = a.pf_round_robin ? (long long)a.pf_units : (long long)(c2 + 1) * a.pf_total / a.pf_grid;
-          for (long long v = v0; v < v1 && v < v0 + a.pf_units; ++v) {
-            const int wt = a.pf_round_robin ? c2 + (int)(v / a.pf_kbt) * a.pf_grid : (int)(v / a.pf_kbt);
-            const int kb = (int)(v % a.pf_kbt);
-            if (wt >= a.pf_n_work) break;
-            for (int sub = 0; sub < a.pf_sub; ++sub) {
-              const int tile = wt * a.pf_sub + sub;
-              if (tile >= a.pf_n_tiles) break;
-              const CUtensorMap* pm = &pm0;
-              int row = tile * kTile;
-              if (a.pf_interleave) {
-                pm = (tile & 1) ? &pm1 : &pm0;
-                row = (tile >> 1) * kTile;
-              } else if (tile >= a.pf_seg_tiles[0]) {
-                if (tile >= a.pf_seg_tiles[1]) {
-                  pm = &pm2;
-                  row = (tile - a.pf_seg_tiles[1]) * kTile;
-                } else {
-                  pm = &pm1;
-                  row = (tile - a.pf_seg_tiles[0]) * kTile;
-                }
-              }
-              tma_prefetch_l2(pm, kb * kBK, row);
-            }
-          }
         }
       }
       {
@@ -910,38 +872,22 @@ cudaError_t gemm_setup() {
 
 template <int BN, int EPI>
 static cudaError_t launch_tc(Model& m, const GemmW& g, const CUtensorMap& amap, int grid, const GemmArgs& a,
-                             const GemmW* next, cudaStream_t st) {
+                             cudaStream_t st) {
   const CUtensorMap& w1 = g.n_seg > 1 ? g.map[1] : g.map[0];
   const CUtensorMap& w2 = g.n_seg > 2 ? g.map[2] : g.map[0];
-  const GemmW& p = next ? *next : g;
-  const CUtensorMap& p1 = p.n_seg > 1 ? p.map[1] : p.map[0];
-  const CUtensorMap& p2 = p.n_seg > 2 ? p.map[2] : p.map[0];
   return launch(m.pdl, k_gemm_tc<BN, EPI>, dim3(grid), dim3(192), (size_t)TcCfg<BN, SubOf<EPI>::v>::SMEM, st,
-                g.map[0], w1, w2, amap, p.map[0], p1, p2, a);
+                g.map[0], w1, w2, amap, a);
 }
 
 template <int EPI>
 static cudaError_t dispatch_tc(Model& m, const GemmW& g, const CUtensorMap* amaps, int T, int grid, GemmArgs& a,
-                               const GemmW* next, cudaStream_t st) {
+                               cudaStream_t st) {
   const int bi = bn_index(T);
-  if (next) {
-    // about 64 KB of the next GEMM's weights per CTA index
-    a.pf_units = 4 / next->sub;
-    a.pf_n_tiles = (next->N + kTile - 1) / kTile;
-    a.pf_n_work = next->plan.n_tiles;
-    a.pf_kbt = next->plan.kbt;
-    a.pf_total = next->plan.total;
-    a.pf_grid = next->plan.grid;
-    a.pf_sub = next->sub;
-    a.pf_interleave = next->interleave2;
-    a.pf_round_robin = next->round_robin;
-    for (int s = 0; s < 3; ++s) a.pf_seg_tiles[s] = next->seg_tiles[s < next->n_seg ? s : next->n_seg - 1];
-  }
   switch (bi) {
-    case 0: return launch_tc<16, EPI>(m, g, amaps[0], grid, a, next, st);
-    case 1: return launch_tc<32, EPI>(m, g, amaps[1], grid, a, next, st);
-    case 2: return launch_tc<64, EPI>(m, g, amaps[2], grid, a, next, st);
-    default: return launch_tc<128, EPI>(m, g, amaps[3], grid, a, next, st);
+    case 0: return launch_tc<16, EPI>(m, g, amaps[0], grid, a, st);
+    case 1: return launch_tc<32, EPI>(m, g, amaps[1], grid, a, st);
+    case 2: return launch_tc<64, EPI>(m, g, amaps[2], grid, a, st);
+    default: return launch_tc<128, EPI>(m, g, amaps[3], grid, a, st);
   }
 }
 
@@ -968,7 +914,7 @@ static GemmArgs base_args(Model& m, const GemmW& g, int T, int* cnt) {
   return a;
 }
 
-cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int T, const GemmW* next, cudaStream_t st) {
+cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int T, cudaStream_t st) {
   const auto& c = m.cfg;
   const oos_layer_weights& L = m.layers[layer];
   GemmArgs a = base_args(m, m.g_qkv[layer], T, gemm_counters(m, layer, 0));
@@ -985,34 +931,33 @@ cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int T, cons
   a.vc = (__nv_bfloat16*)vc;
   a.ctx = m.ws.ctx;
   a.kv_f16 = c.kv_f16 ? 1 : 0;
-  return dispatch_tc<EPI_QKV>(m, m.g_qkv[layer], m.amap_xn, T, m.g_qkv[layer].plan.grid, a, next, st);
+  return dispatch_tc<EPI_QKV>(m, m.g_qkv[layer], m.amap_xn, T, m.g_qkv[layer].plan.grid, a, st);
 }
 
 static cudaError_t launch_resid(Model& m, const GemmW& g, const CUtensorMap* amaps, const void* gain, int* cnt, int T,
-                                const GemmW* next, cudaStream_t st) {
+                                cudaStream_t st) {
   GemmArgs a = base_args(m, g, T, cnt);
   a.x = m.ws.x;
   a.gain = (const __nv_bfloat16*)gain;
   a.y_out = (__nv_bfloat16*)m.ws.xn;
   a.ss_out = m.ws.ss;
-  return dispatch_tc<EPI_RESID>(m, g, amaps, T, g.plan.grid, a, next, st);
+  return dispatch_tc<EPI_RESID>(m, g, amaps, T, g.plan.grid, a, st);
 }
 
-cudaError_t launch_gemm_o(Model& m, int layer, int T, const GemmW* next, cudaStream_t st) {
-  return launch_resid(m, m.g_o[layer], m.amap_attn, m.layers[layer].mlp_norm, gemm_counters(m, layer, 1), T, next,
-                      st);
+cudaError_t launch_gemm_o(Model& m, int layer, int T, cudaStream_t st) {
+  return launch_resid(m, m.g_o[layer], m.amap_attn, m.layers[layer].mlp_norm, gemm_counters(m, layer, 1), T, st);
 }
 
-cudaError_t launch_gemm_down(Model& m, int layer, int T, const GemmW* next, cudaStream_t st) {
+cudaError_t launch_gemm_down(Model& m, int layer, int T, cudaStream_t st) {
   const void* gain = layer + 1 < m.cfg.n_layers ? m.layers[layer + 1].attn_norm : m.w.final_norm;
-  return launch_resid(m, m.g_down[layer], m.amap_act, gain, gemm_counters(m, layer, 3), T, next, st);
+  return launch_resid(m, m.g_down[layer], m.amap_act, gain, gemm_counters(m, layer, 3), T, st);
 }
 
-cudaError_t launch_gemm_gu(Model& m, int layer, int T, const GemmW* next, cudaStream_t st) {
+cudaError_t launch_gemm_gu(Model& m, int layer, int T, cudaStream_t st) {
   GemmArgs a = base_args(m, m.g_gu[layer], T, gemm_counters(m, layer, 2));
   a.act_out = (__nv_bfloat16*)m.ws.act;
   a.I = m.cfg.intermediate;
-  return dispatch_tc<EPI_SILU>(m, m.g_gu[layer], m.amap_xn, T, m.g_gu[layer].plan.grid, a, next, st);
+  return dispatch_tc<EPI_SILU>(m, m.g_gu[layer], m.amap_xn, T, m.g_gu[layer].plan.grid, a, st);
 }
 
 cudaError_t launch_lm_head_tc(Model& m, int T, cudaStream_t st) {
@@ -1020,7 +965,7 @@ cudaError_t launch_lm_head_tc(Model& m, int T, cudaStream_t st) {
   a.am_v1 = m.ws.lm_v1;
   a.am_i = m.ws.lm_i;
   a.am_v2 = m.ws.lm_v2;
-  return dispatch_tc<EPI_ARGMAX>(m, m.g_lm, m.amap_xn, T, m.lm_grid, a, nullptr, st);
+  return dispatch_tc<EPI_ARGMAX>(m, m.g_lm, m.amap_xn, T, m.lm_grid, a, st);
 }
 
 // ------------------------------------------------------------ fp32 CUDA-core path

@@ -94,13 +94,17 @@ struct Workspace {
   int32_t* pf_scratch;       // prefill's unused accept outputs: len, bonus, nodes[kMaxT], tokens[kMaxT]
 };
 
-// shape + addresses a captured verify graph was recorded with
+// shape + addresses a captured verify graph was recorded with.  The committed
+// length is not part of it: only the tree-prep kernel takes it as an argument
+// (every later kernel reads it from ws.ctx), so a call at another length
+// updates that one node.  What the length does decide on the host, the
+// attention's key-split count, is.
 struct GraphKey {
   unsigned long long kv_hash;   // FNV-1a over every layer's K and V pointer
-  int capacity, ctx_len, T;
+  int capacity, splits, T;
   const void* io[10];
   bool operator==(const GraphKey& o) const {
-    if (kv_hash != o.kv_hash || capacity != o.capacity || ctx_len != o.ctx_len || T != o.T) return false;
+    if (kv_hash != o.kv_hash || capacity != o.capacity || splits != o.splits || T != o.T) return false;
     for (int i = 0; i < 10; ++i)
       if (io[i] != o.io[i]) return false;
     return true;
@@ -135,7 +139,10 @@ struct Model {
   StreamK p_qkv, p_o, p_gu, p_down;
   // CUDA graph of the last call shape
   cudaStream_t cap_stream = nullptr;
+  cudaGraph_t graph = nullptr;          // the graph gexec was instantiated from
   cudaGraphExec_t gexec = nullptr;
+  cudaGraphNode_t prep_node = nullptr;  // its tree-prep kernel node
+  int g_ctx = -1;                       // committed length that node was last given
   GraphKey gkey{};
   bool have_graph = false;
 };
@@ -163,6 +170,10 @@ inline cudaError_t launch(bool pdl, void (*kernel)(KArgs...), dim3 grid, dim3 bl
 // ctx from the host, or from device memory when ctx_dev is not null
 cudaError_t launch_tree_prep(Model& m, const int32_t* tokens, const int32_t* parent, int T, int ctx,
                              const int32_t* ctx_dev, cudaStream_t st);
+// the tree-prep kernel node of a captured graph, and a new committed length for it
+cudaGraphNode_t find_tree_prep_node(cudaGraph_t g);
+cudaError_t set_tree_prep_ctx(Model& m, cudaGraphExec_t ex, cudaGraphNode_t node, const int32_t* tokens,
+                              const int32_t* parent, int T, int ctx);
 cudaError_t launch_embed_norm(Model& m, const int32_t* tokens, int T, cudaStream_t st);
 cudaError_t launch_embed_tc(Model& m, const int32_t* tokens, int T, cudaStream_t st);
 cudaError_t launch_final_hidden(Model& m, float* hidden, int T, cudaStream_t st);
@@ -191,12 +202,10 @@ bool encode_bf16_map(CUtensorMap* map, const void* ptr, int rank, const uint64_t
 bool encode_act_map(CUtensorMap* map, const void* ptr, int K, int box_rows);
 int bn_index(int T);   // N-tile variant for T tree nodes: 0..3 -> 16/32/64/128
 cudaError_t gemm_setup();
-// `next`: the weight GEMM that follows; its first stages are prefetched into L2
-// during this GEMM's tail (nullptr: none)
-cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int T, const GemmW* next, cudaStream_t st);
-cudaError_t launch_gemm_o(Model& m, int layer, int T, const GemmW* next, cudaStream_t st);
-cudaError_t launch_gemm_gu(Model& m, int layer, int T, const GemmW* next, cudaStream_t st);
-cudaError_t launch_gemm_down(Model& m, int layer, int T, const GemmW* next, cudaStream_t st);
+cudaError_t launch_gemm_qkv(Model& m, int layer, void* kc, void* vc, int T, cudaStream_t st);
+cudaError_t launch_gemm_o(Model& m, int layer, int T, cudaStream_t st);
+cudaError_t launch_gemm_gu(Model& m, int layer, int T, cudaStream_t st);
+cudaError_t launch_gemm_down(Model& m, int layer, int T, cudaStream_t st);
 cudaError_t launch_lm_head_tc(Model& m, int T, cudaStream_t st);
 int* gemm_counters(Model& m, int layer, int kind);   // kind 0 qkv, 1 o, 2 gate/up, 3 down
 cudaError_t launch_gemm_f32(Model& m, const void* w0, const void* w1, const void* w2, int rows0, int rows1,

@@ -185,12 +185,11 @@ static int enqueue_layers(Model& m, const oos_kv_cache* kv, int ctx, const int32
     float* hid = (l + 1 < L) ? nullptr : hidden;
     if (c.dtype == OOS_DTYPE_BF16) {
       // five kernels per layer; every elementwise step runs in a GEMM epilogue
-      const GemmW* after_down = (l + 1 < L) ? &m.g_qkv[l + 1] : &m.g_lm;
-      OOS_TRY(launch_gemm_qkv(m, l, kv->k[l], kv->v[l], T, &m.g_o[l], st));
+      OOS_TRY(launch_gemm_qkv(m, l, kv->k[l], kv->v[l], T, st));
       OOS_TRY(launch_attention(m, l, kv->k[l], kv->v[l], kv->capacity, ctx_hint, T, st));
-      OOS_TRY(launch_gemm_o(m, l, T, &m.g_gu[l], st));
-      OOS_TRY(launch_gemm_gu(m, l, T, &m.g_down[l], st));
-      OOS_TRY(launch_gemm_down(m, l, T, after_down, st));
+      OOS_TRY(launch_gemm_o(m, l, T, st));
+      OOS_TRY(launch_gemm_gu(m, l, T, st));
+      OOS_TRY(launch_gemm_down(m, l, T, st));
     } else {
       OOS_TRY(launch_gemm_f32(m, W.w_q, W.w_k, W.w_v, qd, kvd, kvd, c.hidden, m.ws.xn, T, st));
       OOS_TRY(launch_qkv_post(m, l, m.p_qkv, kv->k[l], kv->v[l], T, st));
@@ -273,11 +272,29 @@ static int verify_impl(oos_model* mp, const oos_kv_cache* kv, int32_t ctx, const
   GraphKey key;
   key.kv_hash = kv_hash(kv);
   key.capacity = kv->capacity;
-  key.ctx_len = ctx;
+  key.splits = m.cfg.dtype == OOS_DTYPE_BF16 ? attn_splits(m, ctx, T) : 0;
   key.T = T;
   const void* io[10] = {tokens, parent, len, nodes, toks, bonus, hidden, dbg_arg, dbg_t1, dbg_t2};
   for (int i = 0; i < 10; ++i) key.io[i] = io[i];
-  if (!(m.have_graph && key == m.gkey)) {
+  bool capture = !(m.have_graph && key == m.gkey);
+  if (!capture && ctx != m.g_ctx) {
+    // same graph at another committed length: only the tree-prep node changes
+    if (set_tree_prep_ctx(m, m.gexec, m.prep_node, tokens, parent, T, ctx) == cudaSuccess) {
+      m.g_ctx = ctx;
+    } else {
+      cudaGetLastError();
+      capture = true;
+    }
+  }
+  if (capture) {
+    // a new shape or new buffers: capture again and instantiate afresh (the
+    // tree-prep node handle must come from the graph the executable was made from)
+    m.have_graph = false;
+    if (m.gexec) cudaGraphExecDestroy(m.gexec);
+    if (m.graph) cudaGraphDestroy(m.graph);
+    m.gexec = nullptr;
+    m.graph = nullptr;
+    m.prep_node = nullptr;
     cudaGraph_t graph = nullptr;
     OOS_TRY(cudaStreamBeginCapture(m.cap_stream, cudaStreamCaptureModeThreadLocal));
     int rc = enqueue_verify(m, kv, ctx, nullptr, tokens, parent, T, nullptr, len, nodes, toks, bonus, hidden, dbg_arg,
@@ -287,25 +304,16 @@ static int verify_impl(oos_model* mp, const oos_kv_cache* kv, int32_t ctx, const
       if (graph) cudaGraphDestroy(graph);
       return rc != OOS_OK ? rc : OOS_ECUDA;
     }
-    bool updated = false;
-    if (m.gexec) {
-      cudaGraphExecUpdateResultInfo info;
-      updated = cudaGraphExecUpdate(m.gexec, graph, &info) == cudaSuccess;
-      if (!updated) {
-        cudaGetLastError();
-        cudaGraphExecDestroy(m.gexec);
-        m.gexec = nullptr;
-      }
+    cudaGraphNode_t prep = find_tree_prep_node(graph);
+    if (!prep || cudaGraphInstantiate(&m.gexec, graph, 0) != cudaSuccess) {
+      cudaGetLastError();
+      cudaGraphDestroy(graph);
+      m.gexec = nullptr;
+      return OOS_ECUDA;
     }
-    if (!updated) {
-      if (cudaGraphInstantiate(&m.gexec, graph, 0) != cudaSuccess) {
-        cudaGraphDestroy(graph);
-        m.gexec = nullptr;
-        m.have_graph = false;
-        return OOS_ECUDA;
-      }
-    }
-    cudaGraphDestroy(graph);
+    m.graph = graph;
+    m.prep_node = prep;
+    m.g_ctx = ctx;
     m.gkey = key;
     m.have_graph = true;
   }
@@ -464,6 +472,7 @@ int oos_model_create(const oos_model_config* cfg, const oos_weights* w, void* wo
 int oos_model_destroy(oos_model* m) {
   if (!m) return OOS_EINVAL;
   if (m->gexec) cudaGraphExecDestroy(m->gexec);
+  if (m->graph) cudaGraphDestroy(m->graph);
   if (m->cap_stream) cudaStreamDestroy(m->cap_stream);
   delete m;
   return OOS_OK;
@@ -539,9 +548,9 @@ int oos_launch_stage(oos_model* m, int32_t layer, int32_t stage, int32_t T, void
         const int kind = stage == OOS_STAGE_O ? 1 : stage == OOS_STAGE_GATE_UP ? 2 : 3;
         e = cudaMemsetAsync(gemm_counters(*m, layer, kind), 0, kCntPer * sizeof(int), st);
         if (e != cudaSuccess) break;
-        e = stage == OOS_STAGE_O ? launch_gemm_o(*m, layer, T, nullptr, st)
-            : stage == OOS_STAGE_GATE_UP ? launch_gemm_gu(*m, layer, T, nullptr, st)
-                                         : launch_gemm_down(*m, layer, T, nullptr, st);
+        e = stage == OOS_STAGE_O ? launch_gemm_o(*m, layer, T, st)
+            : stage == OOS_STAGE_GATE_UP ? launch_gemm_gu(*m, layer, T, st)
+                                         : launch_gemm_down(*m, layer, T, st);
         break;
       }
       default: e = launch_lm_head_tc(*m, T, st); break;

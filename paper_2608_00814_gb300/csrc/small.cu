@@ -3,6 +3,8 @@
 // merge with the greedy-acceptance walk, and KV compaction.
 #include <math.h>
 
+#include <vector>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -67,6 +69,41 @@ cudaError_t launch_tree_prep(Model& m, const int32_t* tokens, const int32_t* par
                              const int32_t* ctx_dev, cudaStream_t st) {
   return launch(false, k_tree_prep, dim3(1), dim3(kMaxT), 0, st, tokens, parent, T, ctx, ctx_dev, m.ws.ctx,
                 m.cfg.vocab, m.ws.status, m.ws.depth, m.ws.pos, m.ws.anc);
+}
+
+cudaGraphNode_t find_tree_prep_node(cudaGraph_t g) {
+  size_t n = 0;
+  if (cudaGraphGetNodes(g, nullptr, &n) != cudaSuccess || n == 0) return nullptr;
+  std::vector<cudaGraphNode_t> nodes(n);
+  if (cudaGraphGetNodes(g, nodes.data(), &n) != cudaSuccess) return nullptr;
+  for (size_t i = 0; i < n; ++i) {
+    cudaGraphNodeType t;
+    if (cudaGraphNodeGetType(nodes[i], &t) != cudaSuccess || t != cudaGraphNodeTypeKernel) continue;
+    cudaKernelNodeParams p;
+    if (cudaGraphKernelNodeGetParams(nodes[i], &p) != cudaSuccess) continue;
+    if (p.func == (void*)k_tree_prep) return nodes[i];
+  }
+  return nullptr;
+}
+
+// the same arguments launch_tree_prep passes, with another committed length
+cudaError_t set_tree_prep_ctx(Model& m, cudaGraphExec_t ex, cudaGraphNode_t node, const int32_t* tokens,
+                              const int32_t* parent, int T, int ctx) {
+  const int32_t* ctx_in = nullptr;
+  int32_t* ctx_out = m.ws.ctx;
+  int vocab = m.cfg.vocab;
+  uint32_t* status = m.ws.status;
+  int32_t* depth = m.ws.depth;
+  int32_t* pos = m.ws.pos;
+  unsigned long long* anc = m.ws.anc;
+  void* args[] = {&tokens, &parent, &T, &ctx, &ctx_in, &ctx_out, &vocab, &status, &depth, &pos, &anc};
+  cudaKernelNodeParams p = {};
+  p.func = (void*)k_tree_prep;
+  p.gridDim = dim3(1);
+  p.blockDim = dim3(kMaxT);
+  p.sharedMemBytes = 0;
+  p.kernelParams = args;
+  return cudaGraphExecKernelNodeSetParams(ex, node, &p);
 }
 
 // ============================================================ embedding + first RMSNorm

@@ -35,23 +35,24 @@ def _bits(t):
     return t.view(torch.int16) if t.element_size() == 2 else t.view(torch.int32)
 
 
-def run(model, kv, ctx, tokens, parent):
+def run(model, kv, ctx, tokens, parent, outs=None):
     """One tree through both verify entry points on the same cache: first
     oos_tree_verify (the call the benchmark times), then
     oos_tree_verify_debug (the same step plus final hidden rows and per-node
     argmax / top-1 / top-2).  The two must agree bit for bit on the accept
     outputs and on the tree K/V they write; the debug call's intermediates
     are returned for the comparison with the CPU checker, and the plain call's
-    accept outputs feed the compaction check."""
+    accept outputs feed the compaction check.  `outs`, when given, is a pair of
+    output buffer sets (plain, debug) reused from call to call."""
     tok = torch.as_tensor(np.asarray(tokens, np.int32), device="cuda")
     par = torch.as_tensor(np.asarray(parent, np.int32), device="cuda")
     T = len(tokens)
-    plain = B.tree_verify(model, kv, ctx, tok, par, debug=False)
+    plain = B.tree_verify(model, kv, ctx, tok, par, outs=outs[0] if outs else None, debug=False)
     torch.cuda.synchronize()
     plain_status = B.oos_last_status(model)
     plain_k = [_bits(kv.k[l][ctx:ctx + T]).clone() for l in range(len(kv.k))]
     plain_v = [_bits(kv.v[l][ctx:ctx + T]).clone() for l in range(len(kv.v))]
-    outs = B.tree_verify(model, kv, ctx, tok, par, debug=True)
+    outs = B.tree_verify(model, kv, ctx, tok, par, outs=outs[1] if outs else None, debug=True)
     torch.cuda.synchronize()
     status = B.oos_last_status(model)
     assert status == plain_status, (status, plain_status)

@@ -158,6 +158,44 @@ def test_graph_replay_matches_direct_launch(tiny_models):
         assert a["accepted_nodes"] == x["accepted_nodes"] and a["bonus"] == x["bonus"]
 
 
+
+@pytest.mark.parametrize("name,overrides", [("tiny", None), ("mini-bf16", None),
+                                            ("mini-bf16", dict(cache_dtype="f16"))])
+def test_graph_reused_across_committed_lengths(name, overrides):
+    """oos_tree_verify keeps its captured graph when only the committed length
+    changes (the new length goes to the tree-prep node alone) and captures
+    again when the length changes the attention's split count.  Every call,
+    with the same output buffers, equals a direct launch bit for bit and the
+    checker at its own length."""
+    case = build_case(name, 0, cfg_overrides=overrides)
+    graph_model, w = gpu_model(case)
+    direct = B.OosModel(case.cfg, w, use_graph=False)
+    T = len(case.tokens)
+    kv_g = gpu_cache(case, case.ctx_len + T)
+    kv_d = gpu_cache(case, case.ctx_len + T)
+    snap = [t.clone() for t in kv_g.k], [t.clone() for t in kv_g.v]
+    outs_g = (B.VerifyOutputs(T), B.VerifyOutputs(T, case.cfg.hidden))
+    outs_d = (B.VerifyOutputs(T), B.VerifyOutputs(T, case.cfg.hidden))
+    c = case.ctx_len
+    gated = 0
+    for ctx in (c, c - 37, c - 1, 5, c - 100, c):
+        for kv in (kv_g, kv_d):   # every call starts from the committed cache
+            for l in range(case.cfg.n_layers):
+                kv.k[l].copy_(snap[0][l])
+                kv.v[l].copy_(snap[1][l])
+        g = run(graph_model, kv_g, ctx, case.tokens, case.parent, outs=outs_g)
+        d = run(direct, kv_d, ctx, case.tokens, case.parent, outs=outs_d)
+        assert np.array_equal(g["final_hidden"], d["final_hidden"]), ctx
+        assert np.array_equal(g["argmax"], d["argmax"]) and np.array_equal(g["top1"], d["top1"]), ctx
+        assert g["accepted_nodes"] == d["accepted_nodes"] and g["bonus"] == d["bonus"], ctx
+        for l in range(case.cfg.n_layers):
+            assert np.array_equal(g["tree_k"][l], d["tree_k"][l]) and np.array_equal(g["tree_v"][l], d["tree_v"][l])
+        r = oracle.verify_tree(case.view, [k[:ctx] for k in case.cache_k64], [v[:ctx] for v in case.cache_v64], ctx,
+                               case.tokens, case.parent)
+        gated += check_case(case, g, r)
+    assert gated >= 3
+
+
 # ------------------------------------------------------------------ accept walk and compaction alone
 
 def test_accept_walk_hand_fixtures_and_random():
