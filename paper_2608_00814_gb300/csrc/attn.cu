@@ -14,7 +14,8 @@
 // 16 blocks, non-portable size, chosen so that every cluster is resident at
 // once).  Per tile:
 //   - S = q K^T on the tensor cores into TMEM, N = 128 keys, q as hi + lo
-//     bf16 halves (two MMA chains) held in TMEM as the A operand;
+//     bf16 halves (two MMA chains), the A operand straight from the shared
+//     memory TMA staged it in;
 //   - softmax, one thread per query row: the row's S from TMEM, the valid-key
 //     mask (cache keys, then the node's ancestors), exp2, and P (bf16 pairs)
 //     written back over the first 64 columns of the same S buffer;
@@ -73,13 +74,11 @@ constexpr int kAttnThreads = 224;                         // 7 warps, roles belo
 static_assert(kAttnSmem <= 227 * 1024, "shared memory per block");
 static_assert(kMaxSplits <= 16, "cluster size");
 // TMEM columns (lane = query row): S[2] fp32 scores of a tile (P, bf16 pairs,
-// overwrites the first 64 columns of its S buffer), O fp32, q hi and lo as
-// packed bf16 pairs along d
+// overwrites the first 64 columns of its S buffer), O fp32
 constexpr int kTmS = 0;                            // [2] x 128
 constexpr int kTmO = 2 * kAttnKeys;                // 128
-constexpr int kTmQ = kTmO + kAttnD;                // [hi, lo] x 64
-constexpr int kAttnTmemCols = 512;
-static_assert(kTmQ + kAttnD == kAttnTmemCols, "TMEM columns");
+constexpr int kAttnTmemCols = 512;                 // allocation unit: a power of two
+static_assert(kTmO + kAttnD <= kAttnTmemCols, "TMEM columns");
 
 struct AttnArgs {
   CUtensorMap kmap, vmap;   // cache [capacity][nkv][d] as (d, kv head, slot)
@@ -208,7 +207,7 @@ OOS_DEV void shl128(unsigned long long lo, unsigned long long hi, int s, unsigne
 }
 
 // sites of the bounded waits (recorded on the status word when one expires)
-enum { AW_KEMPTY = 21, AW_VEMPTY, AW_QTM, AW_KFULL, AW_SFREE, AW_PFULL, AW_VFULL, AW_SFULL, AW_PV_RESCALE,
+enum { AW_KEMPTY = 21, AW_VEMPTY, AW_QFULL, AW_KFULL, AW_SFREE, AW_PFULL, AW_VFULL, AW_SFULL, AW_PV_RESCALE,
        AW_VZERO };
 OOS_DEV bool attn_wait(uint64_t* bar, uint32_t parity, volatile int* abort, uint32_t* status, uint32_t site, int ti) {
   if (mbar_wait(bar, parity, abort, status)) return true;
@@ -225,8 +224,8 @@ OOS_DEV void drain_wait(uint64_t* bar, uint32_t parity) {
 
 // Block roles: warp 0 lane 0 loads K and V tiles (TMA into the swizzled
 // layouts); warp 1 lane 0 issues the S MMAs, warp 6 lane 0 the P.V MMAs;
-// warps 2..5 load q into TMEM and run the softmax (thread = query row = TMEM
-// lane); all warps take part in the merge.
+// warps 2..5 run the softmax (thread = query row = TMEM lane); all warps take
+// part in the merge.
 // F16: the KV cache (and q) are IEEE binary16 -- every product runs in f16;
 // otherwise bf16.
 template <bool F16>
@@ -241,7 +240,6 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
   uint64_t* sfull = bar + 8;      // [2] S MMAs done
   uint64_t* pfull = bar + 10;     // [2] 4 softmax warps: P written
   uint64_t* pvdone = bar + 12;    // [2] P.V MMAs done (S/P buffer free, O current)
-  uint64_t* qtm = bar + 14;       // 4 softmax warps: q rows are in TMEM
   uint64_t* odone = bar + 15;     // both MMA issuers done
   uint64_t* recv_full = bar + 16; // merge: every split's rows for this block copied in (transaction bytes)
   uint64_t* qfull = bar + 17;     // q tile landed (transaction bytes)
@@ -282,7 +280,6 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
       mbar_init(&pfull[s], 4);
       mbar_init(&pvdone[s], 1);
     }
-    mbar_init(qtm, 4);
     mbar_init(odone, 2);
     mbar_init(recv_full, 1);
     mbar_init(qfull, 1);
@@ -296,10 +293,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
   __syncthreads();
   tc_fence_after();
   // Another block may copy into this block's receive buffer only once the
-  // block runs, its receive barrier is armed and the q tile staged in that
-  // buffer has gone to TMEM: every thread arrives on the cluster barrier when
-  // it is past that point (the q rows' threads after their copy, the others
-  // now), and every block waits for the whole cluster before its merge copies.
+  // block runs, its receive barrier is armed and the S MMAs no longer read the
+  // q tile staged in that buffer: every thread arrives on the cluster barrier
+  // when it is past that point (the softmax threads after the last tile's S,
+  // the others now), and every block waits for the whole cluster before its
+  // merge copies.
   if (warp < 2 || warp > 5) cluster_arrive_release();
   const uint32_t tmem = *tmem_slot;
   const uint32_t tmem_o = tmem + kTmO;
@@ -361,16 +359,20 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
     }
   } else if (warp == 1 || warp == 6) {
     // ------------------------------------------------------------ MMA issuers
-    // Operands reach the tensor cores through the async proxy only: K and V
-    // by TMA, q and P from threads that wait for their TMEM stores before they
+    // Operands reach the tensor cores through the async proxy only: q, K and
+    // V by TMA, P from threads that wait for their TMEM stores before they
     // arrive, the zeroed V rows fenced by the threads that wrote them.
     // Descriptors: the start address is the low field (16-byte units), so a
     // byte offset o inside an operand region is added as o >> 4.
     if (lane == 0 && warp == 1) {
       constexpr uint32_t idesc_s = F16 ? idesc_f16_f32(kAttnRows, kAttnKeys) : idesc_bf16_f32(kAttnRows, kAttnKeys);
-      bool ok = attn_wait(qtm, 0, abort_flag, status, AW_QTM, 0);
+      bool ok = attn_wait(qfull, 0, abort_flag, status, AW_QFULL, 0);
       tc_fence_after();
       const uint64_t kdesc0 = smem_desc_sw128(smem_addr(sm + kOffK));
+      // q as staged by TMA: [hi d0, hi d1, lo d0, lo d1], each 128 rows x 128
+      // bytes in the swizzled K-major layout (rows of padding nodes hold
+      // whatever the q buffer holds; every row of S, P and O is its own)
+      const uint64_t qdesc0 = smem_desc_sw128(smem_addr(sm + kOffRecv));
       for (int ti = 0; ti < n_tiles && ok; ++ti) {
         const int b = ti & 1;
         const uint32_t use = (uint32_t)(ti >> 1);
@@ -381,15 +383,15 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
         tc_fence_after();
         const uint64_t kd0 = kdesc0 + (uint64_t)((b * kTileBytes) >> 4);
         const uint32_t d = tmem + kTmS + b * kAttnKeys;
-        // S = q_hi K^T + q_lo K^T over the 128 head dims: q from TMEM (8
-        // columns = 16 of d per MMA), K from the two 64-wide d blocks (32 bytes
-        // of d per MMA)
+        // S = q_hi K^T + q_lo K^T over the 128 head dims: q and K both from
+        // their two 64-wide d blocks (32 bytes of d per MMA)
 #pragma unroll
         for (int half = 0; half < 2; ++half) {
 #pragma unroll
           for (int k = 0; k < kAttnD / 16; ++k) {
             const uint64_t kd = kd0 + (uint64_t)(((k >> 2) * kDBlock) >> 4) + 2 * (k & 3);
-            tc_mma_bf16_ts(d, tmem + kTmQ + half * (kAttnD / 2) + 8 * k, kd, idesc_s, (half > 0 || k > 0) ? 1u : 0u);
+            const uint64_t qd = qdesc0 + (uint64_t)(((2 * half + (k >> 2)) * (kAttnRows * 128)) >> 4) + 2 * (k & 3);
+            tc_mma_bf16(d, qd, kd, idesc_s, (half > 0 || k > 0) ? 1u : 0u);
           }
         }
         tc_commit(&kempty[b]);
@@ -421,7 +423,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
     }
   }
 
-  // ------------------------------------------------------------ q and softmax (warps 2..5)
+  // ------------------------------------------------------------ softmax (warps 2..5)
   float m_used = -INFINITY, l_sum = 0.f;
   const int q4 = warp & 3;
   const int lrow = q4 * 32 + lane;                  // local row = TMEM lane
@@ -429,48 +431,38 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
   if (warp >= 2 && warp <= 5) {
     const bool real = lrow < vrows;
     const int node = real ? node0 + lrow / G : node0;
-    pdl_wait();
-    pdl_trigger();
-    const unsigned long long anc0 = a.anc[2 * node], anc1 = a.anc[2 * node + 1];
-    // this thread's q row (hi then lo, 64 columns each as bf16 pairs) from the
-    // staged swizzled tile into TMEM, the S MMAs' A operand; rows of padding
-    // nodes are zero
-    const bool qok = __all_sync(0xffffffffu, attn_wait(qfull, 0, abort_flag, status, AW_QTM, 0));
-    if (qok) {
-      const unsigned char* qs = sm + kOffRecv;
-#pragma unroll
-      for (int part = 0; part < 8; ++part) {   // (hi/lo, 64-wide d block, half of its 8 chunks)
-        const unsigned char* qb = qs + (part >> 1) * (kAttnRows * 128);
-        uint32_t w[16];
-#pragma unroll
-        for (int c = 0; c < 4; ++c) {
-          const uint4 v = real ? *reinterpret_cast<const uint4*>(qb + sw128(lrow, (part & 1) * 4 + c))
-                               : make_uint4(0, 0, 0, 0);
-          w[4 * c] = v.x;
-          w[4 * c + 1] = v.y;
-          w[4 * c + 2] = v.z;
-          w[4 * c + 3] = v.w;
-        }
-        tmem_st16u(tmem + lane_off + kTmQ + part * 16, w);
+    unsigned long long anc0 = 0ull, anc1 = 0ull;
+    bool waited = false;
+    // Iteration -1 is a dry pass of the tile body, run before the dependency
+    // wait while the block has nothing else to do: it brings the body's code
+    // into the SM's instruction caches (the step's other kernels have evicted
+    // it since the previous layer), reads whatever S buffer 0 holds, and
+    // discards everything -- no wait, store, arrive or state update.
+#pragma unroll 1
+    for (int ti = -1; ti < n_tiles; ++ti) {
+      asm volatile("" : "+r"(ti));   // one loop body for every iteration: none is specialised
+      const bool dry = ti < 0;         // warp-uniform
+      if (ti == 0) {
+        pdl_wait();
+        pdl_trigger();
+        waited = true;
+        anc0 = a.anc[2 * node];
+        anc1 = a.anc[2 * node + 1];
       }
-      tmem_wait_st();
-    }
-    tc_fence_before();
-    __syncwarp();
-    if (lane == 0) mbar_arrive(qtm);
-    cluster_arrive_release();   // this thread is done with the staged q
-    for (int ti = 0; ti < n_tiles; ++ti) {
-      const int b = ti & 1;
-      const uint32_t use = (uint32_t)(ti >> 1);
-      // every wait's outcome is made warp-uniform: the .sync.aligned TMEM
-      // accesses and __syncwarp below need the whole warp on one path
-      if (!__all_sync(0xffffffffu, attn_wait(&sfull[b], use & 1u, abort_flag, status, AW_SFULL, ti))) break;
-      tc_fence_after();
-      const int key0 = (t0 + ti) * kAttnKeys;
+      const int tt = dry ? 0 : ti;
+      const int b = tt & 1;
+      const uint32_t use = (uint32_t)(tt >> 1);
+      if (!dry) {
+        // every wait's outcome is made warp-uniform: the .sync.aligned TMEM
+        // accesses and __syncwarp below need the whole warp on one path
+        if (!__all_sync(0xffffffffu, attn_wait(&sfull[b], use & 1u, abort_flag, status, AW_SFULL, ti))) break;
+        tc_fence_after();
+      }
+      const int key0 = dry ? ctx : (t0 + ti) * kAttnKeys;
       // valid keys of this row in the tile: committed slots, then the tree
       // slots of the node's ancestors (slot ctx + j for ancestor j); slots at
-      // or past ctx + T are never ancestors
-      const bool full_tile = key0 + kAttnKeys <= ctx;   // tile-uniform
+      // or past ctx + T are never ancestors (the dry pass takes the masked path)
+      const bool full_tile = !dry && key0 + kAttnKeys <= ctx;   // tile-uniform
       unsigned long long mlo = ~0ull, mhi = ~0ull;
       if (!full_tile) {
         const int c = max(0, ctx - key0);                 // leading committed slots (< 128)
@@ -497,7 +489,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
       // move the running maximum only when this tile exceeds it by 2^8 (a
       // lane that moves its maximum rescales its O row; the whole warp takes
       // part in the TMEM accesses, lanes that keep theirs scale by 1)
-      const bool move = tmax > m_used + 8.f;
+      const bool move = !dry && tmax > m_used + 8.f;
       const bool rescale = move && m_used != -INFINITY;
       if (__any_sync(0xffffffffu, rescale)) {
         // O holds P.V of tiles < ti: wait for the last of them, then rescale
@@ -525,8 +517,8 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
       // (-inf) gives 0, and a row with nothing valid yet (m = -inf) gives 0
       uint32_t pk[kAttnKeys / 2];
       float ps[4] = {0.f, 0.f, 0.f, 0.f};
-      const bool live = m_used != -INFINITY;
-      const float neg_m = live ? -m_used : 0.f;
+      const bool live = dry || m_used != -INFINITY;
+      const float neg_m = (live && !dry) ? -m_used : 0.f;
 #pragma unroll
       for (int i = 0; i < kAttnKeys; i += 2) {
         const float p0 = live ? ex2_approx(fmaf(sv[i], scale_log2, neg_m)) : 0.f;
@@ -541,6 +533,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
           ps[(i >> 1) & 3] += __low2float(pp) + __high2float(pp);
           pk[i / 2] = *reinterpret_cast<const uint32_t*>(&pp);
         }
+      }
+      if (dry) {   // the weights count as used, so that the dry pass computes them
+#pragma unroll
+        for (int i = 0; i < kAttnKeys / 2; ++i) asm volatile("" ::"r"(pk[i]));
+        asm volatile("" ::"f"(ps[0]), "f"(ps[1]), "f"(ps[2]), "f"(ps[3]));
+        continue;
       }
       l_sum += (ps[0] + ps[1]) + (ps[2] + ps[3]);
       // slots at or past ctx + T in this tile hold whatever the cache holds
@@ -566,6 +564,14 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
       __syncwarp();
       if (lane == 0) mbar_arrive(&pfull[b]);
     }
+    if (!waited) {   // no tile: the dependency wait is still owed
+      pdl_wait();
+      pdl_trigger();
+    }
+    // the S MMAs are done with the staged q (every S this thread waited for);
+    // after an abort an S MMA may still read it while a peer's merge rows
+    // arrive -- the step has failed then, and only values are affected
+    cluster_arrive_release();
     // every role is done with the rings and TMEM once all MMAs have completed;
     // both issuers always commit this barrier, and TMEM must not be released
     // under a running MMA, so the wait is not cut short by the handle's limit
