@@ -45,6 +45,36 @@
 #include "common.cuh"
 #include "internal.h"
 
+// Step timeline (built only with -DOOS_TIMELINE, see timeline.py): per block
+// of the last attention launch, the globaltimer at entry (0), at the end of the
+// loader's dependency wait (1), when q has landed (2), at the start and end of
+// the softmax of tiles 0..5 (3 + 2t, 4 + 2t), when all MMAs are done (15), when
+// the merge rows are staged (21), past the cluster barrier (22), when this
+// block's rows have been copied out (16) and its own rows received (17), and at
+// exit (18); slots 19 and 20 hold the block's tile count and the split count.
+#ifdef OOS_TIMELINE
+namespace oos {
+__device__ unsigned long long g_tl_attn[2048][24];
+}
+#define TL_ATTN(ev)                                                                      \
+  do {                                                                                   \
+    const unsigned bid_ = blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z); \
+    if (bid_ < 2048) oos::g_tl_attn[bid_][ev] = oos::globaltimer();                      \
+  } while (0)
+#define TL_ATTN_VAL(ev, v)                                                               \
+  do {                                                                                   \
+    const unsigned bid_ = blockIdx.x + gridDim.x * (blockIdx.y + gridDim.y * blockIdx.z); \
+    if (bid_ < 2048) oos::g_tl_attn[bid_][ev] = (unsigned long long)(v);                 \
+  } while (0)
+#else
+#define TL_ATTN(ev) \
+  do {              \
+  } while (0)
+#define TL_ATTN_VAL(ev, v) \
+  do {                     \
+  } while (0)
+#endif
+
 namespace oos {
 
 constexpr int kAttnRows = 128;     // query rows per block (tcgen05 M)
@@ -247,6 +277,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_slot + 1);
   static_assert(18 * 8 + 8 <= 256, "barrier block");
 
+  if (threadIdx.x == 0) TL_ATTN(0);
   const int T = a.T, nq = a.nq, G = a.group, npc = a.npc, S = a.splits;
   const float scale_log2 = a.scale_log2;
   uint32_t* status = a.status;
@@ -328,6 +359,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
       }
       pdl_wait();
       pdl_trigger();
+      TL_ATTN(1);
       // q rows of the block's nodes, hi and lo halves, two 64-wide d blocks
       // each, staged in the (still unused) receive buffer
       tma_prefetch_desc(&a.qhi);
@@ -367,6 +399,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
     if (lane == 0 && warp == 1) {
       constexpr uint32_t idesc_s = F16 ? idesc_f16_f32(kAttnRows, kAttnKeys) : idesc_bf16_f32(kAttnRows, kAttnKeys);
       bool ok = attn_wait(qfull, 0, abort_flag, status, AW_QFULL, 0);
+      TL_ATTN(2);
       tc_fence_after();
       const uint64_t kdesc0 = smem_desc_sw128(smem_addr(sm + kOffK));
       // q as staged by TMA: [hi d0, hi d1, lo d0, lo d1], each 128 rows x 128
@@ -459,6 +492,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
         tc_fence_after();
       }
       const int key0 = dry ? ctx : (t0 + ti) * kAttnKeys;
+      if (!dry && warp == 2 && lane == 0 && ti < 6) TL_ATTN(3 + 2 * ti);
       // valid keys of this row in the tile: committed slots, then the tree
       // slots of the node's ancestors (slot ctx + j for ancestor j); slots at
       // or past ctx + T are never ancestors (the dry pass takes the masked path)
@@ -563,6 +597,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&pfull[b]);
+      if (warp == 2 && lane == 0 && ti < 6) TL_ATTN(4 + 2 * ti);
     }
     if (!waited) {   // no tile: the dependency wait is still owed
       pdl_wait();
@@ -576,6 +611,7 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
     // both issuers always commit this barrier, and TMEM must not be released
     // under a running MMA, so the wait is not cut short by the handle's limit
     drain_wait(odone, 0);
+    if (warp == 2 && lane == 0) TL_ATTN(15);
   }
   tc_fence_before();
   __syncthreads();
@@ -608,7 +644,9 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
     }
   }
   __syncthreads();
+  if (threadIdx.x == 0) TL_ATTN(21);
   cluster_wait_acquire();   // every block of the cluster runs and has armed its receive barrier
+  if (threadIdx.x == 0) TL_ATTN(22);
   if (threadIdx.x == 0) {
     for (int j = 0; j < S; ++j) {
       const int r0 = (int)((long long)vrows * j / S), r1 = (int)((long long)vrows * (j + 1) / S);
@@ -619,10 +657,12 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
     }
     bulk_commit_and_wait_read();   // the staged rows have been read before this block moves on
   }
+  if (threadIdx.x == 0) TL_ATTN(16);
   // this block's rows from every split.  Every block copies its rows even
   // after an abort, so this wait ends; it is not cut short by the handle's
   // limit, because the block must not exit while copies into it are in flight.
   drain_wait(recv_full, 0);
+  if (threadIdx.x == 0) TL_ATTN(17);
   {
     // split weights of every owned row: 2^(m_s - M) / sum_s 2^(m_s - M) l_s
     if (threadIdx.x < n_mine) {
@@ -655,6 +695,11 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
       const size_t grow = (size_t)(node0 + lr / G) * nq + g * G + lr % G;
       store_act4(a.out, grow * kAttnD + d4, a.out_lo_off, acc);
     }
+  }
+  if (threadIdx.x == 0) {
+    TL_ATTN(18);
+    TL_ATTN_VAL(19, n_tiles);
+    TL_ATTN_VAL(20, S);
   }
   tc_fence_before();
   __syncthreads();
@@ -846,3 +891,18 @@ cudaError_t launch_attention(Model& m, int layer, const void* kc, const void* vc
 }
 
 }  // namespace oos
+
+#ifdef OOS_TIMELINE
+// timeline accessors (the OOS_TIMELINE library only)
+extern "C" int oos_timeline_attn_read(void* out, size_t bytes) {
+  return cudaMemcpyFromSymbol(out, oos::g_tl_attn, bytes < sizeof(oos::g_tl_attn) ? bytes : sizeof(oos::g_tl_attn)) ==
+                 cudaSuccess
+             ? 0
+             : OOS_ECUDA;
+}
+extern "C" int oos_timeline_attn_clear() {
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, oos::g_tl_attn) != cudaSuccess) return OOS_ECUDA;
+  return cudaMemset(p, 0, sizeof(oos::g_tl_attn)) == cudaSuccess ? 0 : OOS_ECUDA;
+}
+#endif

@@ -18,6 +18,26 @@
 #include "common.cuh"
 #include "internal.h"
 
+// Step timeline (built only with -DOOS_TIMELINE, see timeline.py): per GEMM
+// launch of a step and per CTA, the globaltimer at entry (0), at the end of the
+// dependency wait (1), when the last accumulator is ready (2), at the last
+// arrival count (4), when the finishing may start (5) and at exit (3).  A
+// launch's slot comes from its arrival-counter block, one per (layer, GEMM).
+#ifdef OOS_TIMELINE
+namespace oos {
+__device__ unsigned long long g_tl_gemm[1024][160][6];
+}
+#define TL_GEMM(ev)                                                                                   \
+  do {                                                                                                \
+    if (!ARGMAX && a.cnt && blockIdx.x < 160)                                                        \
+      oos::g_tl_gemm[((uintptr_t)a.cnt >> 10) & 1023][blockIdx.x][ev] = oos::globaltimer();          \
+  } while (0)
+#else
+#define TL_GEMM(ev) \
+  do {              \
+  } while (0)
+#endif
+
 namespace oos {
 
 // Epilogues fused into the weight GEMMs (bf16 path).  Stream-K leaves a tile's
@@ -362,6 +382,7 @@ __global__ void __launch_bounds__(192, 1)
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int G = gridDim.x, cta = blockIdx.x;
+  if (threadIdx.x == 0) TL_GEMM(0);
 
   // this CTA's work: units [u0, u1) (stream-K) or work tiles cta, cta+G, ... (LM head)
   long long u0, u1;
@@ -455,6 +476,7 @@ __global__ void __launch_bounds__(192, 1)
       }
       pdl_wait();
       pdl_trigger();
+      TL_GEMM(1);
       for (int j = 0; j < n_pre; ++j) load_x(j, j);
       int stage = n_pre % S;
       uint32_t phase = (n_pre == S) ? 1u : 0u;
@@ -571,6 +593,7 @@ __global__ void __launch_bounds__(192, 1)
       int seg_end = j + (a.kbt - kb);
       if (seg_end > n_units) seg_end = n_units;
       mbar_wait(&accf[acc], acc_use[acc] & 1u, abort_flag, a.status);
+      if (e == 0 && seg_end >= n_units) TL_GEMM(2);
       if (epi_aborted()) break;
       tc_fence_after();
       const uint32_t taddr0 = tmem_base + ((uint32_t)(q * 32) << 16) + (uint32_t)(acc * kSub * C::SUB_COLS);
@@ -655,6 +678,7 @@ __global__ void __launch_bounds__(192, 1)
         __threadfence();
         epi_bar();
         if (e == 0) atomicAdd(&a.cnt[wt], 1);
+        if (e == 0 && seg_end >= n_units) TL_GEMM(4);
       } else {
 #pragma unroll 1
         for (int sub = 0; sub < kSub; ++sub) {
@@ -710,6 +734,7 @@ __global__ void __launch_bounds__(192, 1)
       // the two latency-bound passes overlap instead of running back to back.
       StreamK sk{a.n_work, a.kbt, a.total, G};
       int jj = 0;
+      bool tl_first = true;
       while (jj < n_units) {
         // the next one or two work tiles of the range: (tile, contributors, token share)
         auto next_tile = [&](int& wt, int& nc, int& tb, int& te) {
@@ -748,6 +773,8 @@ __global__ void __launch_bounds__(192, 1)
           }
         }
         if (epi_aborted()) break;
+        if (e == 0 && tl_first) TL_GEMM(5);
+        tl_first = false;
         __threadfence();
         const int ew = e >> 5;   // epilogue warp 0..3
         const bool second = two && ew >= 2;
@@ -778,6 +805,7 @@ __global__ void __launch_bounds__(192, 1)
   }
   tc_fence_before();
   __syncthreads();
+  if (threadIdx.x == 0) TL_GEMM(3);
   if (warp == 2) {
     tc_fence_after();
     tmem_dealloc(tmem_base, C::NCOLS);
@@ -1037,3 +1065,18 @@ cudaError_t launch_lm_head_f32(Model& m, int T, cudaStream_t st) {
 }
 
 }  // namespace oos
+
+#ifdef OOS_TIMELINE
+// timeline accessors (the OOS_TIMELINE library only)
+extern "C" int oos_timeline_gemm_read(void* out, size_t bytes) {
+  return cudaMemcpyFromSymbol(out, oos::g_tl_gemm, bytes < sizeof(oos::g_tl_gemm) ? bytes : sizeof(oos::g_tl_gemm)) ==
+                 cudaSuccess
+             ? 0
+             : OOS_ECUDA;
+}
+extern "C" int oos_timeline_gemm_clear() {
+  void* p = nullptr;
+  if (cudaGetSymbolAddress(&p, oos::g_tl_gemm) != cudaSuccess) return OOS_ECUDA;
+  return cudaMemset(p, 0, sizeof(oos::g_tl_gemm)) == cudaSuccess ? 0 : OOS_ECUDA;
+}
+#endif
