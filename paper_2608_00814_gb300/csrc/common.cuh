@@ -209,7 +209,6 @@ OOS_DEV void tma_load_2d(void* smem_dst, const void* tmap, uint64_t* bar, int x,
       : "memory");
 }
 
-// L2 prefetch of one 2-D box (no shared-memory destination, no completion)
 // 3-D / 4-D tile loads (coordinates innermost first; x * 2 bytes a multiple of 16)
 OOS_DEV void tma_load_3d(void* smem_dst, const void* tmap, uint64_t* bar, int x, int y, int z, uint64_t policy) {
   asm volatile(
