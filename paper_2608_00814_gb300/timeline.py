@@ -21,7 +21,6 @@ workload's tree comes from bench.py).
 import argparse
 import ctypes
 import dataclasses
-import os
 import sys
 
 import numpy as np
