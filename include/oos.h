@@ -92,7 +92,11 @@ typedef struct {
     float rms_eps;
     float rope_theta;      /* RoPE base; pair (m, m + d/2) turns by pos * theta^(-2m/d) */
     int32_t max_T;         /* largest tree this handle verifies, 1..128 */
-    int32_t use_graph;     /* nonzero: replay a captured CUDA graph when the call's shape repeats */
+    int32_t use_graph;     /* nonzero: oos_tree_verify replays one captured CUDA graph while the
+                              cache buffers, T, the I/O pointers and the attention's key-split
+                              count repeat; a new committed length updates only the graph's
+                              tree-preparation node (the other kernels read it from the
+                              workspace); anything else is captured again */
     /* Rotary frequency rescaling of Llama-3.1 targets (the paper's Llama-3.1-8B),
      * as published with that model.  With factor F > 1, low-frequency factor lo,
      * high-frequency factor hi (hi > lo > 0) and original context L > 0, the
