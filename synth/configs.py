@@ -11,6 +11,7 @@ in the main comparison table): one greedy path of `plant` draft nodes is
 planted under the root, the remaining nodes are random draft tokens.
 """
 
+import dataclasses
 from dataclasses import dataclass, field, asdict
 
 
@@ -140,9 +141,15 @@ MINI_BF16 = ModelConfig("mini-bf16", n_layers=2, hidden=256, n_q_heads=4, n_kv_h
                         rope_theta=1e6, dtype="bf16", qk_norm=True, qkv_bias=False, tied=False,
                         init_std=0.08)
 
+# The same decoder with the FP16 KV cache (binary16 K/V, bf16 weights): the
+# cache backend the paper runs Qwen2.5 and Llama with.
+MINI_F16 = dataclasses.replace(MINI_BF16, name="mini-f16", cache_dtype="f16")
+
 TEST_WORKLOADS = {
     "mini-bf16": Workload(MINI_BF16, ctx_len=200, T=16, plant=3,
                           tree=dict(kind="uniform", max_depth=6), prefill=True),
+    "mini-f16": Workload(MINI_F16, ctx_len=200, T=16, plant=3,
+                         tree=dict(kind="uniform", max_depth=6), prefill=True),
 }
 
 MODELS = {w.model.name: w.model for w in list(WORKLOADS.values()) + list(TEST_WORKLOADS.values())}

@@ -305,13 +305,22 @@ def _gated_roots_sweep(name, base, model, min_gated):
             assert g["accepted_len"] >= len(case.planted_path)
         gated += ok
         n += 1
-    print("%s: %d of %d bf16 cases gated (accept outputs compared exactly)" % (name, gated, n))
+    print("%s: %d of %d cases gated (accept outputs compared exactly)" % (name, gated, n))
     assert gated >= min_gated, "%s: only %d of %d cases passed the margin gate" % (name, gated, n)
 
 
 def test_mini_bf16_gated_roots(mini_models):
     base, model = _mini(mini_models, 0)
     _gated_roots_sweep("mini-bf16", base, model, 20)
+
+
+def test_mini_f16_cache_gated_roots():
+    """The FP16 KV cache (binary16 K/V under bf16 weights): 24 trees around
+    well-separated greedy paths of the FP16-cache model, every node against
+    the full oracle step."""
+    base = build_case("mini-f16", 0)
+    model, _ = gpu_model(base)
+    _gated_roots_sweep("mini-f16", base, model, 20)
 
 
 def test_bf16_qwen3_06b_gated_roots():
@@ -500,6 +509,7 @@ def test_bf16_qwen25_32b_sampled():
     ("tiny", 128, 129),        # after a cached prefix; one full chain and a one-token chain
     ("mini-bf16", 200, 290),   # bf16 tensor-core path
     ("mini-bf16", 0, 1),       # one-token prompt
+    ("mini-f16", 200, 150),    # FP16 KV cache
 ])
 def test_prefill_matches_causal_decoding(tiny_models, mini_models, name, ctx, n):
     """oos_prefill == causal decoding of the prompt after ctx cached positions:
@@ -507,6 +517,8 @@ def test_prefill_matches_causal_decoding(tiny_models, mini_models, name, ctx, n)
     its margin clears the gate)."""
     if name == "tiny":
         case, model = _tiny(tiny_models, 4, ctx_len=ctx)
+    elif name == "mini-f16":
+        case, model = _mini(mini_models, 4, ctx_len=ctx, cfg_overrides=dict(cache_dtype="f16"))
     else:
         case, model = _mini(mini_models, 4, ctx_len=ctx)
     cfg = case.cfg
