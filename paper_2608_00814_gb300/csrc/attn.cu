@@ -665,31 +665,51 @@ __global__ void __launch_bounds__(kAttnThreads, 1) k_attn_tc(const __grid_consta
   if (threadIdx.x == 0) TL_ATTN(17);
   {
     // split weights of every owned row: 2^(m_s - M) / sum_s 2^(m_s - M) l_s
+    // (every split's value of a row is loaded before any is used: the loops
+    // run over the largest split count, guarded, so they unroll)
     if (threadIdx.x < n_mine) {
       const int i = threadIdx.x;
+      float ms[kMaxSplits], ls[kMaxSplits];
       float M = -INFINITY;
-      for (int s2 = 0; s2 < S; ++s2) M = fmaxf(M, recv[(size_t)(s2 * n_max + i) * kMergeLd + kAttnD]);
-      float den = 0.f;
-      for (int s2 = 0; s2 < S; ++s2) {
-        const float* ml = recv + (size_t)(s2 * n_max + i) * kMergeLd + kAttnD;
-        const float w = ml[0] == -INFINITY ? 0.f : exp2f(ml[0] - M);
-        wgt[i * kMaxSplits + s2] = w;
-        den += w * ml[1];
+#pragma unroll
+      for (int s2 = 0; s2 < kMaxSplits; ++s2) {
+        if (s2 < S) {
+          const float2 ml = *reinterpret_cast<const float2*>(recv + (size_t)(s2 * n_max + i) * kMergeLd + kAttnD);
+          ms[s2] = ml.x;
+          ls[s2] = ml.y;
+          M = fmaxf(M, ml.x);
+        }
+      }
+      float den = 0.f, w[kMaxSplits];
+#pragma unroll
+      for (int s2 = 0; s2 < kMaxSplits; ++s2) {
+        if (s2 < S) {
+          w[s2] = ms[s2] == -INFINITY ? 0.f : exp2f(ms[s2] - M);
+          den += w[s2] * ls[s2];
+        }
       }
       const float inv = den > 0.f ? 1.f / den : 0.f;
-      for (int s2 = 0; s2 < S; ++s2) wgt[i * kMaxSplits + s2] *= inv;
+#pragma unroll
+      for (int s2 = 0; s2 < kMaxSplits; ++s2)
+        if (s2 < S) wgt[i * kMaxSplits + s2] = w[s2] * inv;
     }
     __syncthreads();
     for (int idx = threadIdx.x; idx < n_mine * (kAttnD / 4); idx += blockDim.x) {
       const int i = idx / (kAttnD / 4), d4 = (idx % (kAttnD / 4)) * 4;
+      float4 v[kMaxSplits];
+#pragma unroll
+      for (int s2 = 0; s2 < kMaxSplits; ++s2)
+        if (s2 < S) v[s2] = *reinterpret_cast<const float4*>(recv + (size_t)(s2 * n_max + i) * kMergeLd + d4);
       float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int s2 = 0; s2 < S; ++s2) {
-        const float w = wgt[i * kMaxSplits + s2];
-        const float4 v = *reinterpret_cast<const float4*>(recv + (size_t)(s2 * n_max + i) * kMergeLd + d4);
-        acc.x += w * v.x;
-        acc.y += w * v.y;
-        acc.z += w * v.z;
-        acc.w += w * v.w;
+#pragma unroll
+      for (int s2 = 0; s2 < kMaxSplits; ++s2) {
+        if (s2 < S) {
+          const float ws = wgt[i * kMaxSplits + s2];
+          acc.x += ws * v[s2].x;
+          acc.y += ws * v[s2].y;
+          acc.z += ws * v[s2].z;
+          acc.w += ws * v[s2].w;
+        }
       }
       const int lr = lr0_mine + i;
       const size_t grow = (size_t)(node0 + lr / G) * nq + g * G + lr % G;
