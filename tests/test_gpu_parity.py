@@ -483,20 +483,9 @@ def test_llama31_8b_fp16_cache_sampled():
 
 def test_bf16_qwen3_32b_sampled():
     """Qwen3-32B shape of the paper's scaling study (64 layers, hidden 5120,
-    64/8 heads, q/k norm, SwiGLU 25600; about 63 GB of bf16 weights): a random
-    tree of 64 nodes, sampled nodes against the oracle (tensors at tolerance,
-    argmax and accept outputs where the margins gate)."""
-    case = build_case("qwen3-32b", 0, plant=0)
-    model, _ = gpu_model(case)
-    kv = gpu_cache(case, case.ctx_len + case.tokens.shape[0])
-    g = run(model, kv, case.ctx_len, case.tokens, case.parent)
-    T = len(case.tokens)
-    leaves = [i for i in range(T) if i not in set(case.parent[1:].tolist())]
-    rng = np.random.default_rng(3)
-    sample = list(rng.choice(leaves, size=3, replace=False))
-    r = _oracle(case, only=sample)
-    check_case(case, g, r, rows=r["nodes"])
-    check_compaction(model, kv, case.ctx_len, g)
+    64/8 heads, q/k norm, SwiGLU 25600; about 63 GB of bf16 weights): the
+    planted path and two leaves, with their ancestors, against the oracle."""
+    _sampled_check("qwen3-32b")
 
 
 def test_bf16_qwen25_32b_sampled():
