@@ -42,6 +42,8 @@ __global__ void __launch_bounds__(kHintThreads) k_hint_match(const int32_t* __re
                                                              uint8_t* __restrict__ mlen, uint8_t* __restrict__ cmax,
                                                              int* __restrict__ smax, int* __restrict__ best) {
   __shared__ int suf[kHintMaxN];
+  pdl_wait();   // the committed tokens and their count may come from the previous kernel
+  pdl_trigger();
   if (prefix_len_dev) prefix_len = *prefix_len_dev;
   const int nmax = prefix_len < kHintMaxN ? prefix_len : kHintMaxN;
   // suf[j] is the token j places before y's last token
@@ -182,6 +184,8 @@ __global__ void __launch_bounds__(kHintThreads) k_hint_pack(const int32_t* __res
   __shared__ int s_wcnt[kHintThreads / 32];
   __shared__ int s_n, s_nc, s_ns, s_done;
   const int warp = threadIdx.x >> 5, lane_id = threadIdx.x & 31;
+  pdl_wait();   // the match kernel's results
+  pdl_trigger();
   const int n = *best;
   if (prefix_len_dev) prefix_len = *prefix_len_dev;
   int T = 1, lanes = 0, hint_lanes = 0;       // warp 0's copies are the authoritative ones
@@ -269,10 +273,14 @@ __global__ void __launch_bounds__(kHintThreads) k_hint_pack(const int32_t* __res
 
 // workspace: [best | pad to 256][mlen: one byte per position, padded to 256]
 //            [cmax: one byte per chunk, padded to 256][smax: one int per span]
+// Workspace: the call's n (best) and the span maxima first, so that one
+// zeroing copy covers both; then one match byte per position and the chunk maxima.
+static size_t hint_head_bytes(size_t spans) { return (4 + spans * 4 + 255) / 256 * 256; }
+
 size_t hint_workspace_bytes(long long bank_len) {
   const size_t chunks = (size_t)((bank_len + kHintThreads - 1) / kHintThreads);
   const size_t spans = (chunks + kHintThreads - 1) / kHintThreads;
-  return 256 + chunks * kHintThreads + spans * kHintThreads + spans * 4;
+  return hint_head_bytes(spans) + chunks * kHintThreads + spans * kHintThreads;
 }
 
 cudaError_t launch_hint_tree(const int32_t* bank, int N, int eos, const int32_t* prefix, int prefix_len,
@@ -280,14 +288,13 @@ cudaError_t launch_hint_tree(const int32_t* bank, int N, int eos, const int32_t*
                              int n_native, int native_stride, int max_lanes, int depth, int max_nodes, int pad_to,
                              void* ws, int32_t* out_tok, int32_t* out_par, int32_t* out_T, int32_t* out_info,
                              cudaStream_t st) {
-  int* best = (int*)ws;
-  uint8_t* mlen = (uint8_t*)ws + 256;
   const long long n_chunks = ((long long)N + kHintThreads - 1) / kHintThreads;
   const long long n_spans = (n_chunks + kHintThreads - 1) / kHintThreads;
+  int* best = (int*)ws;
+  int* smax = best + 1;
+  uint8_t* mlen = (uint8_t*)ws + hint_head_bytes((size_t)n_spans);
   uint8_t* cmax = mlen + n_chunks * kHintThreads;
-  int* smax = (int*)(cmax + n_spans * kHintThreads);
-  cudaError_t e = cudaMemsetAsync(best, 0, sizeof(int), st);
-  if (e == cudaSuccess) e = cudaMemsetAsync(smax, 0, (size_t)n_spans * sizeof(int), st);
+  cudaError_t e = cudaMemsetAsync(best, 0, (size_t)(1 + n_spans) * sizeof(int), st);
   if (e != cudaSuccess) return e;
   int dev = 0, sms = 0;
   cudaGetDevice(&dev);
@@ -296,14 +303,15 @@ cudaError_t launch_hint_tree(const int32_t* bank, int N, int eos, const int32_t*
   const long long want = (n_chunks + kHintThreads / 32 - 1) / (kHintThreads / 32);
   const int grid = (int)(want < (long long)sms * 8 ? want : (long long)sms * 8);
   const int vec = ((uintptr_t)bank & 15) == 0 ? 1 : 0;
-  k_hint_match<<<grid, kHintThreads, 0, st>>>(bank, N, eos, prefix, prefix_len, prefix_len_dev, vec, mlen, cmax, smax,
-                                              best);
-  e = cudaGetLastError();
+  // the packing block launches while the match kernel runs (programmatic
+  // dependent launch) and waits for it before reading its results
+  e = launch(true, k_hint_match, dim3(grid), dim3(kHintThreads), 0, st, bank, N, eos, prefix, prefix_len,
+             prefix_len_dev, vec, mlen, cmax, smax, best);
   if (e != cudaSuccess) return e;
-  k_hint_pack<<<1, kHintThreads, 0, st>>>(bank, N, eos, prefix, prefix_len, mlen, cmax, smax, best, native,
-                                          native_len, n_native, native_stride, max_lanes, depth, max_nodes,
-                                          prefix_len_dev, pad_to, out_tok, out_par, out_T, out_info);
-  return cudaGetLastError();
+  return launch(true, k_hint_pack, dim3(1), dim3(kHintThreads), 0, st, bank, N, eos, prefix, prefix_len,
+                (const uint8_t*)mlen, (const uint8_t*)cmax, (const int*)smax, (const int*)best, native, native_len,
+                n_native, native_stride, max_lanes, depth, max_nodes, prefix_len_dev, pad_to, out_tok, out_par, out_T,
+                out_info);
 }
 
 }  // namespace oos
