@@ -121,7 +121,7 @@ WORKLOADS = {
                            tree=dict(kind="branch", bmin=1, bmax=4, max_depth=8)),
     "qwen3-8b": Workload(QWEN3_8B, ctx_len=2048, T=64, plant=10,
                          tree=dict(kind="branch", bmin=1, bmax=4, max_depth=12)),
-    "llama3.1-8b": Workload(LLAMA31_8B, ctx_len=8192, T=128, plant=4,
+    "llama3.1-8b": Workload(LLAMA31_8B, ctx_len=8192, T=128, plant=12,
                             tree=dict(kind="wide", level_branch=8, max_depth=16)),
     "qwen2.5-32b": Workload(QWEN25_32B, ctx_len=4096, T=64, plant=10,
                             tree=dict(kind="branch", bmin=1, bmax=4, max_depth=12)),
